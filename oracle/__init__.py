@@ -1,0 +1,173 @@
+"""CPU oracle of the OutlierTune per-channel quantized linear (arXiv 2406.18832).
+
+TEST INFRASTRUCTURE ONLY: imported by the tests, by ``__graft_entry__.smoke()``
+and by the ``cpu_baseline`` leg of ``bench.py``; never by the product package.
+It shares no code with the CUDA library.  The arithmetic lives in plain C
+(``ot_oracle.c``, compiled here with gcc, no FMA contraction, no fast-math);
+this module only builds it and marshals numpy arrays.
+
+Functions follow the paper's steps in order:
+  calibrate  - per-channel min/max (Appendix A; Section 3.2)
+  params     - z = (max+min)/2 and the static scale s (Section 3.2; Eq. 1)
+  fold       - W_s = W (.) s (Eq. 5), per-output-channel codes (Eq. 6),
+               b' = b + z W^T (Eq. 7)
+  quantize   - round((X - z) / s) (Eq. 6, Eq. 7)
+  matmul     - sum_k q[m,k] qw[n,k] in int64 (Eq. 6)
+  epilogue   - acc * sw + b' rounded to fp16 (Eq. 6, Eq. 7)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ot_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libot_oracle.so")
+_CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile ot_oracle.c into oracle/_build/libot_oracle.so (gcc)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.run(["gcc", *_CFLAGS, _SRC, "-o", tmp, "-lm"], check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            I64 = ctypes.c_int64
+            I = ctypes.c_int
+            lib.ot_half_to_float.argtypes = [ctypes.c_uint16]
+            lib.ot_half_to_float.restype = ctypes.c_float
+            lib.ot_double_to_half.argtypes = [ctypes.c_double]
+            lib.ot_double_to_half.restype = ctypes.c_uint16
+            lib.oracle_calibrate.argtypes = [P, I64, I64, I64, P, P, I]
+            lib.oracle_params.argtypes = [P, P, I64, I, I, P, P, P]
+            lib.oracle_fold.argtypes = [P, P, I64, I64, P, P, I, P, P, P]
+            lib.oracle_quantize.argtypes = [P, I64, I64, I64, P, P, I, P]
+            lib.oracle_matmul.argtypes = [P, P, I64, I64, I64, P]
+            lib.oracle_epilogue.argtypes = [P, I64, I64, P, P, I, P]
+            for f in ("oracle_calibrate", "oracle_params", "oracle_fold", "oracle_quantize",
+                      "oracle_matmul", "oracle_epilogue"):
+                getattr(lib, f).restype = None
+            _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _f16(a) -> np.ndarray:
+    a = np.ascontiguousarray(a)
+    if a.dtype != np.float16:
+        raise TypeError(f"expected float16, got {a.dtype}")
+    return a
+
+
+def _f32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.float32)
+
+
+def qmax(bits: int) -> int:
+    return (1 << (bits - 1)) - 1
+
+
+def half_to_float(bits: np.ndarray) -> np.ndarray:
+    """Binary16 bit patterns -> float32, element by element through the C oracle."""
+    lib = _load()
+    flat = np.ascontiguousarray(bits, dtype=np.uint16).ravel()
+    return np.array([lib.ot_half_to_float(int(b)) for b in flat], dtype=np.float32).reshape(np.shape(bits))
+
+
+def double_to_half(values: np.ndarray) -> np.ndarray:
+    """float64 -> binary16 bit patterns (round half to even), through the C oracle."""
+    lib = _load()
+    flat = np.ascontiguousarray(values, dtype=np.float64).ravel()
+    return np.array([lib.ot_double_to_half(float(v)) for v in flat], dtype=np.uint16).reshape(np.shape(values))
+
+
+def calibrate(x: np.ndarray, mn: np.ndarray | None = None, mx: np.ndarray | None = None):
+    """Per-channel (min, max) of fp16 X_cal[T, K]; pass mn/mx to continue a running calibration."""
+    x = _f16(x)
+    T, K = x.shape
+    reset = mn is None
+    mn = np.empty(K, np.float32) if reset else _f32(mn).copy()
+    mx = np.empty(K, np.float32) if reset else _f32(mx).copy()
+    _load().oracle_calibrate(_ptr(x), T, K, K, _ptr(mn), _ptr(mx), 1 if reset else 0)
+    return mn, mx
+
+
+def params(mn: np.ndarray, mx: np.ndarray, bits: int, symmetrize: bool = True):
+    """(z, s, r) per channel: symmetrization factor, scale, reciprocal scale."""
+    mn, mx = _f32(mn), _f32(mx)
+    K = mn.shape[0]
+    z, s, r = (np.empty(K, np.float32) for _ in range(3))
+    _load().oracle_params(_ptr(mn), _ptr(mx), K, bits, 1 if symmetrize else 0, _ptr(z), _ptr(s), _ptr(r))
+    return z, s, r
+
+
+def fold(w: np.ndarray, b: np.ndarray | None, z: np.ndarray, s: np.ndarray, bits_w: int):
+    """(qw int8 [N,K], sw fp32 [N], b' fp32 [N]) from fp16 W[N,K], fp16 b[N] (or None)."""
+    w = _f16(w)
+    N, K = w.shape
+    z, s = _f32(z), _f32(s)
+    bb = None if b is None else _f16(b)
+    qw = np.empty((N, K), np.int8)
+    sw = np.empty(N, np.float32)
+    bf = np.empty(N, np.float32)
+    _load().oracle_fold(_ptr(w), None if bb is None else _ptr(bb), N, K, _ptr(z), _ptr(s), bits_w,
+                        _ptr(qw), _ptr(sw), _ptr(bf))
+    return qw, sw, bf
+
+
+def quantize(x: np.ndarray, z: np.ndarray, r: np.ndarray, bits_a: int) -> np.ndarray:
+    """int8 codes [M, K] of fp16 X[M, K]."""
+    x = _f16(x)
+    M, K = x.shape
+    q = np.empty((M, K), np.int8)
+    _load().oracle_quantize(_ptr(x), M, K, K, _ptr(_f32(z)), _ptr(_f32(r)), bits_a, _ptr(q))
+    return q
+
+
+def matmul(q: np.ndarray, qw: np.ndarray) -> np.ndarray:
+    """int64 acc[M, N] = q[M, K] . qw[N, K]^T."""
+    q = np.ascontiguousarray(q, dtype=np.int8)
+    qw = np.ascontiguousarray(qw, dtype=np.int8)
+    M, K = q.shape
+    N = qw.shape[0]
+    assert qw.shape[1] == K
+    acc = np.empty((M, N), np.int64)
+    _load().oracle_matmul(_ptr(q), _ptr(qw), M, N, K, _ptr(acc))
+    return acc
+
+
+def epilogue(acc: np.ndarray, sw: np.ndarray, bfold: np.ndarray, relu: bool = False) -> np.ndarray:
+    """fp16 Y[M, N] = fp16(acc * sw + b'), optional ReLU."""
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
+    M, N = acc.shape
+    y = np.empty((M, N), np.uint16)
+    _load().oracle_epilogue(_ptr(acc), M, N, _ptr(_f32(sw)), _ptr(_f32(bfold)), 1 if relu else 0, _ptr(y))
+    return y.view(np.float16)
+
+
+def linear(x: np.ndarray, qw: np.ndarray, sw: np.ndarray, bfold: np.ndarray, z: np.ndarray,
+           r: np.ndarray, bits_a: int, relu: bool = False):
+    """Online path for one layer: codes, int64 accumulators and fp16 output."""
+    q = quantize(x, z, r, bits_a)
+    acc = matmul(q, qw)
+    return q, acc, epilogue(acc, sw, bfold, relu)

@@ -1,0 +1,253 @@
+/*
+ * ot_oracle.c -- plain CPU oracle of the OutlierTune per-channel quantized
+ * linear layer (arXiv 2406.18832).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may call this file:
+ * it is used by the tests, by __graft_entry__.smoke() and by the cpu_baseline
+ * leg of bench.py.  It shares no code, header, table or constant with the CUDA
+ * library; its only inputs are the raw arrays the tests generate.
+ *
+ * The method is an approximation (a quantizer), so this file takes the
+ * algorithm's steps in the paper's order and notation, written plainly:
+ *
+ *   1. calibration: per-channel min / max over calibration tokens
+ *      (Appendix A "min-max calibration"; Section 3.2 uses max/min per channel)
+ *   2. symmetrization factor z_k = (max X[:,k] + min X[:,k]) / 2 and the static
+ *      per-channel scale s_k of the symmetrized range (Section 3.2, Eq. 1 with
+ *      z = 0, i.e. symmetric)
+ *   3. pre-execution of dequantization: W_s = W (.) s^X (Eq. 5), per-output-
+ *      channel quantization of W_s (Eq. 6 right-hand side) and the bias fold
+ *      b' = b + z W^T (Eq. 7)
+ *   4. per-channel activation quantization round(X_hat / s^X) (Eq. 6 / Eq. 7)
+ *   5. the integer matrix product sum_k X~_ik (W~_s)_kj (Eq. 6)
+ *   6. external scaling by s^{W_s}_j and the folded bias (Eq. 6, Eq. 7)
+ *
+ * Readings where the paper is silent (each is stated where it is used):
+ *   R1 rounding  round() is round-half-to-even, evaluated in fp32.
+ *   R2 division  X_hat / s is evaluated as X_hat * r with r = qmax / amp
+ *                computed once per channel (fp32), likewise for the weights.
+ *   R3 range     symmetric codes are restricted to [-qmax, qmax],
+ *                qmax = 2^(bits-1) - 1; out-of-range values saturate.
+ *   R4 scale     amp_k = max(max_k - z_k, z_k - min_k), s_k = amp_k / qmax.
+ *   R5 degenerate a channel with amp = 0 (or no finite data) gets s = r = 0
+ *                (codes 0); a weight row with amax = 0 gets sw = 0, codes 0.
+ *   R6 non-finite NaN codes to 0; +-inf saturates to +-qmax.  Calibration
+ *                ignores NaN.
+ *   R7 bias      b' is formed in fp64 (k ascending) and rounded once to fp32.
+ *   R8 epilogue  y = acc * sw + b' evaluated in fp64, rounded once to fp16
+ *                (round-half-to-even, overflow to +-inf); optional ReLU.
+ *
+ * Floating point: compile with -ffp-contract=off and no fast-math, so every
+ * fp32 expression below rounds once per operation as written.
+ */
+#include <stdint.h>
+#include <stddef.h>
+#include <math.h>
+#include <string.h>
+
+/* ---------------------------------------------------------------------------
+ * IEEE 754 binary16 <-> binary32 / binary64, written from the format
+ * definition: 1 sign bit, 5 exponent bits (bias 15), 10 fraction bits.
+ * ------------------------------------------------------------------------- */
+float ot_half_to_float(uint16_t h)
+{
+    int sign = (h >> 15) & 1;
+    int e = (h >> 10) & 0x1f;
+    int f = h & 0x3ff;
+    double v;
+    if (e == 0x1f)
+        v = f ? NAN : INFINITY;
+    else if (e == 0)
+        v = ldexp((double)f, -24);             /* subnormal: f * 2^-14 * 2^-10 */
+    else
+        v = ldexp((double)(f + 1024), e - 25); /* (1 + f/1024) * 2^(e-15) */
+    return (float)(sign ? -v : v);             /* exact: 11 bits fit in fp32 */
+}
+
+/* Round-half-to-even of a finite double to binary16; overflow gives +-inf. */
+uint16_t ot_double_to_half(double v)
+{
+    uint16_t sign = signbit(v) ? 0x8000 : 0;
+    double a = fabs(v);
+    if (isnan(v)) return 0x7e00;
+    if (isinf(v)) return sign | 0x7c00;
+    /* binary16 numbers are n * 2^q with integer n < 2048; q = -24 for the
+       subnormal / smallest normal binade, q = e - 10 for the binade [2^e, 2^(e+1)). */
+    int e;
+    frexp(a, &e);            /* a = m * 2^e, m in [0.5, 1): a in [2^(e-1), 2^e) */
+    int q = (e - 1) - 10;
+    if (q < -24) q = -24;
+    double n = ldexp(a, -q); /* exact: scaling by a power of two */
+    double n_int = nearbyint(n); /* default rounding mode: half to even */
+    if (n_int >= 2048.0) {   /* rounded up into the next binade */
+        n_int /= 2.0;
+        q += 1;
+    }
+    if (q > 15 - 10 || (q == 5 && n_int >= 2048.0)) return sign | 0x7c00;
+    uint16_t bits;
+    if (n_int < 1024.0) {    /* subnormal (q == -24) */
+        bits = (uint16_t)n_int;
+    } else {
+        int exp_field = q + 10 + 15; /* n in [1024, 2048): value = (n/1024) * 2^(q+10) */
+        bits = (uint16_t)((exp_field << 10) | ((int)n_int - 1024));
+    }
+    return sign | bits;
+}
+
+static int qmax_of(int bits) { return (1 << (bits - 1)) - 1; }
+
+/* Round half to even in fp32, then saturate to [-qmax, qmax] (R1, R3, R6). */
+static int quantize_code(float u, int qmax)
+{
+    if (isnan(u)) return 0;
+    if (u >= (float)qmax) return qmax;
+    if (u <= -(float)qmax) return -qmax;
+    return (int)nearbyintf(u);
+}
+
+/* ---------------------------------------------------------------------------
+ * Step 1: calibration (Appendix A, Section 3.2).  Running per-channel min and
+ * max of X_cal[T, K] (fp16, row stride ldx elements).  reset = 1 starts from
+ * (+inf, -inf); reset = 0 continues from the values already in mn / mx, so a
+ * calibration set can be fed batch by batch.
+ * ------------------------------------------------------------------------- */
+void oracle_calibrate(const uint16_t *x, int64_t T, int64_t K, int64_t ldx,
+                      float *mn, float *mx, int reset)
+{
+    if (reset)
+        for (int64_t k = 0; k < K; ++k) { mn[k] = INFINITY; mx[k] = -INFINITY; }
+    for (int64_t t = 0; t < T; ++t)
+        for (int64_t k = 0; k < K; ++k) {
+            float v = ot_half_to_float(x[t * ldx + k]);
+            if (isnan(v)) continue;          /* R6 */
+            if (v < mn[k]) mn[k] = v;
+            if (v > mx[k]) mx[k] = v;
+        }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step 2: symmetrization factor and static scale (Section 3.2; Eq. 1, z = 0).
+ *   z_k   = (max_k + min_k) / 2
+ *   amp_k = max(max_k - z_k, z_k - min_k)                              (R4)
+ *   s_k   = amp_k / qmax,   r_k = qmax / amp_k                         (R2)
+ * With symmetrize = 0 (the "Non-Sym" ablation of Table 6) z_k = 0 and
+ * amp_k = max(|max_k|, |min_k|).
+ * ------------------------------------------------------------------------- */
+void oracle_params(const float *mn, const float *mx, int64_t K, int bits,
+                   int symmetrize, float *z, float *s, float *r)
+{
+    const float qmax = (float)qmax_of(bits);
+    for (int64_t k = 0; k < K; ++k) {
+        float lo = mn[k], hi = mx[k];
+        float zk, amp;
+        if (!(lo <= hi) || isinf(lo) || isinf(hi)) {    /* no finite data (R5) */
+            z[k] = 0.0f; s[k] = 0.0f; r[k] = 0.0f;
+            continue;
+        }
+        if (symmetrize) {
+            zk = (hi + lo) * 0.5f;
+            float up = hi - zk, down = zk - lo;
+            amp = up > down ? up : down;
+        } else {
+            zk = 0.0f;
+            float a = fabsf(hi), b = fabsf(lo);
+            amp = a > b ? a : b;
+        }
+        z[k] = zk;
+        if (amp > 0.0f && isfinite(amp)) {
+            s[k] = amp / qmax;
+            r[k] = qmax / amp;
+        } else {
+            s[k] = 0.0f; r[k] = 0.0f;
+        }
+    }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step 3: pre-execution of dequantization and bias correction.
+ *   W_s[n,k] = W[n,k] * s_k                         (Eq. 5, W is [N, K])
+ *   amax_n   = max_k |W_s[n,k]|
+ *   sw_n     = amax_n / qmax_w,  rw_n = qmax_w / amax_n              (R2, R5)
+ *   qw[n,k]  = round(W_s[n,k] * rw_n) in [-qmax_w, qmax_w]   (Eq. 6 right side)
+ *   b'_n     = b_n + sum_k z_k W[n,k]                      (Eq. 7, R7)
+ * b may be NULL (no bias).
+ * ------------------------------------------------------------------------- */
+void oracle_fold(const uint16_t *w, const uint16_t *b, int64_t N, int64_t K,
+                 const float *z, const float *s, int bits_w,
+                 int8_t *qw, float *sw, float *bfold)
+{
+    const int qmax = qmax_of(bits_w);
+    for (int64_t n = 0; n < N; ++n) {
+        const uint16_t *wrow = w + n * K;
+        float amax = 0.0f;
+        for (int64_t k = 0; k < K; ++k) {
+            float ws = ot_half_to_float(wrow[k]) * s[k];
+            float a = fabsf(ws);
+            if (a > amax) amax = a;
+        }
+        float swn = 0.0f, rwn = 0.0f;
+        if (amax > 0.0f && isfinite(amax)) {
+            swn = amax / (float)qmax;
+            rwn = (float)qmax / amax;
+        }
+        sw[n] = swn;
+        for (int64_t k = 0; k < K; ++k) {
+            float ws = ot_half_to_float(wrow[k]) * s[k];
+            qw[n * K + k] = (int8_t)quantize_code(ws * rwn, qmax);
+        }
+        double acc = b ? (double)ot_half_to_float(b[n]) : 0.0;
+        for (int64_t k = 0; k < K; ++k)
+            acc += (double)z[k] * (double)ot_half_to_float(wrow[k]);
+        bfold[n] = (float)acc;
+    }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step 4: per-channel static activation quantization, round(X_hat / s^X) with
+ * X_hat = X - z (Eq. 6, Eq. 7; R1-R3, R6):
+ *   t = x - z_k (fp32),  u = t * r_k (fp32),  q = round_half_even(u) saturated.
+ * X is [M, K] fp16 with row stride ldx; q is [M, K] int8, dense.
+ * ------------------------------------------------------------------------- */
+void oracle_quantize(const uint16_t *x, int64_t M, int64_t K, int64_t ldx,
+                     const float *z, const float *r, int bits_a, int8_t *q)
+{
+    const int qmax = qmax_of(bits_a);
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t k = 0; k < K; ++k) {
+            float t = ot_half_to_float(x[m * ldx + k]) - z[k];
+            float u = t * r[k];
+            q[m * K + k] = (int8_t)quantize_code(u, qmax);
+        }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step 5: the integer product of Eq. 6, acc[m,n] = sum_k q[m,k] * qw[n,k],
+ * in int64 (the caller checks that it fits the int32 accumulator).
+ * ------------------------------------------------------------------------- */
+void oracle_matmul(const int8_t *q, const int8_t *qw, int64_t M, int64_t N,
+                   int64_t K, int64_t *acc)
+{
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t n = 0; n < N; ++n) {
+            int64_t sum = 0;
+            for (int64_t k = 0; k < K; ++k)
+                sum += (int64_t)q[m * K + k] * (int64_t)qw[n * K + k];
+            acc[m * N + n] = sum;
+        }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step 6: external scaling (Eq. 6) plus the folded bias (Eq. 7), R8:
+ *   y[m,n] = fp16( acc[m,n] * sw_n + b'_n ),  ReLU applied before rounding
+ * when relu != 0.  y holds binary16 bit patterns.
+ * ------------------------------------------------------------------------- */
+void oracle_epilogue(const int64_t *acc, int64_t M, int64_t N, const float *sw,
+                     const float *bfold, int relu, uint16_t *y)
+{
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t n = 0; n < N; ++n) {
+            double v = (double)acc[m * N + n] * (double)sw[n] + (double)bfold[n];
+            if (relu && !(v > 0.0)) v = 0.0;
+            y[m * N + n] = ot_double_to_half(v);
+        }
+}
