@@ -1,0 +1,165 @@
+/*
+ * outliertune.h -- C ABI of the GB300 (sm_103a) per-channel quantized linear
+ * layer of OutlierTune (arXiv 2406.18832).
+ *
+ * The method: activations X are symmetrized per input channel (X_hat = X - z,
+ * Section 3.2) and quantized per channel with static scales s (Eq. 6); the
+ * weights absorb the activation scales before they are quantized per output
+ * channel ("pre-execution of dequantization", Eq. 5, Eq. 6); the integer
+ * product is rescaled per output channel only and the symmetrization shift
+ * comes back through the bias b' = b + z W^T (Eq. 7).
+ *
+ * Conventions shared by every entry point
+ *   - Every pointer is DEVICE memory owned by the caller, unless stated.  The
+ *     library allocates no device memory and keeps no per-call state.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Work is enqueued asynchronously; outputs are valid once the
+ *     stream has reached that point.  Nothing here synchronizes the stream
+ *     except ot_get_device_status.
+ *   - Layouts are row-major.  X is [tokens, K] with row stride ldx elements,
+ *     W is [N, K] (out x in, the nn.Linear layout that Eq. 6's W^T implies),
+ *     Y is [M, N] with row stride ldy elements.
+ *   - bits (bits_a for activations, bits_w for weights) is in [2, 8];
+ *     qmax = 2^(bits-1) - 1 and codes lie in [-qmax, qmax] (127 for Int8,
+ *     31 for Int6).  Rounding is round-half-to-even in fp32.
+ *   - Argument errors are detected on the host before anything is launched
+ *     and return OT_ERR_INVALID_ARG or OT_ERR_UNSUPPORTED; a failed launch
+ *     returns OT_ERR_CUDA.  No exception crosses the ABI.  Device-side waits
+ *     are bounded: a wait that gives up records OT_ERR_TIMEOUT in a device
+ *     status word that ot_get_device_status reads.
+ */
+#ifndef OUTLIERTUNE_H
+#define OUTLIERTUNE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    OT_OK = 0,
+    OT_ERR_INVALID_ARG = 1,  /* null pointer, bad size, alignment or bits */
+    OT_ERR_UNSUPPORTED = 2,  /* valid request this build does not run (e.g. K too large) */
+    OT_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed */
+    OT_ERR_TIMEOUT = 4       /* a bounded device-side wait gave up */
+} ot_status;
+
+/* Storage format of activation codes written by ot_quantize_act. */
+typedef enum {
+    OT_CODE_I8 = 0,   /* int8 codes, 1 byte per element */
+    OT_CODE_F16 = 1   /* the same integers stored exactly as fp16 (the operand
+                         format ot_linear reads: sm_103a has no integer tcgen05
+                         MMA, so the product runs on the fp16 tensor path) */
+} ot_code_format;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *ot_status_string(ot_status st);
+
+/* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
+int ot_version(void);
+
+/*
+ * ot_calibrate -- per-channel running min / max of calibration activations
+ * (Appendix A "min-max calibration"; the max and min of Section 3.2).
+ *   x_f16   fp16 [T, K], row stride ldx elements (ldx >= K); 16-byte aligned,
+ *           K and ldx multiples of 8.
+ *   ch_min, ch_max  fp32 [K], in/out.  reset != 0 first sets them to
+ *           (+inf, -inf); reset == 0 folds this batch into their current
+ *           values, so a calibration set can be streamed batch by batch.
+ *   NaN inputs are ignored.  T == 0 only applies the reset.
+ */
+ot_status ot_calibrate(const void *x_f16, int64_t T, int64_t K, int64_t ldx,
+                       float *ch_min, float *ch_max, int reset, void *stream);
+
+/*
+ * ot_derive_params -- symmetrization factor and static scale per channel
+ * (Section 3.2; Eq. 1 with zero point 0):
+ *   z = (max + min) / 2, amp = max(max - z, z - min),
+ *   s = amp / qmax, r = qmax / amp            (fp32, IEEE division)
+ * symmetrize == 0 gives the Table 6 "Non-Sym" variant: z = 0,
+ * amp = max(|max|, |min|).  A channel with amp == 0, or without finite
+ * calibration data, gets s = r = 0 (its codes are 0; a constant channel is
+ * then carried exactly by z through the folded bias).
+ *   ch_min, ch_max  fp32 [K] in;  z, s, r  fp32 [K] out.
+ */
+ot_status ot_derive_params(const float *ch_min, const float *ch_max, int64_t K,
+                           int bits_a, int symmetrize, float *z, float *s,
+                           float *r, void *stream);
+
+/*
+ * ot_fold_weights -- pre-execution of dequantization and bias correction,
+ * done once per layer (Eq. 5, Eq. 6 right-hand side, Eq. 7; Section 3.2
+ * "predetermined offline"):
+ *   W_s[n,k] = W[n,k] * s_k                              (fp32)
+ *   sw_n = max_k |W_s[n,k]| / qmax_w,  rw_n = qmax_w / max_k |W_s[n,k]|
+ *   qw[n,k] = round(W_s[n,k] * rw_n)  in [-qmax_w, qmax_w]
+ *   b'_n = b_n + sum_k z_k W[n,k]       (fp64, k ascending, rounded to fp32)
+ * The parameters z, s, r come from (ch_min, ch_max) as in ot_derive_params
+ * and are written out as well.
+ *   ch_min, ch_max fp32 [K] in; w_f16 fp16 [N, K] (16-byte aligned, K % 16 == 0);
+ *   b_f16 fp16 [N] or NULL (no bias);  z, s, r fp32 [K] out;
+ *   qw int8 [N, K] out (16-byte aligned);  sw fp32 [N] out;  b_fold fp32 [N] out.
+ */
+ot_status ot_fold_weights(const float *ch_min, const float *ch_max, int bits_a,
+                          int symmetrize, const void *w_f16, const void *b_f16,
+                          int64_t N, int64_t K, int bits_w, float *z, float *s,
+                          float *r, int8_t *qw, float *sw, float *b_fold,
+                          void *stream);
+
+/*
+ * ot_quantize_act -- symmetrize and quantize activations per channel with
+ * the static parameters (round(X_hat / s) of Eq. 6 / Eq. 7):
+ *   q[m,k] = clamp(round_half_even((x[m,k] - z_k) * r_k), -qmax_a, qmax_a)
+ * evaluated in fp32 (subtract, multiply, round: two roundings as written).
+ * NaN gives code 0, +-inf and out-of-range values saturate.
+ *   x_f16   fp16 [M, K], row stride ldx (16-byte aligned; K, ldx % 8 == 0)
+ *   z, r    fp32 [K]
+ *   q       [M, K] dense, int8 (OT_CODE_I8) or fp16 (OT_CODE_F16); 16-byte aligned
+ */
+ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
+                          const float *z, const float *r, int bits_a, void *q,
+                          int q_format, void *stream);
+
+/*
+ * ot_linear -- the quantized linear with external per-output-channel scaling
+ * (Eq. 6) and the folded bias (Eq. 7):
+ *   acc[m,n] = sum_k q[m,k] * qw[n,k]            exact integer
+ *   y[m,n]   = fp16( fma((float)acc[m,n], sw_n, b'_n) ), then ReLU if relu != 0
+ *   q_f16   activation codes as fp16 integers [M, K] (OT_CODE_F16 output of
+ *           ot_quantize_act), |q| <= qmax(bits_a); 16-byte aligned, K % 16 == 0
+ *   qw      int8 [N, K] from ot_fold_weights, |qw| <= qmax(bits_w); 16-byte aligned
+ *   sw, b_fold  fp32 [N]
+ *   y_f16   fp16 [M, N], row stride ldy >= N
+ * Exactness: the tensor cores accumulate in fp32, which holds integers
+ * exactly up to 2^24; the kernel therefore sums K in chunks short enough
+ * that no partial sum can pass 2^24 for the promised bits, and adds the
+ * chunks in int32.  Codes outside [-qmax, qmax] void that guarantee.
+ * K * qmax_a * qmax_w must be < 2^31 (K <= 133144 for W8A8).
+ */
+ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
+                    const float *sw, const float *b_fold, int64_t N, int bits_a,
+                    int bits_w, void *y_f16, int64_t ldy, int relu, void *stream);
+
+/*
+ * ot_linear_s32 -- the same integer product as ot_linear, written out as the
+ * int32 accumulators acc[m,n] (dense [M, N]) instead of the scaled fp16
+ * output; the accumulators of Eq. 6 before external scaling, for checking.
+ */
+ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
+                        int64_t N, int bits_a, int bits_w, int32_t *acc,
+                        void *stream);
+
+/*
+ * ot_get_device_status -- synchronize `stream`, then return and clear the
+ * device status word of the current device: OT_ERR_TIMEOUT if a bounded
+ * device wait gave up since the last call, else OT_OK (or OT_ERR_CUDA if the
+ * synchronization itself failed).
+ */
+ot_status ot_get_device_status(void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OUTLIERTUNE_H */

@@ -1,0 +1,175 @@
+"""Thin Python binding of the C ABI in include/outliertune.h.
+
+Argument marshalling only: every function takes CUDA torch tensors, checks
+that they live on the GPU with the dtype and layout the C function expects,
+and passes raw pointers, sizes and the current CUDA stream.  All arithmetic
+runs in the CUDA library; there is no CPU fallback: if the library is not
+built, or a tensor is not on a CUDA device, the call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+OT_OK, OT_ERR_INVALID_ARG, OT_ERR_UNSUPPORTED, OT_ERR_CUDA, OT_ERR_TIMEOUT = range(5)
+OT_CODE_I8, OT_CODE_F16 = 0, 1
+
+_lock = threading.Lock()
+_handle = None
+
+_P, _I64, _I, _F = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float
+_SIGNATURES = {
+    "ot_status_string": ([_I], ctypes.c_char_p),
+    "ot_version": ([], _I),
+    "ot_calibrate": ([_P, _I64, _I64, _I64, _P, _P, _I, _P], _I),
+    "ot_derive_params": ([_P, _P, _I64, _I, _I, _P, _P, _P, _P], _I),
+    "ot_fold_weights": ([_P, _P, _I, _I, _P, _P, _I64, _I64, _I, _P, _P, _P, _P, _P, _P, _P], _I),
+    "ot_quantize_act": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _I, _P], _I),
+    "ot_linear": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P], _I),
+    "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P], _I),
+    "ot_get_device_status": ([_P], _I),
+}
+
+
+class OTError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)}")
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def load() -> ctypes.CDLL:
+    """Load lib/libot_gb300.so (built by paper_2406_18832_gb300.build)."""
+    global _handle
+    with _lock:
+        if _handle is None:
+            path = _build.LIB_PATH
+            if not os.path.exists(path):
+                raise RuntimeError(f"CUDA library not built: {path} is missing "
+                                   "(run __graft_entry__.build() or python -m paper_2406_18832_gb300.build)")
+            lib = ctypes.CDLL(path)
+            for name, (args, res) in _SIGNATURES.items():
+                fn = getattr(lib, name)
+                fn.argtypes = args
+                fn.restype = res
+            _handle = lib
+    return _handle
+
+
+def status_string(status: int) -> str:
+    return load().ot_status_string(int(status)).decode()
+
+
+def version() -> int:
+    return load().ot_version()
+
+
+def _check(status: int, where: str):
+    if status != OT_OK:
+        raise OTError(status, where)
+
+
+def _dev(t: torch.Tensor, name: str, dtype=None) -> int:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor (the library takes device pointers)")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    return t.data_ptr()
+
+
+def _dense(t: torch.Tensor, name: str):
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _rows(t: torch.Tensor, name: str):
+    """(rows, cols, row stride) of a 2-D tensor with unit column stride."""
+    if t.dim() != 2 or (t.shape[1] > 1 and t.stride(1) != 1):
+        raise ValueError(f"{name} must be 2-D with unit stride along its last dimension")
+    return t.shape[0], t.shape[1], t.stride(0) if t.shape[0] > 1 else t.shape[1]
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def ot_calibrate(x: torch.Tensor, ch_min: torch.Tensor, ch_max: torch.Tensor, reset: bool = True, stream=None):
+    """Per-channel running min / max of fp16 X[T, K] into fp32 ch_min, ch_max [K]."""
+    T, K, ldx = _rows(x, "x")
+    px = _dev(x, "x", torch.float16)
+    _check(load().ot_calibrate(px, T, K, ldx, _dev(ch_min, "ch_min", torch.float32),
+                               _dev(ch_max, "ch_max", torch.float32), 1 if reset else 0, _stream(stream)),
+           "ot_calibrate")
+
+
+def ot_derive_params(ch_min, ch_max, bits_a: int, z, s, r, symmetrize: bool = True, stream=None):
+    K = ch_min.numel()
+    _check(load().ot_derive_params(_dev(ch_min, "ch_min", torch.float32), _dev(ch_max, "ch_max", torch.float32), K,
+                                   bits_a, 1 if symmetrize else 0, _dev(z, "z", torch.float32),
+                                   _dev(s, "s", torch.float32), _dev(r, "r", torch.float32), _stream(stream)),
+           "ot_derive_params")
+
+
+def ot_fold_weights(ch_min, ch_max, bits_a: int, w, b, bits_w: int, z, s, r, qw, sw, b_fold,
+                    symmetrize: bool = True, stream=None):
+    _dense(w, "w")
+    N, K = w.shape
+    pb = None if b is None else _dev(b, "b", torch.float16)
+    _check(load().ot_fold_weights(_dev(ch_min, "ch_min", torch.float32), _dev(ch_max, "ch_max", torch.float32),
+                                  bits_a, 1 if symmetrize else 0, _dev(w, "w", torch.float16), pb, N, K, bits_w,
+                                  _dev(z, "z", torch.float32), _dev(s, "s", torch.float32),
+                                  _dev(r, "r", torch.float32), _dev(qw, "qw", torch.int8),
+                                  _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32),
+                                  _stream(stream)),
+           "ot_fold_weights")
+
+
+def ot_quantize_act(x, z, r, bits_a: int, q, q_format: int = OT_CODE_F16, stream=None):
+    M, K, ldx = _rows(x, "x")
+    _dense(q, "q")
+    want = torch.float16 if q_format == OT_CODE_F16 else torch.int8
+    _check(load().ot_quantize_act(_dev(x, "x", torch.float16), M, K, ldx, _dev(z, "z", torch.float32),
+                                  _dev(r, "r", torch.float32), bits_a, _dev(q, "q", want), q_format,
+                                  _stream(stream)),
+           "ot_quantize_act")
+
+
+def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False, stream=None):
+    _dense(q, "q")
+    _dense(qw, "qw")
+    M, K = q.shape
+    N = qw.shape[0]
+    ym, yn, ldy = _rows(y, "y")
+    if ym != M or yn != N:
+        raise ValueError("y must be [M, N]")
+    _check(load().ot_linear(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8),
+                            _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32), N, bits_a,
+                            bits_w, _dev(y, "y", torch.float16), ldy, 1 if relu else 0, _stream(stream)),
+           "ot_linear")
+
+
+def ot_linear_s32(q, qw, bits_a: int, bits_w: int, acc, stream=None):
+    _dense(q, "q")
+    _dense(qw, "qw")
+    _dense(acc, "acc")
+    M, K = q.shape
+    N = qw.shape[0]
+    _check(load().ot_linear_s32(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8), N, bits_a,
+                                bits_w, _dev(acc, "acc", torch.int32), _stream(stream)),
+           "ot_linear_s32")
+
+
+def ot_get_device_status(stream=None) -> int:
+    return load().ot_get_device_status(_stream(stream))

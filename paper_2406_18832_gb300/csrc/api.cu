@@ -1,0 +1,129 @@
+// api.cu -- the C ABI (include/outliertune.h): argument validation on the
+// host, then one or two kernel launches on the caller's stream.  Nothing here
+// allocates device memory.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "outliertune.h"
+#include "ot_kernels.h"
+
+namespace ot {
+
+int num_sms() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
+    if (dev < 64 && cache[dev]) return cache[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    if (dev < 64) cache[dev] = n;
+    return n;
+}
+
+}  // namespace ot
+
+namespace {
+
+constexpr int kVersion = 100;  // 0.1.0
+
+inline bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+inline bool bits_ok(int b) { return b >= 2 && b <= 8; }
+inline int64_t qmax_of(int b) { return (int64_t(1) << (b - 1)) - 1; }
+inline ot_status from_cuda(cudaError_t e) { return e == cudaSuccess ? OT_OK : OT_ERR_CUDA; }
+inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+constexpr int64_t kIntMax = 2147483647;
+
+}  // namespace
+
+extern "C" {
+
+const char *ot_status_string(ot_status st) {
+    switch (st) {
+        case OT_OK: return "OT_OK";
+        case OT_ERR_INVALID_ARG: return "OT_ERR_INVALID_ARG: invalid argument (pointer, size, alignment or bits)";
+        case OT_ERR_UNSUPPORTED: return "OT_ERR_UNSUPPORTED: request outside what this build runs";
+        case OT_ERR_CUDA: return "OT_ERR_CUDA: a CUDA call or kernel launch failed";
+        case OT_ERR_TIMEOUT: return "OT_ERR_TIMEOUT: a bounded device wait gave up";
+    }
+    return "unknown ot_status";
+}
+
+int ot_version(void) { return kVersion; }
+
+ot_status ot_calibrate(const void *x_f16, int64_t T, int64_t K, int64_t ldx, float *ch_min, float *ch_max,
+                       int reset, void *stream) {
+    if (T < 0 || K <= 0 || K % 8 != 0 || ldx < K || ldx % 8 != 0) return OT_ERR_INVALID_ARG;
+    if (!ch_min || !ch_max || !aligned(ch_min, 4) || !aligned(ch_max, 4)) return OT_ERR_INVALID_ARG;
+    if (T > 0 && (!x_f16 || !aligned(x_f16, 16))) return OT_ERR_INVALID_ARG;
+    if (T > kIntMax * 64) return OT_ERR_UNSUPPORTED;
+    return from_cuda(ot::launch_calibrate(x_f16, T, K, ldx, ch_min, ch_max, reset, as_stream(stream)));
+}
+
+ot_status ot_derive_params(const float *ch_min, const float *ch_max, int64_t K, int bits_a, int symmetrize,
+                           float *z, float *s, float *r, void *stream) {
+    if (K <= 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;
+    if (!ch_min || !ch_max || !z || !s || !r) return OT_ERR_INVALID_ARG;
+    return from_cuda(ot::launch_params(ch_min, ch_max, K, bits_a, symmetrize, z, s, r, as_stream(stream)));
+}
+
+ot_status ot_fold_weights(const float *ch_min, const float *ch_max, int bits_a, int symmetrize, const void *w_f16,
+                          const void *b_f16, int64_t N, int64_t K, int bits_w, float *z, float *s, float *r,
+                          int8_t *qw, float *sw, float *b_fold, void *stream) {
+    if (N < 0 || K <= 0 || K % 16 != 0 || !bits_ok(bits_a) || !bits_ok(bits_w)) return OT_ERR_INVALID_ARG;
+    if (!ch_min || !ch_max || !z || !s || !r || !sw || !b_fold) return OT_ERR_INVALID_ARG;
+    if (N > 0 && (!w_f16 || !qw || !aligned(w_f16, 16) || !aligned(qw, 16))) return OT_ERR_INVALID_ARG;
+    if (b_f16 && !aligned(b_f16, 2)) return OT_ERR_INVALID_ARG;
+    cudaStream_t st = as_stream(stream);
+    cudaError_t e = ot::launch_params(ch_min, ch_max, K, bits_a, symmetrize, z, s, r, st);
+    if (e != cudaSuccess) return OT_ERR_CUDA;
+    return from_cuda(ot::launch_fold(w_f16, b_f16, N, K, z, s, bits_w, qw, sw, b_fold, st));
+}
+
+ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
+                          int bits_a, void *q, int q_format, void *stream) {
+    if (M < 0 || K <= 0 || K % 8 != 0 || ldx < K || ldx % 8 != 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;
+    if (q_format != OT_CODE_I8 && q_format != OT_CODE_F16) return OT_ERR_INVALID_ARG;
+    if (!z || !r || !aligned(z, 16) || !aligned(r, 16)) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!x_f16 || !q || !aligned(x_f16, 16) || !aligned(q, 16))) return OT_ERR_INVALID_ARG;
+    if ((M + 63) / 64 > 65535) return OT_ERR_UNSUPPORTED;
+    return from_cuda(ot::launch_quantize(x_f16, M, K, ldx, z, r, bits_a, q, q_format, as_stream(stream)));
+}
+
+static ot_status linear_common(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, int64_t N, int bits_a,
+                               int bits_w, const void *out) {
+    if (M < 0 || N <= 0 || K <= 0 || K % 16 != 0 || !bits_ok(bits_a) || !bits_ok(bits_w))
+        return OT_ERR_INVALID_ARG;
+    if (!qw || !aligned(qw, 16)) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!q_f16 || !aligned(q_f16, 16) || !out)) return OT_ERR_INVALID_ARG;
+    if (M > kIntMax || N > kIntMax || K > kIntMax) return OT_ERR_UNSUPPORTED;
+    if (K * qmax_of(bits_a) * qmax_of(bits_w) > kIntMax) return OT_ERR_UNSUPPORTED;  // int32 accumulator
+    return OT_OK;
+}
+
+ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw, const float *b_fold,
+                    int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy, int relu, void *stream) {
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
+    if (v != OT_OK) return v;
+    if (!sw || !b_fold || ldy < N || (y_f16 && !aligned(y_f16, 2))) return OT_ERR_INVALID_ARG;
+    if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
+    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false};
+    return from_cuda(ot::launch_linear(a, as_stream(stream)));
+}
+
+ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, int64_t N, int bits_a,
+                        int bits_w, int32_t *acc, void *stream) {
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, acc);
+    if (v != OT_OK) return v;
+    if (acc && !aligned(acc, 4)) return OT_ERR_INVALID_ARG;
+    ot::LinearArgs a{q_f16, qw, nullptr, nullptr, acc, M, N, K, N, bits_a, bits_w, 0, true};
+    return from_cuda(ot::launch_linear(a, as_stream(stream)));
+}
+
+ot_status ot_get_device_status(void *stream) {
+    int v = 0;
+    if (ot::read_clear_status(&v, as_stream(stream)) != cudaSuccess) return OT_ERR_CUDA;
+    return v == OT_ERR_TIMEOUT ? OT_ERR_TIMEOUT : OT_OK;
+}
+
+}  // extern "C"

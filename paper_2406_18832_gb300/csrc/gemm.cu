@@ -1,0 +1,389 @@
+// gemm.cu -- the quantized linear of Eq. 6 / Eq. 7 on sm_103a tensor cores:
+//   acc[m,n] = sum_k q[m,k] * qw[n,k]           (exact integers)
+//   y[m,n]   = fp16(fma((float)acc, sw_n, b'_n)) (+ ReLU)   or acc as int32
+//
+// sm_103a has no integer tcgen05.mma (kind::i8 is an sm_100a feature), so
+// the product runs on tcgen05.mma kind::f16: integer codes |c| <= 127 are
+// exact in fp16, every product is exact in fp32, and an fp32 sum of integers
+// is exact while it stays below 2^24.  K is therefore summed in chunks of
+// kcb k-blocks with kcb * 64 * qmax_a * qmax_w <= 2^24; each chunk's fp32
+// accumulator is converted to int32 (exact) and summed in registers.
+//
+// Design (one persistent CTA per SM, 16 warps):
+//   warp 0        TMA producer: per 64-wide k-block, the activation-code tile
+//                 (BN tokens x 64, fp16, 128-byte swizzle) and the weight tile
+//                 (128 rows x 64, int8, 64-byte swizzle) into a 6-stage ring.
+//   warp 1        MMA issuer (one thread): D[128 x BN] += A[128 x 16] * B,
+//                 A read from tensor memory, B from shared memory.
+//   warp 2        allocates / frees the 512 TMEM columns.
+//   warps 4-7     converters: each thread takes one weight row of the stage,
+//                 turns its 64 int8 codes into fp16 pairs in registers and
+//                 stores them into the TMEM A buffer of the stage
+//                 (tcgen05.st), so the int8 -> fp16 widening never costs
+//                 shared-memory bandwidth.
+//   warps 8-15    epilogue: drain each finished chunk accumulator (double
+//                 buffered in TMEM) into int32 totals, and at the end of the
+//                 tile apply sw_n, b'_n, ReLU and store.
+// The weight matrix is the MMA's M side (128 output channels = TMEM lanes),
+// tokens are its N side (BN = 16..128), i.e. the kernel computes Y^T tiles.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_fp16.h>
+
+#include <mutex>
+
+#include "ot_common.cuh"
+#include "ot_kernels.h"
+
+namespace ot {
+
+// Device status word of this library (OT_OK or OT_ERR_TIMEOUT), one per device.
+__device__ int g_status;
+
+namespace {
+
+constexpr int kBM = 128;        // weight rows per tile (TMEM lanes, MMA M)
+constexpr int kBK = 64;         // K elements per k-block (128 bytes of fp16)
+constexpr int kStages = 6;      // shared-memory ring and TMEM A buffers
+constexpr int kThreads = 512;   // 16 warps
+constexpr int kWarpTma = 0, kWarpMma = 1, kWarpAlloc = 2, kWarpConv0 = 4, kWarpEpi0 = 8;
+constexpr int kNumEpiWarps = 8;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kTmemAccCol = 256;   // A buffers at columns [0, 32*kStages), accumulators from 256
+static_assert(32 * kStages <= (int)kTmemAccCol, "TMEM A buffers overlap the accumulators");
+
+template <int BN>
+struct alignas(1024) Smem {
+    uint8_t b[kStages][BN * 128];   // activation codes, 128-byte swizzled rows
+    uint8_t w[kStages][kBM * kBK];  // int8 weight codes, 64-byte swizzled rows
+    uint64_t full[kStages];         // TMA landed (tx bytes)
+    uint64_t empty[kStages];        // stage free: MMA done with b[] + 4 converter warps done with w[]
+    uint64_t afull[kStages];        // TMEM A buffer written (4 converter warps)
+    uint64_t aempty[kStages];       // TMEM A buffer consumed (MMA commit)
+    uint64_t accfull[2];            // chunk accumulator complete (MMA commit)
+    uint64_t accempty[2];           // chunk accumulator drained (8 epilogue warps)
+    uint64_t drain;                 // teardown: all issued MMAs complete
+    uint32_t tmem_base;
+    int abort;
+};
+
+// Bounded wait that ignores the abort flag (used only while tearing down).
+__device__ __forceinline__ void wait_teardown(uint32_t bar, uint32_t parity) {
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+            atomicExch(&g_status, (int)OT_ERR_TIMEOUT);
+            return;
+        }
+    }
+}
+
+// 4 signed int8 codes -> two fp16x2 words (exact).  Each byte b is biased to
+// u = b + 128 and placed under the fp16 exponent of 1024 (bit pattern
+// 0x6400 | u = 1024 + u, unit spacing in [1024, 2048)); subtracting 1152
+// leaves b exactly.
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t u = w ^ 0x80808080u;
+    const uint32_t a = __byte_perm(u, 0x64646464u, 0x4140);
+    const uint32_t b = __byte_perm(u, 0x64646464u, 0x4342);
+    const __half2 bias = __half2half2(__ushort_as_half(0x6480));  // 1152
+    const __half2 ha = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
+    const __half2 hb = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
+    lo = *reinterpret_cast<const uint32_t *>(&ha);
+    hi = *reinterpret_cast<const uint32_t *>(&hb);
+}
+
+template <int BN, bool kS32>
+__global__ void __launch_bounds__(kThreads, 1)
+    linear_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
+                  const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
+                  int N, int K, int ldy, int kcb, int relu) {
+    extern __shared__ uint8_t smem_raw[];
+    Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = warp_id(), lane = lane_id();
+    const int m_tiles = (M + BN - 1) / BN;
+    const int n_tiles = (N + kBM - 1) / kBM;
+    const int num_tiles = m_tiles * n_tiles;
+    const int nkb = (K + kBK - 1) / kBK;
+    volatile int *abort = &S.abort;
+    constexpr uint32_t kTxBytes = BN * 128 + kBM * kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_u32(&S.full[s]), 1);
+            mbar_init(smem_u32(&S.empty[s]), 1 + 4);
+            mbar_init(smem_u32(&S.afull[s]), 4);
+            mbar_init(smem_u32(&S.aempty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&S.accfull[b]), 1);
+            mbar_init(smem_u32(&S.accempty[b]), kNumEpiWarps);
+        }
+        mbar_init(smem_u32(&S.drain), 1);
+        S.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == kWarpTma && lane == 0) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_w);
+    }
+    if (warp == kWarpAlloc) {
+        tmem_alloc(smem_u32(&S.tmem_base), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = S.tmem_base;
+
+    if (warp == kWarpTma) {
+        if (lane == 0) {
+            uint32_t it = 0;
+            for (int t = blockIdx.x; t < num_tiles && !*abort; t += gridDim.x) {
+                const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % kStages;
+                    const uint32_t ph = (it / kStages) & 1;
+                    if (!mbar_wait(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status)) break;
+                    mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
+                    tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
+                    tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
+                }
+            }
+            // teardown: every load issued must have landed before the CTA exits
+            const uint32_t issued = it;
+            for (uint32_t j = issued > (uint32_t)kStages ? issued - kStages : 0; j < issued; ++j)
+                wait_teardown(smem_u32(&S.full[j % kStages]), (j / kStages) & 1);
+        }
+    } else if (warp == kWarpMma) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16_f32(kBM, BN);
+            uint32_t it = 0, g = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+                for (int kb0 = 0; kb0 < nkb && ok; kb0 += kcb, ++g) {
+                    const int buf = g & 1;
+                    if (!(ok = mbar_wait(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
+                    tc_fence_after();
+                    const uint32_t d = tmem + kTmemAccCol + buf * BN;
+                    const int kb1 = min(nkb, kb0 + kcb);
+                    for (int kb = kb0; kb < kb1; ++kb, ++it) {
+                        const int s = it % kStages;
+                        const uint32_t ph = (it / kStages) & 1;
+                        if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
+                        if (!(ok = mbar_wait(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
+                        tc_fence_after();
+                        const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
+#pragma unroll
+                        for (int kk = 0; kk < kBK / 16; ++kk)
+                            mma_f16_ts(d, tmem + s * 32 + kk * 8, bdesc + (uint64_t)((kk * 32) >> 4), idesc,
+                                       (kb != kb0 || kk != 0) ? 1u : 0u);
+                        mma_commit(smem_u32(&S.empty[s]));
+                        mma_commit(smem_u32(&S.aempty[s]));
+                    }
+                    if (ok) mma_commit(smem_u32(&S.accfull[buf]));
+                }
+            }
+            // teardown: all issued MMAs complete before TMEM is freed
+            mma_commit(smem_u32(&S.drain));
+            wait_teardown(smem_u32(&S.drain), 0);
+        }
+    } else if (warp >= kWarpConv0 && warp < kWarpConv0 + 4) {
+        const int q = warp & 3;
+        const int row = q * 32 + lane;           // weight row of the tile = TMEM lane
+        const uint32_t sw64 = (row >> 1) & 3;    // 64-byte swizzle phase of this row
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        uint32_t it = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+            for (int kb = 0; kb < nkb; ++kb, ++it) {
+                const int s = it % kStages;
+                const uint32_t ph = (it / kStages) & 1;
+                if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
+                uint4 raw[4];
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    raw[c] = *reinterpret_cast<const uint4 *>(S.w[s] + row * 64 + ((c ^ sw64) << 4));
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&S.empty[s]));
+                uint32_t a[32];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    i8x4_to_f16x4(raw[c].x, a[8 * c + 0], a[8 * c + 1]);
+                    i8x4_to_f16x4(raw[c].y, a[8 * c + 2], a[8 * c + 3]);
+                    i8x4_to_f16x4(raw[c].z, a[8 * c + 4], a[8 * c + 5]);
+                    i8x4_to_f16x4(raw[c].w, a[8 * c + 6], a[8 * c + 7]);
+                }
+                if (!(ok = mbar_wait(smem_u32(&S.aempty[s]), ph ^ 1, abort, &g_status))) break;
+                tc_fence_after();
+                tmem_st32(tmem + lane_base + s * 32, a);
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&S.afull[s]));
+            }
+        }
+    } else if (warp >= kWarpEpi0) {
+        constexpr int CPW = BN / 2;              // accumulator columns per epilogue warp
+        constexpr int PIECE = CPW < 32 ? CPW : 32;
+        const int e = warp - kWarpEpi0;
+        const int q = warp & 3;
+        const int col0 = (e >> 2) * CPW;
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        uint32_t g = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+            const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
+            int32_t tot[CPW];
+#pragma unroll
+            for (int j = 0; j < CPW; ++j) tot[j] = 0;
+            for (int kb0 = 0; kb0 < nkb; kb0 += kcb, ++g) {
+                const int buf = g & 1;
+                if (!(ok = mbar_wait(smem_u32(&S.accfull[buf]), (g >> 1) & 1, abort, &g_status))) break;
+                tc_fence_after();
+                const uint32_t base = tmem + lane_base + kTmemAccCol + buf * BN + col0;
+#pragma unroll
+                for (int p = 0; p < CPW / PIECE; ++p) {
+                    uint32_t v[PIECE];
+                    if constexpr (PIECE == 32) tmem_ld32(base + p * 32, v);
+                    else if constexpr (PIECE == 16) tmem_ld16(base + p * 16, v);
+                    else tmem_ld8(base + p * 8, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int j = 0; j < PIECE; ++j) tot[p * PIECE + j] += __float2int_rn(__uint_as_float(v[j]));
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&S.accempty[buf]));
+            }
+            if (!ok) break;
+            const int n = n0 + q * 32 + lane;
+            if (n < N) {
+                if constexpr (kS32) {
+                    int32_t *o = reinterpret_cast<int32_t *>(out);
+#pragma unroll
+                    for (int j = 0; j < CPW; ++j) {
+                        const int m = m0 + col0 + j;
+                        if (m < M) o[(int64_t)m * N + n] = tot[j];
+                    }
+                } else {
+                    const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
+                    __half *o = reinterpret_cast<__half *>(out);
+#pragma unroll
+                    for (int j = 0; j < CPW; ++j) {
+                        const int m = m0 + col0 + j;
+                        float v = __fmaf_rn(__int2float_rn(tot[j]), scale, bias);
+                        if (relu) v = fmaxf(v, 0.f);
+                        if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                    }
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kWarpAlloc) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void *p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+bool make_tmap_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
+                  uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, rows};
+    cuuint64_t strides[1] = {row_bytes};
+    cuuint32_t box[2] = {box_inner, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(tm, dt, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int BN, bool kS32>
+cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
+    CUtensorMap tm_q, tm_w;
+    if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
+                      (uint64_t)a.K * 2, kBK, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
+                      kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
+        return cudaErrorInvalidValue;
+    // at least 120 KB so two CTAs never share an SM (each takes all 512 TMEM columns)
+    const size_t smem = sizeof(Smem<BN>) + 1024 > 120 * 1024 ? sizeof(Smem<BN>) + 1024 : 120 * 1024;
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)smem);
+    });
+    if (attr_err != cudaSuccess) return attr_err;
+    const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
+    const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
+    linear_kernel<BN, kS32><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
+                                                         (int)a.K, (int)a.ldy, kcb, a.relu);
+    return cudaGetLastError();
+}
+
+template <bool kS32>
+cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
+    if (a.M <= 16) return run_linear<16, kS32>(a, kcb, st);
+    if (a.M <= 32) return run_linear<32, kS32>(a, kcb, st);
+    if (a.M <= 64) return run_linear<64, kS32>(a, kcb, st);
+    return run_linear<128, kS32>(a, kcb, st);
+}
+
+}  // namespace
+
+// Largest number of 64-wide k-blocks whose fp32 partial sums stay exact:
+// kcb * 64 * qmax_a * qmax_w <= 2^24.
+int exact_chunk_kblocks(int bits_a, int bits_w) {
+    const int64_t qa = (1 << (bits_a - 1)) - 1, qw = (1 << (bits_w - 1)) - 1;
+    int64_t kc = ((int64_t)1 << 24) / (qa * qw);
+    kc /= kBK;
+    return kc < 1 ? 1 : (int)kc;
+}
+
+cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
+    if (a.M == 0 || a.N == 0) return cudaSuccess;
+    const int nkb = (int)((a.K + kBK - 1) / kBK);
+    int kcb = exact_chunk_kblocks(a.bits_a, a.bits_w);
+    if (kcb > nkb) kcb = nkb;
+    return a.out_s32 ? dispatch_bn<true>(a, kcb, st) : dispatch_bn<false>(a, kcb, st);
+}
+
+}  // namespace ot
+
+namespace ot {
+
+cudaError_t read_clear_status(int *value, cudaStream_t st) {
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return e;
+    int v = 0;
+    e = cudaMemcpyFromSymbol(&v, g_status, sizeof(int));
+    if (e != cudaSuccess) return e;
+    const int zero = 0;
+    e = cudaMemcpyToSymbol(g_status, &zero, sizeof(int));
+    *value = v;
+    return e;
+}
+
+}  // namespace ot

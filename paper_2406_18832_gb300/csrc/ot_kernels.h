@@ -1,0 +1,37 @@
+// ot_kernels.h -- host-side launchers of the sm_103a kernels (internal to the
+// library; the public boundary is include/outliertune.h).  Every launcher
+// assumes its arguments were validated by the C-ABI layer in api.cu and
+// returns the launch error of its kernel(s).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace ot {
+
+cudaError_t launch_calibrate(const void *x, int64_t T, int64_t K, int64_t ldx, float *mn, float *mx, int reset,
+                             cudaStream_t st);
+cudaError_t launch_params(const float *mn, const float *mx, int64_t K, int bits, int symmetrize, float *z,
+                          float *s, float *r, cudaStream_t st);
+cudaError_t launch_fold(const void *w, const void *b, int64_t N, int64_t K, const float *z, const float *s,
+                        int bits_w, int8_t *qw, float *sw, float *bfold, cudaStream_t st);
+cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
+                            int bits, void *q, int fmt, cudaStream_t st);
+
+struct LinearArgs {
+    const void *q;        // fp16 codes [M, K]
+    const int8_t *qw;     // int8 codes [N, K]
+    const float *sw;      // [N] (fp16 output only)
+    const float *bfold;   // [N] (fp16 output only)
+    void *out;            // fp16 y [M, ldy] or int32 acc [M, N]
+    int64_t M, N, K, ldy;
+    int bits_a, bits_w, relu;
+    bool out_s32;
+};
+cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
+
+int num_sms();
+int exact_chunk_kblocks(int bits_a, int bits_w);
+cudaError_t read_clear_status(int *value, cudaStream_t st);
+
+}  // namespace ot

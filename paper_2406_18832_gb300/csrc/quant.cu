@@ -1,0 +1,107 @@
+// quant.cu -- per-channel static activation quantization, round(X_hat / s)
+// with X_hat = X - z (Eq. 6, Eq. 7): q = clamp(rne((x - z_k) * r_k)).
+// HBM-bound: one 16-byte fp16 load and one 16-byte (fp16 codes) or 8-byte
+// (int8 codes) store per 8 elements, coalesced across the warp.
+#include <cuda_fp16.h>
+
+#include "ot_common.cuh"
+#include "ot_kernels.h"
+
+namespace ot {
+
+namespace {
+
+constexpr int kQRowsPerThread = 8;              // rows a thread walks with the same z, r
+constexpr int kQRowsPerBlock = 8 * kQRowsPerThread;
+
+__device__ __forceinline__ int code_of(float x, float z, float r, int qmax) {
+    // two fp32 roundings as written (no contraction), then round half to even;
+    // cvt.rni.s32.f32 maps NaN to 0 and saturates out-of-range values
+    const float u = __fmul_rn(__fsub_rn(x, z), r);
+    const int c = __float2int_rn(u);
+    return max(-qmax, min(qmax, c));
+}
+
+// fp16 holding the integer c (|c| <= 128): 1152 + c lies in [1024, 2048) where
+// fp16 has unit spacing, so its bit pattern is 0x6400 | (128 + c); subtracting
+// 1152 in fp16 is exact.
+__device__ __forceinline__ uint32_t pack_f16_codes(int c0, int c1) {
+    const uint32_t bits = (uint32_t)(0x6480 + c0) | ((uint32_t)(0x6480 + c1) << 16);
+    const __half2 v = __hsub2(*reinterpret_cast<const __half2 *>(&bits), __half2half2(__ushort_as_half(0x6480)));
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__device__ __forceinline__ uint32_t pack_i8_codes(int c0, int c1, int c2, int c3) {
+    const uint32_t lo = __byte_perm((uint32_t)c0, (uint32_t)c1, 0x0040);
+    const uint32_t hi = __byte_perm((uint32_t)c2, (uint32_t)c3, 0x0040);
+    return __byte_perm(lo, hi, 0x5410);
+}
+
+// Block 32 x 8: threadIdx.x owns 8 consecutive channels of a 256-channel
+// strip (blockIdx.x) and keeps their z, r in registers while it walks
+// kQRowsPerThread rows of the block's row range (blockIdx.y).
+template <bool kF16Out>
+__global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict__ x, int64_t M, int64_t K,
+                                                       int64_t ldx, const float *__restrict__ z,
+                                                       const float *__restrict__ r, int qmax, void *q) {
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int64_t c0 = (int64_t)blockIdx.x * 256 + tx * 8;
+    if (c0 >= K) return;
+    float zz[8], rr[8];
+    {
+        const float4 *zp = reinterpret_cast<const float4 *>(z + c0);
+        const float4 *rp = reinterpret_cast<const float4 *>(r + c0);
+        float4 a = __ldg(zp), b = __ldg(zp + 1), c = __ldg(rp), d = __ldg(rp + 1);
+        zz[0] = a.x; zz[1] = a.y; zz[2] = a.z; zz[3] = a.w; zz[4] = b.x; zz[5] = b.y; zz[6] = b.z; zz[7] = b.w;
+        rr[0] = c.x; rr[1] = c.y; rr[2] = c.z; rr[3] = c.w; rr[4] = d.x; rr[5] = d.y; rr[6] = d.z; rr[7] = d.w;
+    }
+    const int64_t row0 = (int64_t)blockIdx.y * kQRowsPerBlock + ty;
+    uint4 v[kQRowsPerThread];
+#pragma unroll
+    for (int u = 0; u < kQRowsPerThread; ++u) {
+        const int64_t m = row0 + 8 * u;
+        if (m < M) v[u] = __ldcs(reinterpret_cast<const uint4 *>(x + m * ldx + c0));
+    }
+#pragma unroll
+    for (int u = 0; u < kQRowsPerThread; ++u) {
+        const int64_t m = row0 + 8 * u;
+        if (m >= M) break;
+        const __half2 *h = reinterpret_cast<const __half2 *>(&v[u]);
+        int c[8];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 f = __half22float2(h[j]);
+            c[2 * j] = code_of(f.x, zz[2 * j], rr[2 * j], qmax);
+            c[2 * j + 1] = code_of(f.y, zz[2 * j + 1], rr[2 * j + 1], qmax);
+        }
+        if (kF16Out) {
+            uint4 o;
+            o.x = pack_f16_codes(c[0], c[1]);
+            o.y = pack_f16_codes(c[2], c[3]);
+            o.z = pack_f16_codes(c[4], c[5]);
+            o.w = pack_f16_codes(c[6], c[7]);
+            *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + m * K + c0) = o;
+        } else {
+            uint2 o;
+            o.x = pack_i8_codes(c[0], c[1], c[2], c[3]);
+            o.y = pack_i8_codes(c[4], c[5], c[6], c[7]);
+            *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + m * K + c0) = o;
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
+                            int bits, void *q, int fmt, cudaStream_t st) {
+    if (M == 0) return cudaSuccess;
+    const int qmax = (1 << (bits - 1)) - 1;
+    dim3 grid((unsigned)((K + 255) / 256), (unsigned)((M + kQRowsPerBlock - 1) / kQRowsPerBlock));
+    if (fmt == OT_CODE_F16)
+        quantize_kernel<true><<<grid, 256, 0, st>>>(reinterpret_cast<const __half *>(x), M, K, ldx, z, r, qmax, q);
+    else
+        quantize_kernel<false><<<grid, 256, 0, st>>>(reinterpret_cast<const __half *>(x), M, K, ldx, z, r, qmax, q);
+    return cudaGetLastError();
+}
+
+}  // namespace ot
