@@ -1,0 +1,479 @@
+"""Benchmark of the per-channel quantized linear (OutlierTune, arXiv 2406.18832)
+on GB300.
+
+Workload: the four OPT-6.7B-shaped linears (QKV 4096->12288, out 4096->4096,
+fc1 4096->16384, fc2 16384->4096) at a prefill of 2048 tokens, W8A8, with
+synthetic LayerNorm-like activations carrying 0.5% fixed outlier channels.
+Offline per layer (not in the step, measured separately): calibration over
+65536 tokens and the weight fold.  One step = for every layer, the
+symmetrize+quantize kernel then the tcgen05 GEMM with its fused epilogue.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line.  The value is exact int8 tera-operations per second
+(2*M*N*K per linear) over the whole step.  --impl reference times the CPU
+oracle on a bounded sample of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD_CFG = 2          # OPT-6.7B-shaped linears
+TOKENS = 2048
+BITS = (8, 8)
+METRIC = "W8A8 linear TOPS & % INT8 peak; quantize GB/s % HBM; vs cuBLAS FP16"
+L2_BYTES = 129 * 2 ** 20
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
+                    bf16_sus=float(p["bf16_tflops_sustained"]), source="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def _env_rank():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), \
+        int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def _workload_desc():
+    from paper_2406_18832_gb300 import synth
+    c = synth.CONFIGS[WORKLOAD_CFG]
+    return c, [(l.name, l.K, l.N) for l in c.layers]
+
+
+def _ops_per_step(layers, tokens):
+    return sum(2 * tokens * K * N for _, K, N in layers)
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = "index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active," \
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown," \
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap"
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(parts[1]), max=float(parts[2]), power=float(parts[3]),
+                                 hw=parts[5], hwt=parts[6], swt=parts[7], pcap=parts[8]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        loaded = [r for r in rows if r["power"] > 200.0] or rows
+        reasons = set()
+        for r in loaded:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in loaded), "sm_max_mhz": max(r["max"] for r in rows),
+                "reasons": sorted(reasons), "samples": len(loaded),
+                "power_w_max": max(r["power"] for r in rows)}
+
+
+def _traffic_record():
+    """DRAM bytes per GEMM launch from the committed ncu summary, if the GEMM
+    source is unchanged since it was captured (else None)."""
+    path = os.path.join(ROOT, "profiles", "linear_kernel_traffic.txt")
+    src = os.path.join(ROOT, "paper_2406_18832_gb300", "csrc", "gemm.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        vals = {}
+        for line in open(path):
+            line = line.strip()
+            if "=" in line and not line.startswith("#"):
+                k, v = line.split("=", 1)
+                vals[k.strip()] = v.strip()
+        if vals.get("gemm_cu_sha256_16") != sha:
+            return None
+        return float(vals["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------
+# the CUDA path
+# ----------------------------------------------------------------------------
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2406_18832_gb300 import QuantizedLinear, binding, synth
+
+    rank, world, local = _env_rank()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    binding.load()
+    peaks = _peaks()
+    cfg, layer_shapes = _workload_desc()
+    bits_a, bits_w = BITS
+
+    # ---- offline: inputs, calibration, fold (each rank its own replica) ----
+    layers, xs = [], []
+    calib_ms, calib_bytes, fold_ms = [], 0, []
+    for li, layer in enumerate(cfg.layers):
+        w, b = synth.weights(WORKLOAD_CFG, li, layer, device=dev)
+        t_cal = 8192 if args.profile else cfg.T_cal
+        xc = synth.activations(WORKLOAD_CFG, li, layer, t_cal, 3, device=dev)
+        x = synth.activations(WORKLOAD_CFG, li, layer, TOKENS, 4, device=dev)
+        ql = QuantizedLinear(layer.K, layer.N, bits_a, bits_w, relu=layer.relu_out, device=dev)
+        # calibration: warm once, then time one pass over the calibration tokens
+        ql.calibrate(xc)
+        ql._calibrated = False
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        ql.calibrate(xc)
+        e1.record()
+        torch.cuda.synchronize()
+        calib_ms.append(e0.elapsed_time(e1))
+        calib_bytes += xc.numel() * 2
+        e0.record()
+        ql.fold(w, b)
+        e1.record()
+        torch.cuda.synchronize()
+        fold_ms.append(e0.elapsed_time(e1))
+        del xc
+        layers.append((ql, w, b))
+        xs.append(x)
+    torch.cuda.empty_cache()
+    qbufs = [torch.empty(TOKENS, l.K, dtype=torch.float16, device=dev) for l in cfg.layers]
+    ybufs = [torch.empty(TOKENS, l.N, dtype=torch.float16, device=dev) for l in cfg.layers]
+    ops_step = _ops_per_step(layer_shapes, TOKENS)
+    stream = torch.cuda.current_stream()
+
+    def step(evs=None):
+        for i, (ql, _, _) in enumerate(layers):
+            if evs is not None:
+                evs[i][0].record(stream)
+            ql.quantize(xs[i], qbufs[i])
+            if evs is not None:
+                evs[i][1].record(stream)
+            ql.linear(qbufs[i], ybufs[i])
+            if evs is not None:
+                evs[i][2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    if args.profile:
+        # small, short run for profilers: the steps only, nothing else
+        for _ in range(args.steps):
+            step()
+        torch.cuda.synchronize()
+        if rank == 0:
+            print(json.dumps({"profile_run": True, "steps": args.steps}), flush=True)
+        return
+
+    nl = len(layers)
+    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(nl)]
+              for _ in range(args.steps)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(torch.cuda.current_device() if world == 1 else local) as clk:
+        t0.record(stream)
+        for k in range(args.steps):
+            step(events[k])
+        t1.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    total_ms = t0.elapsed_time(t1)
+    gemm_ms = [[events[k][i][1].elapsed_time(events[k][i][2]) for k in range(args.steps)] for i in range(nl)]
+    quant_ms = [[events[k][i][0].elapsed_time(events[k][i][1]) for k in range(args.steps)] for i in range(nl)]
+    if world > 1:
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    value = world * ops_step * args.steps / (total_ms * 1e-3) / 1e12
+
+    # GEMM roofline (dominant kernel): algorithmic ops / measured launch time
+    gemm_ops = [2 * TOKENS * K * N for _, K, N in layer_shapes]
+    gemm_time = sum(sum(v) for v in gemm_ms)
+    gemm_tops = sum(o * args.steps for o in gemm_ops) / (gemm_time * 1e-3) / 1e12
+    per_layer = []
+    for i, (name, K, N) in enumerate(layer_shapes):
+        g = statistics.median(gemm_ms[i])
+        q = statistics.median(quant_ms[i])
+        qbytes = TOKENS * K * 4 + 8 * K
+        per_layer.append({"layer": name, "K": K, "N": N, "gemm_us": round(g * 1e3, 2),
+                          "gemm_tops": round(gemm_ops[i] / (g * 1e-3) / 1e12, 1),
+                          "quant_us": round(q * 1e3, 2), "quant_gbs": round(qbytes / (q * 1e-3) / 1e9, 1)})
+    qbytes_total = sum(TOKENS * K * 4 + 8 * K for _, K, _ in layer_shapes)
+    quant_time = sum(sum(v) for v in quant_ms) / args.steps
+    quant_gbs = qbytes_total / (quant_time * 1e-3) / 1e9
+    clocks = clk.summary()
+    long_run = total_ms > 4000.0
+    peak = peaks["bf16_sus"] if long_run else peaks["bf16"]
+    roofline = {"kernel": "linear_kernel (tcgen05 kind::f16, exact int8 codes)", "bound": "tensor",
+                "achieved": round(gemm_tops, 1), "peak": peak, "unit": "TFLOP/s",
+                "frac": round(gemm_tops / peak, 4), "traffic": _traffic_record(),
+                "peak_source": f"{peaks['source']} bf16 dense {'sustained' if long_run else 'burst'} "
+                               "(fp16 dense runs at the bf16 rate)"}
+
+    # ---- comparators: cuBLAS fp16 GEMM of the same shapes, cuBLASLt int8 ----
+    reps = max(10, min(200, args.steps))
+    cub = []
+    for i, (ql, w, b) in enumerate(layers):
+        def f():
+            torch.matmul(xs[i], w.t(), out=ybufs[i])
+        for _ in range(3):
+            f()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            f()
+        e1.record()
+        torch.cuda.synchronize()
+        cub.append(e0.elapsed_time(e1) / reps)
+    cub_step_ms = sum(cub)
+    int8_tops = None
+    try:
+        _, K0, N0 = layer_shapes[0]
+        a8 = torch.randint(-127, 128, (TOKENS, K0), device=dev, dtype=torch.int8)
+        b8 = torch.randint(-127, 128, (K0, N0), device=dev, dtype=torch.int8)
+        for _ in range(2):
+            torch._int_mm(a8, b8)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(5):
+            torch._int_mm(a8, b8)
+        e1.record()
+        torch.cuda.synchronize()
+        int8_tops = 2 * TOKENS * K0 * N0 / (e0.elapsed_time(e1) / 5 * 1e-3) / 1e12
+        del a8, b8
+    except Exception:
+        int8_tops = None
+
+    # ---- end to end through the public API, host buffers in and out ----
+    e2e_steps = max(3, min(100, args.steps))
+    hx = [x.cpu().pin_memory() for x in xs]
+    hy = [torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in ybufs]
+    dx = [torch.empty_like(x) for x in xs]
+
+    def e2e_step():
+        for i, (ql, _, _) in enumerate(layers):
+            dx[i].copy_(hx[i], non_blocking=True)
+            ql.forward(dx[i], qbufs[i], ybufs[i])
+            hy[i].copy_(ybufs[i], non_blocking=True)
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    h2d = sum(x.numel() * 2 for x in xs)
+    d2h = sum(y.numel() * 2 for y in ybufs)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(budget_s=args.cpu_budget, layers=layers)
+
+    weights_fp16 = sum(2 * K * N for _, K, N in layer_shapes)
+    weights_int8 = sum(ql.weight_bytes() for ql, _, _ in layers)
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "int8 codes exact on the f16 tensor pipe (fp32 chunk sums, int32 totals)",
+        "data": "synthetic",
+        "config": {"workload": "opt-6.7b-linears-prefill", "tokens": TOKENS, "bits_a": bits_a, "bits_w": bits_w,
+                   "layers": [{"name": n, "K": K, "N": N} for n, K, N in layer_shapes],
+                   "calibration_tokens": cfg.T_cal, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2: one step streams 201 MB of int8 weights and 470 MB of "
+                         "activations and outputs through the 129 MB L2"},
+        "roofline": roofline,
+        "gpu_launches": args.steps * 2 * len(layers),
+        "e2e": {"value": round(ops_step / (e2e_ms * 1e-3) / 1e12 * world, 2), "unit": "TOPS",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4)},
+        "clocks": clocks,
+        "quantize": {"gbs": round(quant_gbs, 1), "hbm_peak_gbs": peaks["hbm"],
+                     "frac": round(quant_gbs / peaks["hbm"], 4),
+                     "bytes_per_step": qbytes_total, "note": "fp16 X in + fp16 codes out + z, r"},
+        "calibrate": {"gbs": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9, 1),
+                      "frac": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9 / peaks["hbm"], 4),
+                      "tokens": cfg.T_cal, "ms_per_layer": [round(v, 3) for v in calib_ms]},
+        "fold_ms_per_layer": [round(v, 3) for v in fold_ms],
+        "cublas_fp16": {"ms_per_step": round(cub_step_ms, 4),
+                        "tflops": round(ops_step / (cub_step_ms * 1e-3) / 1e12, 1),
+                        "ours_over_cublas": round(cub_step_ms / ms_per_step, 4)},
+        "int8_peak": {"cublaslt_int8_tops": None if int8_tops is None else round(int8_tops, 1),
+                      "frac_of_cublaslt_int8": None if not int8_tops else round(gemm_tops / int8_tops, 2),
+                      "note": "GB300 has no tcgen05 int8 MMA; cuBLASLt int8 (torch._int_mm) of the QKV shape, "
+                              "measured in this run"},
+        "per_layer": per_layer,
+        "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
+                   "ratio": round(weights_fp16 / weights_int8, 3)},
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+# ----------------------------------------------------------------------------
+# the CPU oracle (baseline leg and --impl reference)
+# ----------------------------------------------------------------------------
+def _oracle_layers(device_layers=None):
+    """Folded weights for every layer, computed by the oracle on the host."""
+    import numpy as np
+
+    import oracle
+    from paper_2406_18832_gb300 import synth
+    cfg, _ = _workload_desc()
+    out = []
+    for li, layer in enumerate(cfg.layers):
+        w, b = synth.weights(WORKLOAD_CFG, li, layer)
+        xc = synth.activations(WORKLOAD_CFG, li, layer, 4096, 3)   # calibration sample (host)
+        mn, mx = oracle.calibrate(xc.numpy())
+        z, s, r = oracle.params(mn, mx, BITS[0])
+        qw, sw, bf = oracle.fold(w.numpy(), b.numpy(), z, s, BITS[1])
+        x = synth.activations(WORKLOAD_CFG, li, layer, 64, 4).numpy()
+        out.append(dict(qw=qw, sw=sw, bf=bf, z=z, r=r, x=x, K=layer.K, N=layer.N))
+    return out
+
+
+def _oracle_sample(ol, rows, cols):
+    import oracle
+    ops = 0
+    for d in ol:
+        x = d["x"][:rows]
+        q = oracle.quantize(x, d["z"], d["r"], BITS[0])
+        n = min(cols, d["N"])
+        acc = oracle.matmul(q, d["qw"][:n])
+        oracle.epilogue(acc, d["sw"][:n], d["bf"][:n])
+        ops += 2 * rows * n * d["K"]
+    return ops
+
+
+def cpu_baseline(budget_s=12.0, layers=None):
+    """Time the oracle (single-threaded C, as it stands) on a bounded sample of
+    the workload: `rows` tokens through the four layers, all output channels."""
+    ol = _oracle_layers()
+    t = time.perf_counter()
+    ops = _oracle_sample(ol, 1, 10 ** 9)
+    one = time.perf_counter() - t
+    rows = max(1, min(64, int(budget_s / max(one, 1e-6))))
+    t = time.perf_counter()
+    ops = _oracle_sample(ol, rows, 10 ** 9)
+    dt = time.perf_counter() - t
+    return {"value": round(ops / dt / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
+            "sample": f"{rows} token(s) of the 2048 through all four layers (quantize, int64 product, "
+                      f"fp64 epilogue), every output channel; {dt:.1f} s",
+            "host_cores_available": len(os.sched_getaffinity(0))}
+
+
+def run_reference(args):
+    rank, world, _ = _env_rank()
+    if rank != 0:
+        return
+    ol = _oracle_layers()
+    _, layer_shapes = _workload_desc()
+    # size one step so that warmup + steps fit in about two minutes of host time
+    t = time.perf_counter()
+    _oracle_sample(ol, 1, 256)
+    per256 = time.perf_counter() - t
+    budget_step = max(0.01, 120.0 / max(1, args.steps + args.warmup))
+    cols = int(max(16, min(16384, 256 * budget_step / max(per256, 1e-6))))
+    for _ in range(args.warmup):
+        _oracle_sample(ol, 1, cols)
+    t = time.perf_counter()
+    ops = 0
+    for _ in range(args.steps):
+        ops += _oracle_sample(ol, 1, cols)
+    dt = time.perf_counter() - t
+    value = ops / dt / 1e12
+    sample = (f"per step: 1 token through all four layers, first {cols} output channels of each "
+              f"(quantize, int64 product, fp64 epilogue)")
+    line = {"metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int64 (CPU oracle)", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": "opt-6.7b-linears-prefill", "tokens": TOKENS, "bits_a": BITS[0],
+                       "bits_w": BITS[1], "layers": [{"name": n, "K": K, "N": N} for n, K, N in layer_shapes]},
+            "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="profiler run: 8192 calibration tokens, the timed steps only, no report")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()
