@@ -290,66 +290,79 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
-// Wide-tile variant for prefill-sized token counts (M > 128).
+// Wide-tile CTA-pair variant for prefill-sized token counts (M > 128).
 //
-// The tensor core reaches its full rate only with N = 256 instructions
-// (a 128 x N x 16 kind::f16 MMA costs about as much for N = 64 or 128 as for
-// N = 256), and one SM cannot be fed 24 KB of operands per 256 clocks from L2.
-// So each CTA computes 128 weight rows x 256 tokens, and the two CTAs of a
-// cluster (adjacent 128-row weight slices, the same 256 tokens) split the
-// activation-code tile: each loads 128 token rows and multicasts them to both,
-// which halves the L2 -> SM bytes of the shared operand.
-//   TMEM: A buffers (W in fp16) at columns [0, 32*kMcStages), the fp32 chunk
-//   accumulator (128 lanes x 256 columns) at [256, 512).
+// Measured on GB300: a 128 x N x 16 kind::f16 MMA costs about as much for
+// N = 64 or 128 as for N = 256, so only N = 256 instructions reach the tensor
+// peak; and TMA ingest per SM is latency-bound (about 1.6 us per load under
+// load), so the fewer bytes an SM must receive per MMA the better.
+// So the two CTAs of a cluster run one cta_group::2 MMA of 256 weight rows x
+// 256 tokens: each CTA loads its own 128 int8 weight rows (8 KB per 64-wide
+// k-block) and half of the token tile (128 rows of fp16 codes, 16 KB); B is
+// split along N between the pair and each CTA's TMEM receives its 128 rows x
+// 256 tokens of the accumulator.
+// The converters widen each CTA's int8 weight rows into an fp16 A tile in
+// shared memory (128-byte swizzle), so all 512 TMEM columns can hold two
+// 256-column chunk accumulators: while the MMA fills one, the epilogue
+// converts the other (fp32 -> int32 conversions run at a quarter rate and
+// would otherwise stall the tensor core at every chunk boundary).
+//   Rank 0 of the pair issues the MMAs.  The converters and epilogue warps
+//   of both CTAs signal rank 0's barriers; rank 0's commits arrive on the
+//   barriers of both CTAs (multicast).  One commit per k-block (done[s])
+//   frees both the TMA slot and, kAStages k-blocks later, the A tile: each
+//   extra tcgen05.commit per k-block costs about 10% of tensor throughput.
 //   Warpgroups: 0 = TMA producer / MMA issuer / TMEM allocator (56 regs),
 //   1 = converters (88 regs), 2-3 = epilogue (184 regs: 128 int32 totals).
-// The chunk accumulator is single-buffered: the MMA of the next chunk waits
-// until the epilogue has read the previous one out of TMEM.
 // ---------------------------------------------------------------------------
-constexpr int kMcBN = 256;
-constexpr int kMcStages = 5;
-constexpr uint32_t kMcAccCol = 256;
-static_assert(32 * kMcStages <= (int)kMcAccCol, "TMEM A buffers overlap the accumulator");
+constexpr int kPairBN = 256;   // tokens per pair tile (MMA N)
+constexpr int kRing = 6;       // TMA stages: token half-tile + weight rows
+constexpr int kAStages = 3;    // fp16 A tiles written by the converters
+static_assert(kRing % kAStages == 0, "A tile of k-block i is freed by the commit of k-block i - kAStages");
 
-struct alignas(1024) SmemMc {
-    uint8_t b[kMcStages][kMcBN * 128];  // 256 token rows of fp16 codes, 128-byte swizzle (32 KB)
-    uint8_t w[kMcStages][kBM * kBK];    // 128 weight rows of int8 codes, 64-byte swizzle (8 KB)
-    uint64_t full[kMcStages];           // own W + both halves of B landed
-    uint64_t empty[kMcStages];          // both CTAs' MMAs done with b[] + 4 converter warps done with w[]
-    uint64_t afull[kMcStages];
-    uint64_t aempty[kMcStages];
-    uint64_t accfull, accempty, drain;
+struct alignas(1024) SmemPair {
+    uint8_t b[kRing][kBM * 128];      // this CTA's 128 token rows of fp16 codes, 128-byte swizzle (16 KB)
+    uint8_t a[kAStages][kBM * 128];   // this CTA's 128 weight rows widened to fp16, 128-byte swizzle (16 KB)
+    uint8_t w[kRing][kBM * kBK];      // this CTA's 128 weight rows of int8 codes, 64-byte swizzle (8 KB)
+    uint64_t full[kRing];             // own TMA landed
+    uint64_t done[kRing];             // pair MMA of the k-block done (rank 0 commit, both CTAs)
+    uint64_t wread[kRing];            // own 4 converter warps read w[]
+    uint64_t afull[kAStages];         // rank 0 only: both CTAs' converters wrote their A tiles (8 warps)
+    uint64_t accfull[2];              // pair MMA finished the chunk (rank 0 commit)
+    uint64_t accempty[2];             // rank 0 only: both CTAs' epilogues drained the chunk (16 warps)
+    uint64_t drain;
     uint32_t tmem_base;
     int abort;
 };
 
 template <bool kS32>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-    linear_mc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
-                     const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
-                     int N, int K, int ldy, int kcb, int relu) {
+    linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
+                       const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
+                       int N, int K, int ldy, int kcb, int relu) {
     extern __shared__ uint8_t smem_raw[];
-    SmemMc &S = *reinterpret_cast<SmemMc *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    SmemPair &S = *reinterpret_cast<SmemPair *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
     const uint32_t rank = cluster_ctarank();
     const int cluster = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
-    const int m_tiles = (M + kMcBN - 1) / kMcBN;
+    const int m_tiles = (M + kPairBN - 1) / kPairBN;
     const int n_pairs = (N + 2 * kBM - 1) / (2 * kBM);
     const int num_units = m_tiles * n_pairs;
     const int nkb = (K + kBK - 1) / kBK;
     volatile int *abort = &S.abort;
-    constexpr uint32_t kTxBytes = kMcBN * 128 + kBM * kBK;
-    constexpr uint16_t kPair = 0x3;
+    constexpr uint32_t kTxBytes = kBM * 128 + kBM * kBK;
+    constexpr uint16_t kBoth = 0x3;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kMcStages; ++s) {
+        for (int s = 0; s < kRing; ++s) {
             mbar_init(smem_u32(&S.full[s]), 1);
-            mbar_init(smem_u32(&S.empty[s]), 2 + 4);
-            mbar_init(smem_u32(&S.afull[s]), 4);
-            mbar_init(smem_u32(&S.aempty[s]), 1);
+            mbar_init(smem_u32(&S.done[s]), 1);
+            mbar_init(smem_u32(&S.wread[s]), 4);
         }
-        mbar_init(smem_u32(&S.accfull), 1);
-        mbar_init(smem_u32(&S.accempty), kNumEpiWarps);
+        for (int s = 0; s < kAStages; ++s) mbar_init(smem_u32(&S.afull[s]), 8);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&S.accfull[b]), 1);
+            mbar_init(smem_u32(&S.accempty[b]), 2 * kNumEpiWarps);
+        }
         mbar_init(smem_u32(&S.drain), 1);
         S.abort = 0;
         fence_barrier_init();
@@ -359,12 +372,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tma_prefetch_desc(&tm_w);
     }
     if (warp == kWarpAlloc) {
-        tmem_alloc(smem_u32(&S.tmem_base), kTmemCols);
-        tmem_relinquish();
+        tmem_alloc_pair(smem_u32(&S.tmem_base), kTmemCols);
+        tmem_relinquish_pair();
     }
     tc_fence_before();
     __syncthreads();
-    cluster_sync();  // the peer's barriers exist before anything is multicast into them
+    cluster_sync();  // barriers of both CTAs exist before either signals the other
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
 
@@ -373,85 +386,90 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (warp == kWarpTma && lane == 0) {
             uint32_t it = 0;
             for (int u = cluster; u < num_units && !*abort; u += nclusters) {
-                const int m0 = (u % m_tiles) * kMcBN;
+                const int m0 = (u % m_tiles) * kPairBN + (int)rank * kBM;
                 const int n0 = ((u / m_tiles) * 2 + (int)rank) * kBM;
                 for (int kb = 0; kb < nkb; ++kb, ++it) {
-                    const int s = it % kMcStages;
-                    const uint32_t ph = (it / kMcStages) & 1;
-                    if (!mbar_wait(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status)) break;
+                    const int s = it % kRing;
+                    const uint32_t ph = (it / kRing) & 1;
+                    // slot s was last used by k-block it - kRing: the pair MMA and the converters are done with it
+                    if (!mbar_wait(smem_u32(&S.done[s]), ph ^ 1, abort, &g_status)) break;
+                    if (!mbar_wait(smem_u32(&S.wread[s]), ph ^ 1, abort, &g_status)) break;
                     mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
-                    tma_load_2d_mc(smem_u32(S.b[s]) + rank * (kBM * 128), &tm_q, smem_u32(&S.full[s]), kb * kBK,
-                                   m0 + (int)rank * kBM, kPair);
+                    tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
                     tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
                 }
             }
             const uint32_t issued = it;
-            for (uint32_t j = issued > (uint32_t)kMcStages ? issued - kMcStages : 0; j < issued; ++j)
-                wait_teardown(smem_u32(&S.full[j % kMcStages]), (j / kMcStages) & 1);
-        } else if (warp == kWarpMma && lane == 0) {
-            const uint32_t idesc = idesc_f16_f32(kBM, kMcBN);
-            const uint32_t d = tmem + kMcAccCol;
+            for (uint32_t j = issued > (uint32_t)kRing ? issued - kRing : 0; j < issued; ++j)
+                wait_teardown(smem_u32(&S.full[j % kRing]), (j / kRing) & 1);
+        } else if (warp == kWarpMma && lane == 0 && rank == 0) {
+            const uint32_t idesc = idesc_f16_f32(2 * kBM, kPairBN);
             uint32_t it = 0, g = 0;
             bool ok = true;
             for (int u = cluster; u < num_units && ok; u += nclusters) {
                 for (int kb0 = 0; kb0 < nkb && ok; kb0 += kcb, ++g) {
-                    if (!(ok = mbar_wait(smem_u32(&S.accempty), (g & 1) ^ 1, abort, &g_status))) break;
+                    const int buf = g & 1;
+                    if (!(ok = mbar_wait(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
                     tc_fence_after();
+                    const uint32_t d = tmem + buf * kPairBN;
                     const int kb1 = min(nkb, kb0 + kcb);
                     for (int kb = kb0; kb < kb1; ++kb, ++it) {
-                        const int s = it % kMcStages;
-                        const uint32_t ph = (it / kMcStages) & 1;
-                        if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
-                        if (!(ok = mbar_wait(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
+                        const int s = it % kRing, sa = it % kAStages;
+                        if (!(ok = mbar_wait(smem_u32(&S.full[s]), (it / kRing) & 1, abort, &g_status))) break;
+                        if (!(ok = mbar_wait(smem_u32(&S.afull[sa]), (it / kAStages) & 1, abort, &g_status))) break;
                         tc_fence_after();
+                        const uint64_t adesc = smem_desc_sw128(smem_u32(S.a[sa]));
                         const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk)
-                            mma_f16_ts(d, tmem + s * 32 + kk * 8, bdesc + (uint64_t)((kk * 32) >> 4), idesc,
-                                       (kb != kb0 || kk != 0) ? 1u : 0u);
-                        mma_commit_mc(smem_u32(&S.empty[s]), kPair);
-                        mma_commit(smem_u32(&S.aempty[s]));
+                            mma_f16_ss_pair(d, adesc + (uint64_t)((kk * 32) >> 4), bdesc + (uint64_t)((kk * 32) >> 4),
+                                            idesc, (kb != kb0 || kk != 0) ? 1u : 0u);
+                        mma_commit_pair_mc(smem_u32(&S.done[s]), kBoth);
                     }
-                    if (ok) mma_commit(smem_u32(&S.accfull));
+                    if (ok) mma_commit_pair_mc(smem_u32(&S.accfull[buf]), kBoth);
                 }
             }
-            mma_commit(smem_u32(&S.drain));
+            mma_commit_pair_mc(smem_u32(&S.drain), 0x1);
             wait_teardown(smem_u32(&S.drain), 0);
         }
     } else if (warp < 8) {
         regs_dec<88>();
-        const int q = warp & 3;
-        const int row = q * 32 + lane;
+        const int row = (warp & 3) * 32 + lane;
         const uint32_t sw64 = (row >> 1) & 3;
-        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        const uint32_t afull0 = mapa_shared(smem_u32(&S.afull[0]), 0);
         uint32_t it = 0;
         bool ok = true;
         for (int u = cluster; u < num_units && ok; u += nclusters) {
             for (int kb = 0; kb < nkb; ++kb, ++it) {
-                const int s = it % kMcStages;
-                const uint32_t ph = (it / kMcStages) & 1;
-                if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
+                const int s = it % kRing, sa = it % kAStages;
+                if (!(ok = mbar_wait(smem_u32(&S.full[s]), (it / kRing) & 1, abort, &g_status))) break;
                 uint4 raw[4];
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
                     raw[c] = *reinterpret_cast<const uint4 *>(S.w[s] + row * 64 + ((c ^ sw64) << 4));
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&S.empty[s]));
-                uint32_t a[32];
+                if (lane == 0) mbar_arrive(smem_u32(&S.wread[s]));
+                uint4 h[8];
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
-                    i8x4_to_f16x4(raw[c].x, a[8 * c + 0], a[8 * c + 1]);
-                    i8x4_to_f16x4(raw[c].y, a[8 * c + 2], a[8 * c + 3]);
-                    i8x4_to_f16x4(raw[c].z, a[8 * c + 4], a[8 * c + 5]);
-                    i8x4_to_f16x4(raw[c].w, a[8 * c + 6], a[8 * c + 7]);
+                    i8x4_to_f16x4(raw[c].x, h[2 * c].x, h[2 * c].y);
+                    i8x4_to_f16x4(raw[c].y, h[2 * c].z, h[2 * c].w);
+                    i8x4_to_f16x4(raw[c].z, h[2 * c + 1].x, h[2 * c + 1].y);
+                    i8x4_to_f16x4(raw[c].w, h[2 * c + 1].z, h[2 * c + 1].w);
                 }
-                if (!(ok = mbar_wait(smem_u32(&S.aempty[s]), ph ^ 1, abort, &g_status))) break;
-                tc_fence_after();
-                tmem_st32(tmem + lane_base + s * 32, a);
-                tmem_wait_st();
-                tc_fence_before();
+                // A tile sa was last read by the MMA of k-block it - kAStages
+                if (it >= (uint32_t)kAStages) {
+                    const uint32_t prev = it - kAStages;
+                    if (!(ok = mbar_wait(smem_u32(&S.done[prev % kRing]), (prev / kRing) & 1, abort, &g_status)))
+                        break;
+                }
+                // row of 64 fp16 = 8 chunks of 16 bytes; 128-byte swizzle puts chunk c at c ^ (row % 8)
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    *reinterpret_cast<uint4 *>(S.a[sa] + row * 128 + ((c ^ (row & 7)) << 4)) = h[c];
+                fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&S.afull[s]));
+                if (lane == 0) mbar_arrive_remote(afull0 + (uint32_t)(sa * sizeof(uint64_t)));
             }
         }
     } else {
@@ -460,18 +478,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const int q = warp & 3;
         const int col0 = (e >> 2) * 128;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        const uint32_t accempty0 = mapa_shared(smem_u32(&S.accempty[0]), 0);
         uint32_t g = 0;
         bool ok = true;
         for (int u = cluster; u < num_units && ok; u += nclusters) {
-            const int m0 = (u % m_tiles) * kMcBN;
+            const int m0 = (u % m_tiles) * kPairBN;
             const int n0 = ((u / m_tiles) * 2 + (int)rank) * kBM;
             int32_t tot[128];
 #pragma unroll
             for (int j = 0; j < 128; ++j) tot[j] = 0;
             for (int kb0 = 0; kb0 < nkb; kb0 += kcb, ++g) {
-                if (!(ok = mbar_wait(smem_u32(&S.accfull), g & 1, abort, &g_status))) break;
+                const int buf = g & 1;
+                if (!(ok = mbar_wait(smem_u32(&S.accfull[buf]), (g >> 1) & 1, abort, &g_status))) break;
                 tc_fence_after();
-                const uint32_t base = tmem + lane_base + kMcAccCol + col0;
+                const uint32_t base = tmem + lane_base + buf * kPairBN + col0;
 #pragma unroll
                 for (int p = 0; p < 4; ++p) {
                     uint32_t v[32];
@@ -482,7 +502,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&S.accempty));
+                if (lane == 0) mbar_arrive_remote(accempty0 + (uint32_t)(buf * sizeof(uint64_t)));
             }
             if (!ok) break;
             const int n = n0 + q * 32 + lane;
@@ -511,10 +531,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
     tc_fence_before();
     __syncthreads();
-    cluster_sync();  // the peer no longer multicasts into this CTA or arrives on its barriers
+    cluster_sync();  // no CTA of the pair touches the other's memory or barriers after this
     if (warp == kWarpAlloc) {
         tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
+        tmem_dealloc_pair(tmem, kTmemCols);
     }
 }
 
@@ -573,19 +593,19 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
 }
 
 template <bool kS32>
-cudaError_t run_linear_mc(const LinearArgs &a, int kcb, cudaStream_t st) {
+cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
     if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
                       (uint64_t)a.K * 2, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
                       kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
         return cudaErrorInvalidValue;
-    const size_t smem = sizeof(SmemMc) + 1024;
+    const size_t smem = sizeof(SmemPair) + 1024;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     static int max_clusters = 0;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_mc_kernel<kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)smem);
         if (attr_err != cudaSuccess) return;
         cudaLaunchConfig_t cfg = {};
@@ -599,15 +619,15 @@ cudaError_t run_linear_mc(const LinearArgs &a, int kcb, cudaStream_t st) {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&max_clusters, linear_mc_kernel<kS32>, &cfg) != cudaSuccess ||
+        if (cudaOccupancyMaxActiveClusters(&max_clusters, linear_pair_kernel<kS32>, &cfg) != cudaSuccess ||
             max_clusters <= 0)
             max_clusters = num_sms() / 2;
         cudaGetLastError();
     });
     if (attr_err != cudaSuccess) return attr_err;
-    const int64_t units = ((a.M + kMcBN - 1) / kMcBN) * ((a.N + 2 * kBM - 1) / (2 * kBM));
+    const int64_t units = ((a.M + kPairBN - 1) / kPairBN) * ((a.N + 2 * kBM - 1) / (2 * kBM));
     const int clusters = (int)(units < max_clusters ? units : max_clusters);
-    linear_mc_kernel<kS32><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
+    linear_pair_kernel<kS32><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
                                                                 (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu);
     return cudaGetLastError();
 }
@@ -618,7 +638,7 @@ cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
     if (a.M <= 32) return run_linear<32, kS32>(a, kcb, st);
     if (a.M <= 64) return run_linear<64, kS32>(a, kcb, st);
     if (a.M <= 128) return run_linear<128, kS32>(a, kcb, st);
-    return run_linear_mc<kS32>(a, kcb, st);
+    return run_linear_pair<kS32>(a, kcb, st);
 }
 
 }  // namespace
