@@ -61,6 +61,23 @@ def _ops_per_step(layers, tokens):
     return sum(2 * tokens * K * N for _, K, N in layers)
 
 
+def max_over_ranks(value: float, device=None) -> float:
+    """Largest `value` over all ranks (the job is as slow as its slowest replica)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(ops_per_rank_step: int, world: int, steps: int, max_ms: float) -> float:
+    """Whole-job throughput in tera-ops/s: every replica runs the full workload
+    (weak scaling), so the units of all ranks divide by the slowest rank's time."""
+    return world * ops_per_rank_step * steps / (max_ms * 1e-3) / 1e12
+
+
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
 
@@ -232,12 +249,9 @@ def run_ours(args):
     total_ms = t0.elapsed_time(t1)
     gemm_ms = [[events[k][i][1].elapsed_time(events[k][i][2]) for k in range(args.steps)] for i in range(nl)]
     quant_ms = [[events[k][i][0].elapsed_time(events[k][i][1]) for k in range(args.steps)] for i in range(nl)]
-    if world > 1:
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(total_ms, dev)
     ms_per_step = total_ms / args.steps
-    value = world * ops_step * args.steps / (total_ms * 1e-3) / 1e12
+    value = job_value(ops_step, world, args.steps, total_ms)
 
     # GEMM roofline (dominant kernel): algorithmic ops / measured launch time
     gemm_ops = [2 * TOKENS * K * N for _, K, N in layer_shapes]

@@ -158,6 +158,17 @@ ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *q
  */
 ot_status ot_get_device_status(void *stream);
 
+/*
+ * ot_selftest_wait_timeout -- exercise the failure path of the bounded device
+ * waits: one GPU thread waits on a barrier that nothing signals, gives up
+ * after limit_ns (1 ms ... 2 s) and records OT_ERR_TIMEOUT in the device
+ * status word, exactly as a stalled GEMM pipeline would; the kernel then
+ * returns normally and the context stays usable.  The paper has no
+ * counterpart; it exists so tests can check ot_get_device_status without
+ * faulting or hanging a GPU.
+ */
+ot_status ot_selftest_wait_timeout(int64_t limit_ns, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -33,6 +33,7 @@ _SIGNATURES = {
     "ot_linear": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P], _I),
     "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P], _I),
     "ot_get_device_status": ([_P], _I),
+    "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
 
 
@@ -173,3 +174,7 @@ def ot_linear_s32(q, qw, bits_a: int, bits_w: int, acc, stream=None):
 
 def ot_get_device_status(stream=None) -> int:
     return load().ot_get_device_status(_stream(stream))
+
+
+def ot_selftest_wait_timeout(limit_ns: int = 50_000_000, stream=None):
+    _check(load().ot_selftest_wait_timeout(int(limit_ns), _stream(stream)), "ot_selftest_wait_timeout")

@@ -120,6 +120,11 @@ ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *q
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
+ot_status ot_selftest_wait_timeout(int64_t limit_ns, void *stream) {
+    if (limit_ns < 1000000 || limit_ns > 2000000000) return OT_ERR_INVALID_ARG;
+    return from_cuda(ot::launch_wait_timeout(limit_ns, as_stream(stream)));
+}
+
 ot_status ot_get_device_status(void *stream) {
     int v = 0;
     if (ot::read_clear_status(&v, as_stream(stream)) != cudaSuccess) return OT_ERR_CUDA;

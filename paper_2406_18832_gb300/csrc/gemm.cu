@@ -664,6 +664,30 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
 
 namespace ot {
 
+namespace {
+// One thread waits, with the given limit, on an mbarrier that nothing
+// arrives on; the expiry takes the same path as the GEMM's bounded waits
+// (OT_ERR_TIMEOUT in the device status word) and the kernel returns.
+__global__ void wait_timeout_kernel(uint64_t limit_ns) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x != 0) return;
+    mbar_init(smem_u32(&bar), 1);
+    fence_barrier_init();
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(smem_u32(&bar), 0)) {
+        if (globaltimer_ns() - t0 > limit_ns) {
+            atomicExch(&g_status, (int)OT_ERR_TIMEOUT);
+            return;
+        }
+    }
+}
+}  // namespace
+
+cudaError_t launch_wait_timeout(int64_t limit_ns, cudaStream_t st) {
+    wait_timeout_kernel<<<1, 32, 0, st>>>((uint64_t)limit_ns);
+    return cudaGetLastError();
+}
+
 cudaError_t read_clear_status(int *value, cudaStream_t st) {
     cudaError_t e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return e;

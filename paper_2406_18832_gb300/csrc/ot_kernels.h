@@ -33,5 +33,6 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
 int num_sms();
 int exact_chunk_kblocks(int bits_a, int bits_w);
 cudaError_t read_clear_status(int *value, cudaStream_t st);
+cudaError_t launch_wait_timeout(int64_t limit_ns, cudaStream_t st);
 
 }  // namespace ot

@@ -1,0 +1,115 @@
+"""The C-ABI library builds, loads and exports every function declared in
+include/outliertune.h; host-side argument validation rejects bad requests
+before anything is launched (no GPU needed for these calls)."""
+import ctypes
+import os
+import re
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "outliertune.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(ot_\w+)\s*\(", text, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2406_18832_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path), path
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for f in ("ot_calibrate", "ot_derive_params", "ot_fold_weights", "ot_quantize_act", "ot_linear",
+              "ot_linear_s32", "ot_get_device_status", "ot_status_string", "ot_version"):
+        assert f in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    handle, path = lib
+    for name in declared_functions():
+        assert hasattr(handle, name), name
+    nm = shutil.which("nm")
+    if nm:
+        out = subprocess.run([nm, "-D", "--defined-only", path], capture_output=True, text=True).stdout
+        exported = {ln.split()[-1] for ln in out.splitlines() if " T " in ln}
+        for name in declared_functions():
+            assert name in exported, name
+
+
+def test_status_strings_and_version(lib):
+    handle, _ = lib
+    handle.ot_status_string.restype = ctypes.c_char_p
+    handle.ot_status_string.argtypes = [ctypes.c_int]
+    assert handle.ot_status_string(0) == b"OT_OK"
+    assert b"TIMEOUT" in handle.ot_status_string(4)
+    assert handle.ot_status_string(99) == b"unknown ot_status"
+    assert handle.ot_version() >= 100
+
+
+def _linear_args(handle):
+    P, I64, I = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+    handle.ot_linear.argtypes = [P, I64, I64, P, P, P, I64, I, I, P, I64, I, P]
+    handle.ot_linear_s32.argtypes = [P, I64, I64, P, I64, I, I, P, P]
+    handle.ot_quantize_act.argtypes = [P, I64, I64, I64, P, P, I, P, I, P]
+    handle.ot_calibrate.argtypes = [P, I64, I64, I64, P, P, I, P]
+    handle.ot_fold_weights.argtypes = [P, P, I, I, P, P, I64, I64, I, P, P, P, P, P, P, P]
+    handle.ot_selftest_wait_timeout.argtypes = [I64, P]
+
+
+# Fake, 256-byte-aligned addresses: every call below must be rejected on the
+# host before any CUDA call, so they are never dereferenced.
+A = 0x10000000
+A2 = A + 0x100000
+
+
+def test_validation_rejects_bad_arguments_before_launch(lib):
+    handle, _ = lib
+    _linear_args(handle)
+    INV, UNS = 1, 2
+    # K not a multiple of 16
+    assert handle.ot_linear(A, 4, 24, A2, A, A, 16, 8, 8, A, 16, 0, None) == INV
+    # bits outside [2, 8]
+    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 9, 8, A, 16, 0, None) == INV
+    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 8, 1, A, 16, 0, None) == INV
+    # misaligned operands
+    assert handle.ot_linear(A + 2, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, None) == INV
+    assert handle.ot_linear(A, 4, 64, A2 + 8, A, A, 16, 8, 8, A, 16, 0, None) == INV
+    # null pointers, ldy < N, negative sizes
+    assert handle.ot_linear(A, 4, 64, None, A, A, 16, 8, 8, A, 16, 0, None) == INV
+    assert handle.ot_linear(A, 4, 64, A2, None, A, 16, 8, 8, A, 16, 0, None) == INV
+    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 8, 8, A, 8, 0, None) == INV
+    assert handle.ot_linear(A, -1, 64, A2, A, A, 16, 8, 8, A, 16, 0, None) == INV
+    # K beyond the int32 accumulator for W8A8 (K * 127 * 127 >= 2^31)
+    assert handle.ot_linear(A, 4, 133152, A2, A, A, 16, 8, 8, A, 16, 0, None) == UNS
+    assert handle.ot_linear_s32(A, 4, 24, A2, 16, 8, 8, A, None) == INV
+    # quantize: bad format, unaligned z, ldx < K
+    assert handle.ot_quantize_act(A, 4, 64, 64, A, A, 8, A2, 7, None) == INV
+    assert handle.ot_quantize_act(A, 4, 64, 64, A + 4, A, 8, A2, 1, None) == INV
+    assert handle.ot_quantize_act(A, 4, 64, 32, A, A, 8, A2, 1, None) == INV
+    # calibrate: K not a multiple of 8
+    assert handle.ot_calibrate(A, 4, 12, 12, A, A, 1, None) == INV
+    # fold: K not a multiple of 16, unaligned weights
+    assert handle.ot_fold_weights(A, A, 8, 1, A, None, 16, 24, 8, A, A, A, A2, A, A, None) == INV
+    assert handle.ot_fold_weights(A, A, 8, 1, A + 2, None, 16, 64, 8, A, A, A, A2, A, A, None) == INV
+    # self-test limit outside [1 ms, 2 s]
+    assert handle.ot_selftest_wait_timeout(10, None) == INV
+
+
+def test_binding_refuses_host_tensors():
+    import torch
+    from paper_2406_18832_gb300 import binding
+    q = torch.zeros(4, 64, dtype=torch.float16)
+    qw = torch.zeros(16, 64, dtype=torch.int8)
+    with pytest.raises((ValueError, RuntimeError)):
+        binding.ot_linear(q, qw, torch.ones(16), torch.zeros(16), 8, 8, torch.empty(4, 16, dtype=torch.float16))
