@@ -643,6 +643,9 @@ cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
 
 }  // namespace
 
+// Token counts up to this go to the mma.sync weight-streaming kernel (gemv.cu).
+constexpr int64_t kGemvMaxTokens = 32;
+
 // Largest number of 64-wide k-blocks whose fp32 partial sums stay exact:
 // kcb * 64 * qmax_a * qmax_w <= 2^24.
 int exact_chunk_kblocks(int bits_a, int bits_w) {
@@ -657,6 +660,7 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
     const int nkb = (int)((a.K + kBK - 1) / kBK);
     int kcb = exact_chunk_kblocks(a.bits_a, a.bits_w);
     if (kcb > nkb) kcb = nkb;
+    if (a.M <= kGemvMaxTokens) return launch_linear_gemv(a, kcb, st);
     return a.out_s32 ? dispatch_bn<true>(a, kcb, st) : dispatch_bn<false>(a, kcb, st);
 }
 

@@ -29,6 +29,8 @@ struct LinearArgs {
     bool out_s32;
 };
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
+// decode-sized token counts (M <= 32); kcb as in launch_linear
+cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st);
 
 int num_sms();
 int exact_chunk_kblocks(int bits_a, int bits_w);
