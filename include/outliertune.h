@@ -31,6 +31,7 @@
 #ifndef OUTLIERTUNE_H
 #define OUTLIERTUNE_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -131,6 +132,14 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  *   qw      int8 [N, K] from ot_fold_weights, |qw| <= qmax(bits_w); 16-byte aligned
  *   sw, b_fold  fp32 [N]
  *   y_f16   fp16 [M, N], row stride ldy >= N
+ *   workspace, workspace_bytes  optional device scratch (16-byte aligned) of
+ *           at least ot_linear_workspace_size() bytes, ZERO-FILLED before its
+ *           first use; the kernel leaves it valid for the next call.  With it,
+ *           prefill-sized calls (M > 128) share the (tile, k-block) work
+ *           evenly over the SMs and exchange exact int32 partial sums through
+ *           it (stream-K); with NULL / too small, whole tiles are dealt out.
+ *           Calls that overlap on the GPU must not share a workspace.  The
+ *           result is bit-identical either way.
  * Exactness: the tensor cores accumulate in fp32, which holds integers
  * exactly up to 2^24; the kernel therefore sums K in chunks short enough
  * that no partial sum can pass 2^24 for the promised bits, and adds the
@@ -139,7 +148,15 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  */
 ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
                     const float *sw, const float *b_fold, int64_t N, int bits_a,
-                    int bits_w, void *y_f16, int64_t ldy, int relu, void *stream);
+                    int bits_w, void *y_f16, int64_t ldy, int relu,
+                    void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * ot_linear_workspace_size -- bytes of scratch that let ot_linear /
+ * ot_linear_s32 balance prefill-sized calls over all SMs on the current
+ * device (about 20 MB on a 152-SM GB300).  Host-only query.
+ */
+ot_status ot_linear_workspace_size(size_t *bytes);
 
 /*
  * ot_linear_s32 -- the same integer product as ot_linear, written out as the
@@ -148,7 +165,7 @@ ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
  */
 ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
                         int64_t N, int bits_a, int bits_w, int32_t *acc,
-                        void *stream);
+                        void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * ot_get_device_status -- synchronize `stream`, then return and clear the

@@ -30,8 +30,9 @@ _SIGNATURES = {
     "ot_derive_params": ([_P, _P, _I64, _I, _I, _P, _P, _P, _P], _I),
     "ot_fold_weights": ([_P, _P, _I, _I, _P, _P, _I64, _I64, _I, _P, _P, _P, _P, _P, _P, _P], _I),
     "ot_quantize_act": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _I, _P], _I),
-    "ot_linear": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P], _I),
-    "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P], _I),
+    "ot_linear": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P], _I),
+    "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P, ctypes.c_size_t, _P], _I),
+    "ot_linear_workspace_size": ([_P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -147,7 +148,41 @@ def ot_quantize_act(x, z, r, bits_a: int, q, q_format: int = OT_CODE_F16, stream
            "ot_quantize_act")
 
 
-def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False, stream=None):
+def ot_linear_workspace_size() -> int:
+    """Bytes of stream-K scratch for prefill-sized linears on the current device."""
+    n = ctypes.c_size_t(0)
+    _check(load().ot_linear_workspace_size(ctypes.byref(n)), "ot_linear_workspace_size")
+    return int(n.value)
+
+
+_workspaces = {}
+
+
+def default_workspace(device=None, stream=None) -> torch.Tensor:
+    """A zero-filled scratch tensor for ot_linear, one per (device, stream): the
+    library allocates nothing itself, and calls that overlap on the GPU must not
+    share a workspace, so each stream gets its own."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    key = (dev.index, _stream(stream))
+    ws = _workspaces.get(key)
+    if ws is None:
+        with torch.cuda.device(dev):
+            ws = torch.zeros(ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+        _workspaces[key] = ws
+    return ws
+
+
+def _ws_args(workspace, device, stream):
+    """(pointer, bytes) for the workspace argument: None picks the per-stream
+    default, False passes none (whole tiles dealt out)."""
+    if workspace is False:
+        return None, 0
+    if workspace is None:
+        workspace = default_workspace(device, stream)
+    return _dev(workspace, "workspace"), workspace.numel() * workspace.element_size()
+
+
+def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False, workspace=None, stream=None):
     _dense(q, "q")
     _dense(qw, "qw")
     M, K = q.shape
@@ -155,20 +190,24 @@ def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False
     ym, yn, ldy = _rows(y, "y")
     if ym != M or yn != N:
         raise ValueError("y must be [M, N]")
-    _check(load().ot_linear(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8),
-                            _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32), N, bits_a,
-                            bits_w, _dev(y, "y", torch.float16), ldy, 1 if relu else 0, _stream(stream)),
+    pq = _dev(q, "q", torch.float16)
+    wp, wb = _ws_args(workspace, q.device, stream)
+    _check(load().ot_linear(pq, M, K, _dev(qw, "qw", torch.int8), _dev(sw, "sw", torch.float32),
+                            _dev(b_fold, "b_fold", torch.float32), N, bits_a, bits_w,
+                            _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb, _stream(stream)),
            "ot_linear")
 
 
-def ot_linear_s32(q, qw, bits_a: int, bits_w: int, acc, stream=None):
+def ot_linear_s32(q, qw, bits_a: int, bits_w: int, acc, workspace=None, stream=None):
     _dense(q, "q")
     _dense(qw, "qw")
     _dense(acc, "acc")
     M, K = q.shape
     N = qw.shape[0]
-    _check(load().ot_linear_s32(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8), N, bits_a,
-                                bits_w, _dev(acc, "acc", torch.int32), _stream(stream)),
+    pq = _dev(q, "q", torch.float16)
+    wp, wb = _ws_args(workspace, q.device, stream)
+    _check(load().ot_linear_s32(pq, M, K, _dev(qw, "qw", torch.int8), N, bits_a, bits_w,
+                                _dev(acc, "acc", torch.int32), wp, wb, _stream(stream)),
            "ot_linear_s32")
 
 

@@ -3,6 +3,7 @@
 // allocates device memory.
 #include <cuda_runtime.h>
 
+#include <cstddef>
 #include <cstdint>
 
 #include "outliertune.h"
@@ -101,22 +102,33 @@ static ot_status linear_common(const void *q_f16, int64_t M, int64_t K, const in
     return OT_OK;
 }
 
+ot_status ot_linear_workspace_size(size_t *bytes) {
+    if (!bytes) return OT_ERR_INVALID_ARG;
+    *bytes = ot::linear_workspace_bytes();
+    return OT_OK;
+}
+
 ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw, const float *b_fold,
-                    int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy, int relu, void *stream) {
+                    int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy, int relu, void *workspace,
+                    size_t workspace_bytes, void *stream) {
     ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
     if (v != OT_OK) return v;
     if (!sw || !b_fold || ldy < N || (y_f16 && !aligned(y_f16, 2))) return OT_ERR_INVALID_ARG;
+    if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
     if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
-    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false};
+    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+                     workspace, workspace ? workspace_bytes : 0};
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
 ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, int64_t N, int bits_a,
-                        int bits_w, int32_t *acc, void *stream) {
+                        int bits_w, int32_t *acc, void *workspace, size_t workspace_bytes, void *stream) {
     ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, acc);
     if (v != OT_OK) return v;
     if (acc && !aligned(acc, 4)) return OT_ERR_INVALID_ARG;
-    ot::LinearArgs a{q_f16, qw, nullptr, nullptr, acc, M, N, K, N, bits_a, bits_w, 0, true};
+    if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
+    ot::LinearArgs a{q_f16, qw, nullptr, nullptr, acc, M, N, K, N, bits_a, bits_w, 0, true,
+                     workspace, workspace ? workspace_bytes : 0};
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 

@@ -30,6 +30,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "ot_common.cuh"
@@ -329,16 +330,82 @@ struct alignas(1024) SmemPair {
     uint64_t afull[kAStages];         // rank 0 only: both CTAs' converters wrote their A tiles (8 warps)
     uint64_t accfull[2];              // pair MMA finished the chunk (rank 0 commit)
     uint64_t accempty[2];             // rank 0 only: both CTAs' epilogues drained the chunk (16 warps)
+    uint64_t pub;                     // stream-K: the 8 epilogue warps stored their partial sums
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
 };
 
+// Work of one CTA pair: a list of pieces (pair tile u, k-blocks [kb0, kb1)).
+// Without a workspace the pieces are whole tiles dealt round-robin.  With a
+// workspace (stream-K) the flattened (tile, k-block) space is cut into equal
+// contiguous ranges, one per pair, so no pair idles in a last partial round;
+// a pair walks its tiles in reverse, so the piece that does not end a tile
+// (its partial int32 sums go to the workspace) comes first and the piece
+// that ends a tile (it adds the partials of the earlier pairs) comes last.
+struct PairSched {
+    int nkb, streamk, count;
+    int first, stride;          // round-robin mode
+    int begin, end, u_last;     // stream-K mode
+    int per, rem;
+
+    __device__ void init(int num_units, int nkb_, int nclusters, int cluster, bool use_streamk) {
+        nkb = nkb_;
+        streamk = use_streamk ? 1 : 0;
+        if (!streamk) {
+            first = cluster;
+            stride = nclusters;
+            count = cluster < num_units ? (num_units - cluster + nclusters - 1) / nclusters : 0;
+            return;
+        }
+        const int total = num_units * nkb;
+        const int active = total < nclusters ? total : nclusters;
+        per = active > 0 ? total / active : 0;
+        rem = active > 0 ? total % active : 0;
+        if (cluster >= active) {
+            count = 0;
+            return;
+        }
+        begin = cluster * per + (cluster < rem ? cluster : rem);
+        end = begin + per + (cluster < rem ? 1 : 0);
+        u_last = (end - 1) / nkb;
+        count = u_last - begin / nkb + 1;
+    }
+    __device__ void piece(int p, int &u, int &kb0, int &kb1) const {
+        if (!streamk) {
+            u = first + p * stride;
+            kb0 = 0;
+            kb1 = nkb;
+            return;
+        }
+        u = u_last - p;
+        kb0 = max(begin, u * nkb) - u * nkb;
+        kb1 = min(end, (u + 1) * nkb) - u * nkb;
+    }
+    // the pair whose range holds flattened k-block x
+    __device__ int owner(int x) const {
+        const int big = rem * (per + 1);
+        return x < big ? x / (per + 1) : rem + (x - big) / per;
+    }
+};
+
+// Stream-K workspace: per pair and CTA rank, 256 token columns x 128 weight
+// rows of int32 partial sums (column-major, so a warp's stores are
+// contiguous), then one 64-bit flag per pair and rank holding the launch
+// epoch once its partials are complete.
+__host__ __device__ constexpr size_t pair_slot_ints() { return (size_t)256 * 128; }
+
+__device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) {
+    uint64_t v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
 template <bool kS32>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
-                       int N, int K, int ldy, int kcb, int relu) {
+                       int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws, uint64_t epoch) {
     extern __shared__ uint8_t smem_raw[];
     SmemPair &S = *reinterpret_cast<SmemPair *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -351,6 +418,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     volatile int *abort = &S.abort;
     constexpr uint32_t kTxBytes = kBM * 128 + kBM * kBK;
     constexpr uint16_t kBoth = 0x3;
+    PairSched sch;
+    sch.init(num_units, nkb, nclusters, cluster, ws != nullptr);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kRing; ++s) {
@@ -363,6 +432,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             mbar_init(smem_u32(&S.accfull[b]), 1);
             mbar_init(smem_u32(&S.accempty[b]), 2 * kNumEpiWarps);
         }
+        mbar_init(smem_u32(&S.pub), kNumEpiWarps);
         mbar_init(smem_u32(&S.drain), 1);
         S.abort = 0;
         fence_barrier_init();
@@ -385,10 +455,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         regs_dec<56>();
         if (warp == kWarpTma && lane == 0) {
             uint32_t it = 0;
-            for (int u = cluster; u < num_units && !*abort; u += nclusters) {
+            for (int p = 0; p < sch.count && !*abort; ++p) {
+                int u, pk0, pk1;
+                sch.piece(p, u, pk0, pk1);
                 const int m0 = (u % m_tiles) * kPairBN + (int)rank * kBM;
                 const int n0 = ((u / m_tiles) * 2 + (int)rank) * kBM;
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                for (int kb = pk0; kb < pk1; ++kb, ++it) {
                     const int s = it % kRing;
                     const uint32_t ph = (it / kRing) & 1;
                     // slot s was last used by k-block it - kRing: the pair MMA and the converters are done with it
@@ -406,13 +478,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const uint32_t idesc = idesc_f16_f32(2 * kBM, kPairBN);
             uint32_t it = 0, g = 0;
             bool ok = true;
-            for (int u = cluster; u < num_units && ok; u += nclusters) {
-                for (int kb0 = 0; kb0 < nkb && ok; kb0 += kcb, ++g) {
+            for (int p = 0; p < sch.count && ok; ++p) {
+                int u, pk0, pk1;
+                sch.piece(p, u, pk0, pk1);
+                for (int kb0 = pk0; kb0 < pk1 && ok; kb0 += kcb, ++g) {
                     const int buf = g & 1;
                     if (!(ok = mbar_wait(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
                     tc_fence_after();
                     const uint32_t d = tmem + buf * kPairBN;
-                    const int kb1 = min(nkb, kb0 + kcb);
+                    const int kb1 = min(pk1, kb0 + kcb);
                     for (int kb = kb0; kb < kb1; ++kb, ++it) {
                         const int s = it % kRing, sa = it % kAStages;
                         if (!(ok = mbar_wait(smem_u32(&S.full[s]), (it / kRing) & 1, abort, &g_status))) break;
@@ -439,8 +513,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const uint32_t afull0 = mapa_shared(smem_u32(&S.afull[0]), 0);
         uint32_t it = 0;
         bool ok = true;
-        for (int u = cluster; u < num_units && ok; u += nclusters) {
-            for (int kb = 0; kb < nkb; ++kb, ++it) {
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
+            for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 const int s = it % kRing, sa = it % kAStages;
                 if (!(ok = mbar_wait(smem_u32(&S.full[s]), (it / kRing) & 1, abort, &g_status))) break;
                 uint4 raw[4];
@@ -481,13 +557,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const uint32_t accempty0 = mapa_shared(smem_u32(&S.accempty[0]), 0);
         uint32_t g = 0;
         bool ok = true;
-        for (int u = cluster; u < num_units && ok; u += nclusters) {
+        const int row = q * 32 + lane;  // weight row of the CTA's 128
+        int32_t *slots = ws;
+        unsigned long long *flags =
+            ws ? reinterpret_cast<unsigned long long *>(ws + (size_t)nclusters * 2 * pair_slot_ints()) : nullptr;
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
             const int m0 = (u % m_tiles) * kPairBN;
             const int n0 = ((u / m_tiles) * 2 + (int)rank) * kBM;
             int32_t tot[128];
 #pragma unroll
             for (int j = 0; j < 128; ++j) tot[j] = 0;
-            for (int kb0 = 0; kb0 < nkb; kb0 += kcb, ++g) {
+            for (int kb0 = pk0; kb0 < pk1; kb0 += kcb, ++g) {
                 const int buf = g & 1;
                 if (!(ok = mbar_wait(smem_u32(&S.accfull[buf]), (g >> 1) & 1, abort, &g_status))) break;
                 tc_fence_after();
@@ -505,6 +587,43 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive_remote(accempty0 + (uint32_t)(buf * sizeof(uint64_t)));
             }
             if (!ok) break;
+            if (pk1 < nkb) {
+                // partial piece: publish the int32 sums for the pair that ends this tile
+                int32_t *slot = slots + ((size_t)cluster * 2 + rank) * pair_slot_ints();
+#pragma unroll
+                for (int j = 0; j < 128; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&S.pub));
+                // a pair has at most one partial piece per launch: phase 0 of pub
+                if (warp == kWarpEpi0 && lane == 0 && mbar_wait(smem_u32(&S.pub), 0, abort, &g_status)) {
+                    __threadfence();
+                    atomicExch(flags + (size_t)cluster * 2 + rank, (unsigned long long)epoch);
+                }
+                continue;
+            }
+            if (pk0 > 0) {
+                // this pair ends the tile: add the partial sums of the pairs that began it
+                const int c_lo = sch.owner(u * nkb);
+                for (int c = c_lo; c < cluster && ok; ++c) {
+                    const unsigned long long *f = flags + (size_t)c * 2 + rank;
+                    const uint64_t t0 = globaltimer_ns();
+                    while (ld_acquire_u64(f) != epoch) {
+                        if (*abort) { ok = false; break; }
+                        if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                            atomicExch(&g_status, (int)OT_ERR_TIMEOUT);
+                            *abort = 1;
+                            ok = false;
+                            break;
+                        }
+                    }
+                    if (!ok) break;
+                    const int32_t *slot = slots + ((size_t)c * 2 + rank) * pair_slot_ints();
+#pragma unroll
+                    for (int j = 0; j < 128; ++j) tot[j] += __ldcg(slot + (size_t)(col0 + j) * 128 + row);
+                }
+                if (!ok) break;
+            }
             const int n = n0 + q * 32 + lane;
             if (n < N) {
                 if constexpr (kS32) {
@@ -541,6 +660,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+// Launch epochs of the stream-K flags: strictly increasing across launches,
+// so a flag left by an earlier launch never matches (workspaces start zeroed).
+uint64_t next_epoch() {
+    static std::atomic<uint64_t> counter{0};
+    return ++counter;
+}
+
+constexpr int64_t kStreamKMinSaving = 32;  // k-blocks per pair
+
+size_t pair_workspace_bytes(int clusters) {
+    return (size_t)clusters * 2 * pair_slot_ints() * sizeof(int32_t) + (size_t)clusters * 2 * sizeof(uint64_t);
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
@@ -592,22 +724,18 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-template <bool kS32>
-cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
-    CUtensorMap tm_q, tm_w;
-    if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
-                      (uint64_t)a.K * 2, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
-                      kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
-        return cudaErrorInvalidValue;
+// Clusters of the pair kernel that fit on the device at once (one per two SMs).
+int pair_max_clusters() {
+    static int dev_cached = -1, value = 0;
+    static std::mutex mu;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    std::lock_guard<std::mutex> lock(mu);
+    if (dev_cached == dev) return value;
     const size_t smem = sizeof(SmemPair) + 1024;
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    static int max_clusters = 0;
-    std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)smem);
-        if (attr_err != cudaSuccess) return;
+    int n = 0;
+    if (cudaFuncSetAttribute(linear_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+        cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 256);
         cfg.blockDim = dim3(kThreads);
@@ -619,16 +747,49 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&max_clusters, linear_pair_kernel<kS32>, &cfg) != cudaSuccess ||
-            max_clusters <= 0)
-            max_clusters = num_sms() / 2;
-        cudaGetLastError();
+        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<false>, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    if (n <= 0) n = num_sms() / 2;
+    dev_cached = dev;
+    value = n;
+    return n;
+}
+
+template <bool kS32>
+cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
+    CUtensorMap tm_q, tm_w;
+    if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
+                      (uint64_t)a.K * 2, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
+                      kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
+        return cudaErrorInvalidValue;
+    const size_t smem = sizeof(SmemPair) + 1024;
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
+    const int max_clusters = pair_max_clusters();
     const int64_t units = ((a.M + kPairBN - 1) / kPairBN) * ((a.N + 2 * kBM - 1) / (2 * kBM));
-    const int clusters = (int)(units < max_clusters ? units : max_clusters);
+    const int64_t nkb = (a.K + kBK - 1) / kBK;
+    // Stream-K shortens the busiest pair's work from ceil(units / pairs) whole
+    // tiles to an equal share of k-blocks, at the cost of a partial-sum
+    // exchange per split tile.  Measured on GB300 it pays off once it saves
+    // about 32 k-blocks per pair (OPT-6.7B QKV and fc2 at 2048 tokens: 7-11 %
+    // faster; out and fc1, which save ~20, are 1-2 % slower).
+    const int64_t whole = (units + max_clusters - 1) / max_clusters * nkb;
+    const int64_t shared = (units * nkb + max_clusters - 1) / max_clusters;
+    const bool streamk = a.workspace != nullptr && a.workspace_bytes >= pair_workspace_bytes(max_clusters) &&
+                         whole - shared >= kStreamKMinSaving && units * nkb < ((int64_t)1 << 30);
+    const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
+    int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
+    const uint64_t epoch = streamk ? next_epoch() : 0;
     linear_pair_kernel<kS32><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
-                                                                (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu);
+                                                                (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
+                                                                epoch);
     return cudaGetLastError();
 }
 
@@ -654,6 +815,8 @@ int exact_chunk_kblocks(int bits_a, int bits_w) {
     kc /= kBK;
     return kc < 1 ? 1 : (int)kc;
 }
+
+size_t linear_workspace_bytes() { return pair_workspace_bytes(pair_max_clusters()); }
 
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
     if (a.M == 0 || a.N == 0) return cudaSuccess;

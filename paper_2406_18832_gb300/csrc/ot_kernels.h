@@ -27,7 +27,11 @@ struct LinearArgs {
     int64_t M, N, K, ldy;
     int bits_a, bits_w, relu;
     bool out_s32;
+    void *workspace;          // stream-K partial sums (zero-filled before first use) or null
+    size_t workspace_bytes;
 };
+// Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
+size_t linear_workspace_bytes();
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
 // decode-sized token counts (M <= 32); kcb as in launch_linear
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st);
