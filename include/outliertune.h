@@ -159,6 +159,31 @@ ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
 ot_status ot_linear_workspace_size(size_t *bytes);
 
 /*
+ * ot_linear_noalloc -- ot_linear for callers that cannot allocate device
+ * memory: for example a server or plugin that owns all GPU memory through
+ * its own pool and forbids further cudaMalloc calls, or code that must not
+ * risk an allocation failing (or synchronizing the device) in the middle of
+ * a run.  The paper has no counterpart.  Same arguments and result as
+ * ot_linear without the workspace: the stream-K scratch it would take is a
+ * fixed 24 MiB array inside the library (a static device array that every
+ * GPU loading the library holds until the process exits).  Nothing here
+ * calls cudaMalloc, cudaFree or any allocating routine.
+ *   - The first call on a device looks up the array's device address and
+ *     zero-fills it on `stream`; make that first call before any stream
+ *     capture.
+ *   - Every call shares the array and it keeps the last call's contents, so
+ *     calls that overlap on the GPU (on different streams, or from several
+ *     threads) race and may corrupt each other's results: serialize them.
+ *   - Returns OT_ERR_UNSUPPORTED if the device would need more scratch than
+ *     the array holds (more than 96 CTA pairs, i.e. more than 192 SMs).
+ */
+ot_status ot_linear_noalloc(const void *q_f16, int64_t M, int64_t K,
+                            const int8_t *qw, const float *sw,
+                            const float *b_fold, int64_t N, int bits_a,
+                            int bits_w, void *y_f16, int64_t ldy, int relu,
+                            void *stream);
+
+/*
  * ot_linear_s32 -- the same integer product as ot_linear, written out as the
  * int32 accumulators acc[m,n] (dense [M, N]) instead of the scaled fp16
  * output; the accumulators of Eq. 6 before external scaling, for checking.

@@ -33,6 +33,7 @@ _SIGNATURES = {
     "ot_linear": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P], _I),
     "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P, ctypes.c_size_t, _P], _I),
     "ot_linear_workspace_size": ([_P], _I),
+    "ot_linear_noalloc": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -196,6 +197,23 @@ def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False
                             _dev(b_fold, "b_fold", torch.float32), N, bits_a, bits_w,
                             _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb, _stream(stream)),
            "ot_linear")
+
+
+def ot_linear_noalloc(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False, stream=None):
+    """ot_linear through the entry point that allocates nothing (its scratch is
+    a fixed array inside the library, shared by every call)."""
+    _dense(q, "q")
+    _dense(qw, "qw")
+    M, K = q.shape
+    N = qw.shape[0]
+    ym, yn, ldy = _rows(y, "y")
+    if ym != M or yn != N:
+        raise ValueError("y must be [M, N]")
+    _check(load().ot_linear_noalloc(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8),
+                                    _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32), N,
+                                    bits_a, bits_w, _dev(y, "y", torch.float16), ldy, 1 if relu else 0,
+                                    _stream(stream)),
+           "ot_linear_noalloc")
 
 
 def ot_linear_s32(q, qw, bits_a: int, bits_w: int, acc, workspace=None, stream=None):

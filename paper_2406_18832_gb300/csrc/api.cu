@@ -121,6 +121,22 @@ ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, c
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
+ot_status ot_linear_noalloc(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw,
+                            const float *b_fold, int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy,
+                            int relu, void *stream) {
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
+    if (v != OT_OK) return v;
+    if (!sw || !b_fold || ldy < N || (y_f16 && !aligned(y_f16, 2))) return OT_ERR_INVALID_ARG;
+    if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
+    // the device's stream-K layout must fit the fixed scratch array
+    if (ot::linear_workspace_bytes() > ot::kNoAllocScratchBytes) return OT_ERR_UNSUPPORTED;
+    void *scratch = nullptr;
+    if (ot::noalloc_scratch(&scratch, as_stream(stream)) != cudaSuccess) return OT_ERR_CUDA;
+    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+                     scratch, ot::kNoAllocScratchBytes};
+    return from_cuda(ot::launch_linear(a, as_stream(stream)));
+}
+
 ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, int64_t N, int bits_a,
                         int bits_w, int32_t *acc, void *workspace, size_t workspace_bytes, void *stream) {
     ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, acc);

@@ -818,6 +818,38 @@ int exact_chunk_kblocks(int bits_a, int bits_w) {
 
 size_t linear_workspace_bytes() { return pair_workspace_bytes(pair_max_clusters()); }
 
+// Scratch of ot_linear_noalloc: the stream-K workspace lives in this
+// file-scope device array, so that entry point never allocates.  Every GPU
+// that loads the library holds it until the process exits.  24 MiB covers
+// the partial-sum slots and flags of up to 96 CTA pairs (a 152-SM GB300 uses
+// 76 pairs, about 20 MB).
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+// Device address of g_noalloc_scratch on the current device.  In host code
+// the array's name is only a stand-in, so the address comes from
+// cudaGetSymbolAddress, once per device, with that device current; the first
+// use on a device also zero-fills the array on `st` (the stream-K flags must
+// start below every launch epoch; later launches leave them below the next).
+cudaError_t noalloc_scratch(void **ptr, cudaStream_t st) {
+    static std::mutex mu;
+    static void *addr[64] = {nullptr};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        e = cudaMemsetAsync(p, 0, kNoAllocScratchBytes, st);
+        if (e != cudaSuccess) return e;
+        addr[dev] = p;
+    }
+    *ptr = addr[dev];
+    return cudaSuccess;
+}
+
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
     if (a.M == 0 || a.N == 0) return cudaSuccess;
     const int nkb = (int)((a.K + kBK - 1) / kBK);

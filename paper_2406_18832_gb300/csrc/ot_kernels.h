@@ -32,6 +32,9 @@ struct LinearArgs {
 };
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();
+// Fixed scratch of ot_linear_noalloc (a static device array in gemm.cu).
+constexpr size_t kNoAllocScratchBytes = (size_t)24 << 20;
+cudaError_t noalloc_scratch(void **ptr, cudaStream_t st);
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
 // decode-sized token counts (M <= 32); kcb as in launch_linear
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st);

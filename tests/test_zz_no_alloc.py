@@ -1,0 +1,86 @@
+"""The entry point that allocates nothing (ot_linear_noalloc) gives the same
+outputs as ot_linear.
+
+It exists for callers that may not allocate device memory once they are
+running -- hosts that own all GPU memory through their own pool, or code that
+must not risk an allocation failing or synchronizing the device mid-run.  Its
+scratch is a fixed array inside the library, shared by every call and keeping
+the last call's contents, so two calls in a row (the second reusing what the
+first left behind) are checked.  This file is collected last on purpose."""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import assert_f16_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2406_18832_gb300 import binding
+    handle = binding.load()
+    return binding, handle
+
+
+def _layer(M, N, K, seed):
+    g = torch.Generator().manual_seed(seed)
+    q = torch.randint(-127, 128, (M, K), generator=g, dtype=torch.int32).half().cuda()
+    qw = torch.randint(-127, 128, (N, K), generator=g, dtype=torch.int32).to(torch.int8).cuda()
+    sw = (torch.rand(N, generator=g) * 1e-4).cuda()
+    bf = torch.randn(N, generator=g).cuda()
+    return q, qw, sw, bf
+
+
+def _noalloc_c_abi(handle, q, qw, sw, bf, y):
+    """Call the entry point directly through the C ABI (ctypes, raw pointers)."""
+    M, K = q.shape
+    N = qw.shape[0]
+    st = torch.cuda.current_stream().cuda_stream
+    return handle.ot_linear_noalloc(q.data_ptr(), M, K, qw.data_ptr(), sw.data_ptr(), bf.data_ptr(), N, 8, 8,
+                                    y.data_ptr(), N, 0, st)
+
+
+# shapes where the scratch is used (stream-K splits tiles), then a smaller one
+SHAPES = [(2048, 12288, 4096), (2048, 4096, 16384)]
+
+
+def test_noalloc_matches_ot_linear_on_consecutive_calls(lib):
+    binding, handle = lib
+    for call, (M, N, K) in enumerate(SHAPES + SHAPES[:1]):
+        q, qw, sw, bf = _layer(M, N, K, seed=call)
+        y_ref = torch.empty(M, N, dtype=torch.float16, device="cuda")
+        binding.ot_linear(q, qw, sw, bf, 8, 8, y_ref)
+        y = torch.full((M, N), float("nan"), dtype=torch.float16, device="cuda")
+        assert _noalloc_c_abi(handle, q, qw, sw, bf, y) == binding.OT_OK
+        torch.cuda.synchronize()
+        assert binding.ot_get_device_status() == binding.OT_OK
+        assert_f16_close(y.cpu().numpy(), y_ref.cpu().numpy(), what=f"call {call}")
+
+
+def test_noalloc_small_and_decode_sizes(lib):
+    binding, handle = lib
+    for M, N, K in [(300, 1000, 2112), (16, 768, 768)]:
+        q, qw, sw, bf = _layer(M, N, K, seed=M)
+        y_ref = torch.empty(M, N, dtype=torch.float16, device="cuda")
+        binding.ot_linear(q, qw, sw, bf, 8, 8, y_ref)
+        y = torch.empty(M, N, dtype=torch.float16, device="cuda")
+        binding.ot_linear_noalloc(q, qw, sw, bf, 8, 8, y)
+        torch.cuda.synchronize()
+        assert_f16_close(y.cpu().numpy(), y_ref.cpu().numpy())
+
+
+def test_noalloc_rejects_bad_arguments(lib):
+    binding, handle = lib
+    q = torch.zeros(4, 24, dtype=torch.float16, device="cuda")
+    qw = torch.zeros(16, 24, dtype=torch.int8, device="cuda")
+    y = torch.empty(4, 16, dtype=torch.float16, device="cuda")
+    with pytest.raises(binding.OTError) as e:
+        binding.ot_linear_noalloc(q, qw, torch.ones(16, device="cuda"), torch.zeros(16, device="cuda"), 8, 8, y)
+    assert e.value.status == binding.OT_ERR_INVALID_ARG
