@@ -338,52 +338,59 @@ struct alignas(1024) SmemPair {
 
 // Work of one CTA pair: a list of pieces (pair tile u, k-blocks [kb0, kb1)).
 // Without a workspace the pieces are whole tiles dealt round-robin.  With a
-// workspace (stream-K) the flattened (tile, k-block) space is cut into equal
-// contiguous ranges, one per pair, so no pair idles in a last partial round;
-// a pair walks its tiles in reverse, so the piece that does not end a tile
-// (its partial int32 sums go to the workspace) comes first and the piece
-// that ends a tile (it adds the partials of the earlier pairs) comes last.
+// workspace (stream-K) all but the last full round of tiles are still dealt
+// whole (neighbouring pairs then share weight and token tiles in L2), and
+// the remaining tiles' flattened (tile, k-block) space is cut into equal
+// contiguous ranges, one per pair, so no pair idles in a last partial round.
+// A pair walks its stream-K tiles in reverse, so the piece that does not end
+// a tile (its partial int32 sums go to the workspace) comes first and the
+// piece that ends a tile (it adds the partials of the earlier pairs) last.
 struct PairSched {
     int nkb, streamk, count;
-    int first, stride;          // round-robin mode
-    int begin, end, u_last;     // stream-K mode
+    int first, stride, dp;      // whole tiles: u = first + p * stride for p < dp
+    int sk0;                    // first stream-K tile
+    int begin, end, u_last;     // this pair's stream-K range (flattened, relative to sk0)
     int per, rem;
 
     __device__ void init(int num_units, int nkb_, int nclusters, int cluster, bool use_streamk) {
         nkb = nkb_;
         streamk = use_streamk ? 1 : 0;
+        first = cluster;
+        stride = nclusters;
         if (!streamk) {
-            first = cluster;
-            stride = nclusters;
-            count = cluster < num_units ? (num_units - cluster + nclusters - 1) / nclusters : 0;
+            dp = cluster < num_units ? (num_units - cluster + nclusters - 1) / nclusters : 0;
+            count = dp;
             return;
         }
-        const int total = num_units * nkb;
+        const int rounds = num_units / nclusters;
+        dp = rounds >= 2 ? rounds - 1 : 0;
+        sk0 = dp * nclusters;
+        const int total = (num_units - sk0) * nkb;
         const int active = total < nclusters ? total : nclusters;
         per = active > 0 ? total / active : 0;
         rem = active > 0 ? total % active : 0;
-        if (cluster >= active) {
-            count = 0;
-            return;
-        }
+        count = dp;
+        if (cluster >= active) return;
         begin = cluster * per + (cluster < rem ? cluster : rem);
         end = begin + per + (cluster < rem ? 1 : 0);
         u_last = (end - 1) / nkb;
-        count = u_last - begin / nkb + 1;
+        count += u_last - begin / nkb + 1;
     }
     __device__ void piece(int p, int &u, int &kb0, int &kb1) const {
-        if (!streamk) {
+        if (p < dp) {
             u = first + p * stride;
             kb0 = 0;
             kb1 = nkb;
             return;
         }
-        u = u_last - p;
-        kb0 = max(begin, u * nkb) - u * nkb;
-        kb1 = min(end, (u + 1) * nkb) - u * nkb;
+        const int v = u_last - (p - dp);  // stream-K tile, relative to sk0
+        u = sk0 + v;
+        kb0 = max(begin, v * nkb) - v * nkb;
+        kb1 = min(end, (v + 1) * nkb) - v * nkb;
     }
-    // the pair whose range holds flattened k-block x
-    __device__ int owner(int x) const {
+    // the first pair whose stream-K range holds part of tile u
+    __device__ int first_owner(int u) const {
+        const int x = (u - sk0) * nkb;
         const int big = rem * (per + 1);
         return x < big ? x / (per + 1) : rem + (x - big) / per;
     }
@@ -604,7 +611,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
             if (pk0 > 0) {
                 // this pair ends the tile: add the partial sums of the pairs that began it
-                const int c_lo = sch.owner(u * nkb);
+                const int c_lo = sch.first_owner(u);
                 for (int c = c_lo; c < cluster && ok; ++c) {
                     const unsigned long long *f = flags + (size_t)c * 2 + rank;
                     const uint64_t t0 = globaltimer_ns();
