@@ -13,7 +13,7 @@ Functions follow the paper's steps in order:
                b' = b + z W^T (Eq. 7)
   quantize   - round((X - z) / s) (Eq. 6, Eq. 7)
   matmul     - sum_k q[m,k] qw[n,k] in int64 (Eq. 6)
-  epilogue   - acc * sw + b' rounded to fp16 (Eq. 6, Eq. 7)
+  epilogue   - fp16(fma((float)acc, sw, b')) (Eq. 6, Eq. 7)
 """
 from __future__ import annotations
 
@@ -157,7 +157,7 @@ def matmul(q: np.ndarray, qw: np.ndarray) -> np.ndarray:
 
 
 def epilogue(acc: np.ndarray, sw: np.ndarray, bfold: np.ndarray, relu: bool = False) -> np.ndarray:
-    """fp16 Y[M, N] = fp16(acc * sw + b'), optional ReLU."""
+    """fp16 Y[M, N] = fp16(fma((float)acc, sw, b')), optional ReLU."""
     acc = np.ascontiguousarray(acc, dtype=np.int64)
     M, N = acc.shape
     y = np.empty((M, N), np.uint16)

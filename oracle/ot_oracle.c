@@ -34,8 +34,11 @@
  *   R6 non-finite NaN codes to 0; +-inf saturates to +-qmax.  Calibration
  *                ignores NaN.
  *   R7 bias      b' is formed in fp64 (k ascending) and rounded once to fp32.
- *   R8 epilogue  y = acc * sw + b' evaluated in fp64, rounded once to fp16
- *                (round-half-to-even, overflow to +-inf); optional ReLU.
+ *   R8 epilogue  y = fp16( fma((float)acc, sw, b') ): the accumulator is
+ *                rounded to fp32, the external scaling and bias take one
+ *                fp32 fused multiply-add (one rounding), the result is
+ *                rounded once to fp16 (half to even, overflow to +-inf);
+ *                optional ReLU before the fp16 rounding.
  *
  * Floating point: compile with -ffp-contract=off and no fast-math, so every
  * fp32 expression below rounds once per operation as written.
@@ -238,16 +241,17 @@ void oracle_matmul(const int8_t *q, const int8_t *qw, int64_t M, int64_t N,
 
 /* ---------------------------------------------------------------------------
  * Step 6: external scaling (Eq. 6) plus the folded bias (Eq. 7), R8:
- *   y[m,n] = fp16( acc[m,n] * sw_n + b'_n ),  ReLU applied before rounding
- * when relu != 0.  y holds binary16 bit patterns.
+ *   y[m,n] = fp16( fma((float)acc[m,n], sw_n, b'_n) ),  ReLU applied before
+ * the fp16 rounding when relu != 0.  y holds binary16 bit patterns.
  * ------------------------------------------------------------------------- */
 void oracle_epilogue(const int64_t *acc, int64_t M, int64_t N, const float *sw,
                      const float *bfold, int relu, uint16_t *y)
 {
     for (int64_t m = 0; m < M; ++m)
         for (int64_t n = 0; n < N; ++n) {
-            double v = (double)acc[m * N + n] * (double)sw[n] + (double)bfold[n];
-            if (relu && !(v > 0.0)) v = 0.0;
-            y[m * N + n] = ot_double_to_half(v);
+            float a = (float)acc[m * N + n];       /* round to nearest even */
+            float v = fmaf(a, sw[n], bfold[n]);    /* one rounding */
+            if (relu && !(v > 0.0f)) v = 0.0f;
+            y[m * N + n] = ot_double_to_half((double)v);
         }
 }

@@ -6,6 +6,6 @@ behind the C ABI of include/outliertune.h.
 The CUDA library is loaded on first use (``binding.load()``); importing the
 package does not need a GPU.
 """
-from .layer import QuantizedLinear  # noqa: F401
+from .layer import QuantizedBlockLinears, QuantizedLinear  # noqa: F401
 
-__all__ = ["QuantizedLinear"]
+__all__ = ["QuantizedLinear", "QuantizedBlockLinears"]

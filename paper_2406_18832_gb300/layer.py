@@ -82,3 +82,51 @@ class QuantizedLinear:
 
     def weight_bytes(self) -> int:
         return self.qw.numel() + 4 * (self.sw.numel() + self.b_fold.numel())
+
+
+class QuantizedBlockLinears:
+    """The linear path of one OPT-style decoder block, every layer per-channel
+    quantized with its own calibration (the paper applies the method to the
+    linears after LayerNorm and keeps residual / LayerNorm / attention in
+    fp16; those are not part of this path):
+
+        qkv = QKV(x);  v = qkv[:, 2h:3h]   (stand-in for attention: its V slice)
+        o   = out(v);  f = ReLU(fc1(o));   y = fc2(f)
+
+    calibrate() runs the calibration tokens through the already-folded
+    layers, so each layer is calibrated on the activations it receives.
+    """
+
+    def __init__(self, hidden: int, ffn: int, bits_a: int = 8, bits_w: int = 8, device="cuda"):
+        self.h, self.ffn = hidden, ffn
+        mk = lambda K, N, relu=False: QuantizedLinear(K, N, bits_a, bits_w, relu=relu, device=device)
+        self.qkv = mk(hidden, 3 * hidden)
+        self.out = mk(hidden, hidden)
+        self.fc1 = mk(hidden, ffn, relu=True)
+        self.fc2 = mk(ffn, hidden)
+        self.layers = (self.qkv, self.out, self.fc1, self.fc2)
+
+    def calibrate(self, x_cal: torch.Tensor, weights, batch: int = 8192, stream=None):
+        """weights: [(w, b)] for qkv, out, fc1, fc2 (fp16, [N, K] and [N])."""
+        acts = x_cal
+        for i, (ql, (w, b)) in enumerate(zip(self.layers, weights)):
+            for t0 in range(0, acts.shape[0], batch):
+                ql.calibrate(acts[t0:t0 + batch], stream=stream)
+            ql.fold(w, b, stream=stream)
+            if i + 1 < len(self.layers):
+                nxt = torch.empty(acts.shape[0], ql.N, dtype=torch.float16, device=acts.device)
+                for t0 in range(0, acts.shape[0], batch):
+                    ql.forward(acts[t0:t0 + batch], out=nxt[t0:t0 + batch], stream=stream)
+                acts = nxt[:, 2 * self.h:] if ql is self.qkv else nxt
+        return self
+
+    def forward(self, x: torch.Tensor, stream=None):
+        """All intermediate outputs: qkv, o, f, y (fp16)."""
+        qkv = self.qkv(x, stream=stream)
+        o = self.out(qkv[:, 2 * self.h:], stream=stream)
+        f = self.fc1(o, stream=stream)
+        y = self.fc2(f, stream=stream)
+        return dict(qkv=qkv, o=o, f=f, y=y)
+
+    def weight_bytes(self) -> int:
+        return sum(ql.weight_bytes() for ql in self.layers)

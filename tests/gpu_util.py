@@ -89,3 +89,5 @@ def compare_layer(g, o, rows=None, cols=None):
     if acc_g is not None:
         assert np.array_equal(acc_g.astype(np.int64), o["acc"]), "int32 accumulators"
     assert_f16_close(y_g, o["y"])
+    # the epilogue is one fp32 fma rounded to fp16 on both sides: bit-identical
+    assert np.array_equal(np.asarray(y_g, np.float32), np.asarray(o["y"], np.float32)), "fp16 outputs"

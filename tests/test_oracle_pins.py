@@ -280,20 +280,44 @@ def test_matmul_matches_numpy_and_extremes():
     assert acc[0, 0] == 127 * 127 * K and acc[1, 0] == -127 * 127 * K
 
 
+def frac_to_f32(v: Fraction) -> Fraction:
+    """Round a rational to binary32, half to even (finite range only)."""
+    if v == 0:
+        return Fraction(0)
+    a = abs(v)
+    e = math.floor(math.log2(a.numerator) - math.log2(a.denominator))
+    while Fraction(2) ** e > a:
+        e -= 1
+    while Fraction(2) ** (e + 1) <= a:
+        e += 1
+    q = max(e, -126) - 23
+    r = Fraction(round(a / Fraction(2) ** q)) * Fraction(2) ** q
+    return -r if v < 0 else r
+
+
 def test_epilogue_exact_rounding():
+    """fp16(fma((float)acc, sw, b')): acc rounded to fp32, one exact fused
+    multiply-add rounded to fp32, then one rounding to fp16 (all written out
+    with rationals)."""
     rng = np.random.default_rng(8)
     acc = rng.integers(-2 ** 31, 2 ** 31, (7, 13)).astype(np.int64)
     acc[0, :3] = [0, 1, -1]
+    acc[1, :3] = [2 ** 24 + 1, -(2 ** 24 + 3), 2 ** 30 + 7]   # need rounding to fp32
     sw = (rng.standard_normal(13) * 1e-6).astype(np.float32)
     bf = (rng.standard_normal(13) * 3).astype(np.float32)
     y = oracle.epilogue(acc, sw, bf).astype(np.float64)
     yr = oracle.epilogue(acc, sw, bf, relu=True).astype(np.float64)
     for m in range(7):
         for n in range(13):
-            v = Fraction(int(acc[m, n])) * Fraction(float(sw[n])) + Fraction(float(bf[n]))
+            a = frac_to_f32(Fraction(int(acc[m, n])))
+            v = frac_to_f32(a * Fraction(float(sw[n])) + Fraction(float(bf[n])))
             e = frac_to_half(v)
             assert y[m, n] == e or (math.isinf(e) and y[m, n] == e)
             assert yr[m, n] == (e if e > 0 else 0.0)
+    # and within half an fp16 ulp (plus the fp32 steps) of the exact value
+    exact = acc.astype(np.float64) * sw.astype(np.float64) + bf.astype(np.float64)
+    ulp16 = np.spacing(np.abs(exact).astype(np.float16)).astype(np.float64)
+    assert np.all(np.abs(y - exact) <= ulp16 * 0.5 + np.abs(exact) * 2.0 ** -22)
 
 
 # ----------------------------------------------------------------------------
