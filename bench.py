@@ -337,6 +337,8 @@ def run_ours(args):
     h2d = sum(x.numel() * 2 for x in xs)
     d2h = sum(y.numel() * 2 for y in ybufs)
 
+    block = None if args.no_block else bench_block(dev)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(budget_s=args.cpu_budget, layers=layers)
@@ -376,12 +378,69 @@ def run_ours(args):
         "per_layer": per_layer,
         "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
                    "ratio": round(weights_fp16 / weights_int8, 3)},
+        "block": block,
         "cpu_baseline": cpu,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):
+    """The chained linear path of an OPT-30B-shaped decoder block (hidden 7168,
+    FFN 28672; QKV -> V slice -> out -> fc1 + ReLU -> fc2, each layer calibrated
+    on what it receives) at 8 x 512 tokens, Int8 and Int6: latency, weight and
+    activation bytes against the same chain of cuBLAS fp16 GEMMs."""
+    import torch
+
+    from paper_2406_18832_gb300 import QuantizedBlockLinears, synth
+    c = synth.CONFIGS[5]
+    h, ffn = 7168, 28672
+    weights = [synth.weights(5, i, layer, device=dev) for i, layer in enumerate(c.layers)]
+    x_cal = synth.activations(5, 0, c.layers[0], t_cal, 3, device=dev)
+    x = synth.activations(5, 0, c.layers[0], tokens, 4, device=dev)
+    ops = 2 * tokens * sum(l.K * l.N for l in c.layers)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    out = {"workload": "opt-30b-block-linears", "tokens": tokens, "calibration_tokens": t_cal,
+           "ops": ops, "reps": reps}
+    for bits in (8, 6):
+        blk = QuantizedBlockLinears(h, ffn, bits, bits, device=dev)
+        blk.calibrate(x_cal, weights)
+        ms = timed(lambda: blk.forward(x))
+        out[f"int{bits}"] = {"ms": round(ms, 4), "tops": round(ops / (ms * 1e-3) / 1e12, 1),
+                             "weight_bytes": blk.weight_bytes()}
+        del blk
+    w16 = [w for w, _ in weights]
+    b16 = [b for _, b in weights]
+
+    def fp16_chain():
+        qkv = torch.addmm(b16[0], x, w16[0].t())
+        o = torch.addmm(b16[1], qkv[:, 2 * h:], w16[1].t())
+        f = torch.relu(torch.addmm(b16[2], o, w16[2].t()))
+        return torch.addmm(b16[3], f, w16[3].t())
+    ms16 = timed(fp16_chain)
+    out["cublas_fp16"] = {"ms": round(ms16, 4), "tflops": round(ops / (ms16 * 1e-3) / 1e12, 1),
+                          "weight_bytes": sum(w.numel() * 2 + b.numel() * 2 for w, b in weights)}
+    # activation bytes per block: fp16 inputs read (x, v, o, f) and outputs written
+    # (qkv, o, f, y); the quantized path also writes and reads each layer's fp16 codes
+    act16 = 2 * tokens * ((h + h + h + ffn) + (3 * h + h + ffn + h))
+    out["activation_bytes"] = {"fp16_path": act16, "quantized_path": act16 + 4 * tokens * (h + h + h + ffn)}
+    del weights, x_cal, x
+    torch.cuda.empty_cache()
+    return out
 
 
 # ----------------------------------------------------------------------------
@@ -457,7 +516,7 @@ def run_reference(args):
     dt = time.perf_counter() - t
     value = ops / dt / 1e12
     sample = (f"per step: 1 token through all four layers, first {cols} output channels of each "
-              f"(quantize, int64 product, fp64 epilogue)")
+              f"(quantize, int64 product, fp32-fma epilogue)")
     line = {"metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64 (CPU oracle)", "data": "synthetic",
@@ -478,6 +537,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-block", action="store_true", help="skip the OPT-30B block stage")
     ap.add_argument("--profile", action="store_true",
                     help="profiler run: 8192 calibration tokens, the timed steps only, no report")
     args = ap.parse_args()
