@@ -491,7 +491,7 @@ def cpu_baseline(budget_s=12.0, layers=None):
     dt = time.perf_counter() - t
     return {"value": round(ops / dt / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
             "sample": f"{rows} token(s) of the 2048 through all four layers (quantize, int64 product, "
-                      f"fp64 epilogue), every output channel; {dt:.1f} s",
+                      f"fp32-fma epilogue), every output channel; {dt:.1f} s",
             "host_cores_available": len(os.sched_getaffinity(0))}
 
 
