@@ -159,6 +159,47 @@ ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
 ot_status ot_linear_workspace_size(size_t *bytes);
 
 /*
+ * Per-token path (Eq. 3).  The paper quantizes the out and fc2 linears, whose
+ * inputs carry no outlier channels, per token instead of per channel, and
+ * carries the residual stream's symmetrization shift z in their bias (Eq. 8:
+ * pass b + z as `bias`).
+ *
+ * ot_quantize_tokens -- dynamic symmetric quantization per token (Eq. 1 with
+ * zero point 0, one scale per row):
+ *   s_m = max_k |x[m,k]| / qmax_a,  q[m,k] = round_half_even(x[m,k] * qmax_a / max_k |x[m,k]|)
+ * in fp32 (the reciprocal computed once per row); NaN is ignored by the max
+ * and codes to 0; a row whose max is 0 or not finite gets s_m = 0, codes 0.
+ *   x_f16  fp16 [M, K], row stride ldx (16-byte aligned; K, ldx % 8 == 0)
+ *   q      [M, K] dense, int8 or fp16 codes (ot_code_format); 16-byte aligned
+ *   s_tok  fp32 [M] out
+ */
+ot_status ot_quantize_tokens(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
+                             int bits_a, void *q, int q_format, float *s_tok,
+                             void *stream);
+
+/*
+ * ot_quantize_weights -- per-output-channel symmetric weight codes with no
+ * activation scale folded in (Eq. 3's W~):
+ *   sw_n = max_k |W[n,k]| / qmax_w,  qw[n,k] = round(W[n,k] * qmax_w / max_k |W[n,k]|)
+ *   w_f16 fp16 [N, K] (16-byte aligned, K % 16 == 0); qw int8 [N, K]; sw fp32 [N].
+ */
+ot_status ot_quantize_weights(const void *w_f16, int64_t N, int64_t K, int bits_w,
+                              int8_t *qw, float *sw, void *stream);
+
+/*
+ * ot_linear_per_token -- Eq. 3 with the bias:
+ *   y[m,n] = fp16( fma((float)acc[m,n], s_tok[m] * sw[n], bias[n]) ), ReLU if relu
+ * with acc the exact integer product as in ot_linear; s_tok[m] * sw[n] is one
+ * fp32 product.  Arguments as ot_linear plus s_tok fp32 [M] (from
+ * ot_quantize_tokens) and bias fp32 [N] (b, or b + z for Eq. 8).
+ */
+ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
+                              const float *sw, const float *s_tok, const float *bias,
+                              int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy,
+                              int relu, void *workspace, size_t workspace_bytes,
+                              void *stream);
+
+/*
  * ot_linear_noalloc -- ot_linear for callers that cannot allocate device
  * memory: for example a server or plugin that owns all GPU memory through
  * its own pool and forbids further cudaMalloc calls, or code that must not

@@ -14,6 +14,10 @@ Functions follow the paper's steps in order:
   quantize   - round((X - z) / s) (Eq. 6, Eq. 7)
   matmul     - sum_k q[m,k] qw[n,k] in int64 (Eq. 6)
   epilogue   - fp16(fma((float)acc, sw, b')) (Eq. 6, Eq. 7)
+and the per-token path of Eq. 3 (the paper's out / fc2 linears):
+  quantize_tokens   - dynamic per-token scale s_m = max|x[m,:]| / qmax and codes
+  quantize_weights  - per-output-channel codes of W without activation scales
+  epilogue_tokens   - fp16(fma((float)acc, s_m * sw_n, b_n))
 """
 from __future__ import annotations
 
@@ -61,8 +65,10 @@ def _load():
             lib.oracle_quantize.argtypes = [P, I64, I64, I64, P, P, I, P]
             lib.oracle_matmul.argtypes = [P, P, I64, I64, I64, P]
             lib.oracle_epilogue.argtypes = [P, I64, I64, P, P, I, P]
+            lib.oracle_quantize_tokens.argtypes = [P, I64, I64, I64, I, P, P]
+            lib.oracle_epilogue_tokens.argtypes = [P, I64, I64, P, P, P, I, P]
             for f in ("oracle_calibrate", "oracle_params", "oracle_fold", "oracle_quantize",
-                      "oracle_matmul", "oracle_epilogue"):
+                      "oracle_matmul", "oracle_epilogue", "oracle_quantize_tokens", "oracle_epilogue_tokens"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -171,3 +177,32 @@ def linear(x: np.ndarray, qw: np.ndarray, sw: np.ndarray, bfold: np.ndarray, z: 
     q = quantize(x, z, r, bits_a)
     acc = matmul(q, qw)
     return q, acc, epilogue(acc, sw, bfold, relu)
+
+
+def quantize_tokens(x: np.ndarray, bits_a: int):
+    """(int8 codes [M, K], fp32 per-token scales [M]) of fp16 X (Eq. 3, Eq. 1 with z = 0)."""
+    x = _f16(x)
+    M, K = x.shape
+    q = np.empty((M, K), np.int8)
+    s = np.empty(M, np.float32)
+    _load().oracle_quantize_tokens(_ptr(x), M, K, K, bits_a, _ptr(q), _ptr(s))
+    return q, s
+
+
+def quantize_weights(w: np.ndarray, bits_w: int):
+    """(qw int8 [N, K], sw fp32 [N]): per-output-channel symmetric codes of W
+    with no activation scale folded in (Eq. 3's W~): the fold with s = 1, z = 0."""
+    w = _f16(w)
+    K = w.shape[1]
+    qw, sw, _ = fold(w, None, np.zeros(K, np.float32), np.ones(K, np.float32), bits_w)
+    return qw, sw
+
+
+def epilogue_tokens(acc: np.ndarray, s_tok: np.ndarray, sw: np.ndarray, bias: np.ndarray, relu: bool = False):
+    """fp16 Y[M, N] = fp16(fma((float)acc, s_m * sw_n, b_n)), optional ReLU."""
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
+    M, N = acc.shape
+    y = np.empty((M, N), np.uint16)
+    _load().oracle_epilogue_tokens(_ptr(acc), M, N, _ptr(_f32(s_tok)), _ptr(_f32(sw)), _ptr(_f32(bias)),
+                                   1 if relu else 0, _ptr(y))
+    return y.view(np.float16)

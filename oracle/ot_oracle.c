@@ -255,3 +255,56 @@ void oracle_epilogue(const int64_t *acc, int64_t M, int64_t N, const float *sw,
             y[m * N + n] = ot_double_to_half((double)v);
         }
 }
+
+/* ---------------------------------------------------------------------------
+ * Per-token path (Eq. 3; used by the paper for the out and fc2 linears,
+ * whose inputs carry no outlier channels, with Eq. 8 folding the residual
+ * stream's symmetrization shift into their bias).
+ *
+ * Step T1: dynamic symmetric quantization per token (Eq. 1 with z = 0, one
+ * scale per row of X):
+ *   amax_m = max_k |x[m,k]|  (NaN ignored),
+ *   s_m = amax_m / qmax, r_m = qmax / amax_m  (fp32; both 0 when amax_m is 0
+ *   or not finite), q[m,k] = round_half_even(x[m,k] * r_m) in [-qmax, qmax].
+ * ------------------------------------------------------------------------- */
+void oracle_quantize_tokens(const uint16_t *x, int64_t M, int64_t K, int64_t ldx,
+                            int bits, int8_t *q, float *s_tok)
+{
+    const int qmax = qmax_of(bits);
+    for (int64_t m = 0; m < M; ++m) {
+        float amax = 0.0f;
+        for (int64_t k = 0; k < K; ++k) {
+            float a = fabsf(ot_half_to_float(x[m * ldx + k]));
+            if (a > amax) amax = a;          /* NaN compares false: ignored */
+        }
+        float s = 0.0f, r = 0.0f;
+        if (amax > 0.0f && isfinite(amax)) {
+            s = amax / (float)qmax;
+            r = (float)qmax / amax;
+        }
+        s_tok[m] = s;
+        for (int64_t k = 0; k < K; ++k)
+            q[m * K + k] = (int8_t)quantize_code(ot_half_to_float(x[m * ldx + k]) * r, qmax);
+    }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step T3: external scaling of Eq. 3 by the token scale and the output-channel
+ * scale, plus the bias:
+ *   y[m,n] = fp16( fma((float)acc[m,n], s_m * sw_n, b_n) )
+ * where s_m * sw_n is one fp32 product; ReLU before the fp16 rounding.
+ * (The weights of this path are quantized per output channel without any
+ * activation scale: oracle_fold with s = 1, z = 0.)
+ * ------------------------------------------------------------------------- */
+void oracle_epilogue_tokens(const int64_t *acc, int64_t M, int64_t N, const float *s_tok,
+                            const float *sw, const float *bias, int relu, uint16_t *y)
+{
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t n = 0; n < N; ++n) {
+            float a = (float)acc[m * N + n];
+            float scale = s_tok[m] * sw[n];
+            float v = fmaf(a, scale, bias[n]);
+            if (relu && !(v > 0.0f)) v = 0.0f;
+            y[m * N + n] = ot_double_to_half((double)v);
+        }
+}

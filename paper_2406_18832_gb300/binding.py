@@ -34,6 +34,10 @@ _SIGNATURES = {
     "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P, ctypes.c_size_t, _P], _I),
     "ot_linear_workspace_size": ([_P], _I),
     "ot_linear_noalloc": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P], _I),
+    "ot_quantize_tokens": ([_P, _I64, _I64, _I64, _I, _P, _I, _P, _P], _I),
+    "ot_quantize_weights": ([_P, _I64, _I64, _I, _P, _P, _P], _I),
+    "ot_linear_per_token": ([_P, _I64, _I64, _P, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P],
+                            _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -197,6 +201,43 @@ def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False
                             _dev(b_fold, "b_fold", torch.float32), N, bits_a, bits_w,
                             _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb, _stream(stream)),
            "ot_linear")
+
+
+def ot_quantize_tokens(x, bits_a: int, q, s_tok, q_format: int = OT_CODE_F16, stream=None):
+    """Per-token dynamic codes and scales of fp16 X[M, K] (Eq. 3)."""
+    M, K, ldx = _rows(x, "x")
+    _dense(q, "q")
+    want = torch.float16 if q_format == OT_CODE_F16 else torch.int8
+    _check(load().ot_quantize_tokens(_dev(x, "x", torch.float16), M, K, ldx, bits_a, _dev(q, "q", want), q_format,
+                                     _dev(s_tok, "s_tok", torch.float32), _stream(stream)),
+           "ot_quantize_tokens")
+
+
+def ot_quantize_weights(w, bits_w: int, qw, sw, stream=None):
+    """Per-output-channel weight codes without activation scales (Eq. 3's W~)."""
+    _dense(w, "w")
+    N, K = w.shape
+    _check(load().ot_quantize_weights(_dev(w, "w", torch.float16), N, K, bits_w, _dev(qw, "qw", torch.int8),
+                                      _dev(sw, "sw", torch.float32), _stream(stream)),
+           "ot_quantize_weights")
+
+
+def ot_linear_per_token(q, qw, sw, s_tok, bias, bits_a: int, bits_w: int, y, relu: bool = False, workspace=None,
+                        stream=None):
+    _dense(q, "q")
+    _dense(qw, "qw")
+    M, K = q.shape
+    N = qw.shape[0]
+    ym, yn, ldy = _rows(y, "y")
+    if ym != M or yn != N:
+        raise ValueError("y must be [M, N]")
+    pq = _dev(q, "q", torch.float16)
+    wp, wb = _ws_args(workspace, q.device, stream)
+    _check(load().ot_linear_per_token(pq, M, K, _dev(qw, "qw", torch.int8), _dev(sw, "sw", torch.float32),
+                                      _dev(s_tok, "s_tok", torch.float32), _dev(bias, "bias", torch.float32), N,
+                                      bits_a, bits_w, _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb,
+                                      _stream(stream)),
+           "ot_linear_per_token")
 
 
 def ot_linear_noalloc(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False, stream=None):

@@ -91,6 +91,23 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx, 
     return from_cuda(ot::launch_quantize(x_f16, M, K, ldx, z, r, bits_a, q, q_format, as_stream(stream)));
 }
 
+ot_status ot_quantize_tokens(const void *x_f16, int64_t M, int64_t K, int64_t ldx, int bits_a, void *q,
+                             int q_format, float *s_tok, void *stream) {
+    if (M < 0 || K <= 0 || K % 8 != 0 || ldx < K || ldx % 8 != 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;
+    if (q_format != OT_CODE_I8 && q_format != OT_CODE_F16) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!x_f16 || !q || !s_tok || !aligned(x_f16, 16) || !aligned(q, 16) || !aligned(s_tok, 4)))
+        return OT_ERR_INVALID_ARG;
+    if (M > kIntMax) return OT_ERR_UNSUPPORTED;
+    return from_cuda(ot::launch_quantize_tokens(x_f16, M, K, ldx, bits_a, q, q_format, s_tok, as_stream(stream)));
+}
+
+ot_status ot_quantize_weights(const void *w_f16, int64_t N, int64_t K, int bits_w, int8_t *qw, float *sw,
+                              void *stream) {
+    if (N < 0 || K <= 0 || K % 16 != 0 || !bits_ok(bits_w)) return OT_ERR_INVALID_ARG;
+    if (N > 0 && (!w_f16 || !qw || !sw || !aligned(w_f16, 16) || !aligned(qw, 16))) return OT_ERR_INVALID_ARG;
+    return from_cuda(ot::launch_quantize_weights(w_f16, N, K, bits_w, qw, sw, as_stream(stream)));
+}
+
 static ot_status linear_common(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, int64_t N, int bits_a,
                                int bits_w, const void *out) {
     if (M < 0 || N <= 0 || K <= 0 || K % 16 != 0 || !bits_ok(bits_a) || !bits_ok(bits_w))
@@ -118,6 +135,20 @@ ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, c
     if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
     ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
                      workspace, workspace ? workspace_bytes : 0};
+    return from_cuda(ot::launch_linear(a, as_stream(stream)));
+}
+
+ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw,
+                              const float *s_tok, const float *bias, int64_t N, int bits_a, int bits_w, void *y_f16,
+                              int64_t ldy, int relu, void *workspace, size_t workspace_bytes, void *stream) {
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
+    if (v != OT_OK) return v;
+    if (!sw || !bias || ldy < N || (y_f16 && !aligned(y_f16, 2))) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!s_tok || !aligned(s_tok, 4))) return OT_ERR_INVALID_ARG;
+    if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
+    if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
+    ot::LinearArgs a{q_f16, qw, sw, bias, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+                     workspace, workspace ? workspace_bytes : 0, s_tok};
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 

@@ -13,7 +13,8 @@ namespace {
 constexpr int kFoldThreads = 256;
 
 // One CTA per output row n (grid-stride): amax_n = max_k |W[n,k] * s_k|, then
-// sw_n, rw_n and the codes round(W[n,k] * s_k * rw_n).  Each thread handles
+// sw_n, rw_n and the codes round(W[n,k] * s_k * rw_n).  s == null means s_k = 1
+// (per-output-channel weight codes without activation scales, Eq. 3's W~).  Each thread handles
 // 8 consecutive k per step (16-byte loads of W, 8-byte stores of codes).
 __global__ void __launch_bounds__(kFoldThreads) fold_codes_kernel(const __half *__restrict__ w, int64_t N,
                                                                   int64_t K, const float *__restrict__ s,
@@ -29,8 +30,8 @@ __global__ void __launch_bounds__(kFoldThreads) fold_codes_kernel(const __half *
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const float2 f = __half22float2(h[j]);
-                amax = fmaxf(amax, fabsf(__fmul_rn(f.x, __ldg(s + k + 2 * j))));
-                amax = fmaxf(amax, fabsf(__fmul_rn(f.y, __ldg(s + k + 2 * j + 1))));
+                amax = fmaxf(amax, fabsf(__fmul_rn(f.x, (s ? __ldg(s + k + 2 * j) : 1.0f))));
+                amax = fmaxf(amax, fabsf(__fmul_rn(f.y, (s ? __ldg(s + k + 2 * j + 1) : 1.0f))));
             }
         }
 #pragma unroll
@@ -57,8 +58,8 @@ __global__ void __launch_bounds__(kFoldThreads) fold_codes_kernel(const __half *
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const float2 f = __half22float2(h[j]);
-                const int c0 = __float2int_rn(__fmul_rn(__fmul_rn(f.x, __ldg(s + k + 2 * j)), rw));
-                const int c1 = __float2int_rn(__fmul_rn(__fmul_rn(f.y, __ldg(s + k + 2 * j + 1)), rw));
+                const int c0 = __float2int_rn(__fmul_rn(__fmul_rn(f.x, (s ? __ldg(s + k + 2 * j) : 1.0f)), rw));
+                const int c1 = __float2int_rn(__fmul_rn(__fmul_rn(f.y, (s ? __ldg(s + k + 2 * j + 1) : 1.0f)), rw));
                 b[2 * j] = (uint32_t)max(-iqmax, min(iqmax, c0));
                 b[2 * j + 1] = (uint32_t)max(-iqmax, min(iqmax, c1));
             }
@@ -106,6 +107,16 @@ cudaError_t launch_fold(const void *w, const void *b, int64_t N, int64_t K, cons
     fold_bias_kernel<<<(unsigned)((N + 127) / 128), 128, 0, st>>>(reinterpret_cast<const __half *>(w),
                                                                   reinterpret_cast<const __half *>(b), N, K, z,
                                                                   bfold);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_weights(const void *w, int64_t N, int64_t K, int bits_w, int8_t *qw, float *sw,
+                                    cudaStream_t st) {
+    if (N == 0) return cudaSuccess;
+    const int iqmax = (1 << (bits_w - 1)) - 1;
+    const int64_t grid = N < 65535 * 4 ? N : 65535 * 4;
+    fold_codes_kernel<<<(unsigned)grid, kFoldThreads, 0, st>>>(reinterpret_cast<const __half *>(w), N, K, nullptr,
+                                                               (float)iqmax, iqmax, qw, sw);
     return cudaGetLastError();
 }
 

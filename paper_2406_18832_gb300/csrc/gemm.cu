@@ -98,7 +98,7 @@ template <int BN, bool kS32>
 __global__ void __launch_bounds__(kThreads, 1)
     linear_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                   const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
-                  int N, int K, int ldy, int kcb, int relu) {
+                  int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok) {
     extern __shared__ uint8_t smem_raw[];
     Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -273,7 +273,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < CPW; ++j) {
                         const int m = m0 + col0 + j;
-                        float v = __fmaf_rn(__int2float_rn(tot[j]), scale, bias);
+                        // per-token path (Eq. 3): one fp32 product s_m * sw_n
+                        const float sc = s_tok ? __fmul_rn(__ldg(s_tok + (m < M ? m : M - 1)), scale) : scale;
+                        float v = __fmaf_rn(__int2float_rn(tot[j]), sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
                         if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
                     }
@@ -412,7 +414,8 @@ template <bool kS32>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
-                       int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws, uint64_t epoch) {
+                       int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws, uint64_t epoch,
+                       const float *__restrict__ s_tok) {
     extern __shared__ uint8_t smem_raw[];
     SmemPair &S = *reinterpret_cast<SmemPair *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -646,7 +649,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < 128; ++j) {
                         const int m = m0 + col0 + j;
-                        float v = __fmaf_rn(__int2float_rn(tot[j]), scale, bias);
+                        // per-token path (Eq. 3): one fp32 product s_m * sw_n
+                        const float sc = s_tok ? __fmul_rn(__ldg(s_tok + (m < M ? m : M - 1)), scale) : scale;
+                        float v = __fmaf_rn(__int2float_rn(tot[j]), sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
                         if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
                     }
@@ -727,7 +732,7 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     linear_kernel<BN, kS32><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
-                                                         (int)a.K, (int)a.ldy, kcb, a.relu);
+                                                         (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok);
     return cudaGetLastError();
 }
 
@@ -796,7 +801,7 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     const uint64_t epoch = streamk ? next_epoch() : 0;
     linear_pair_kernel<kS32><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
                                                                 (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
-                                                                epoch);
+                                                                epoch, a.s_tok);
     return cudaGetLastError();
 }
 

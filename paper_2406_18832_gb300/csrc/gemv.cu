@@ -63,7 +63,8 @@ __global__ void __launch_bounds__(gv_warps<TG>() * 32, 1) linear_gemv_kernel(con
                                                                     const float *__restrict__ sw,
                                                                     const float *__restrict__ bfold,
                                                                     void *__restrict__ out, int M, int N, int K,
-                                                                    int ldy, int kcb, int relu) {
+                                                                    int ldy, int kcb, int relu,
+                                                                    const float *__restrict__ s_tok) {
     constexpr int kGvWarps = gv_warps<TG>();
     __shared__ int32_t red[kGvWarps][TG * 16][kGvRows + 1];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -193,7 +194,9 @@ __global__ void __launch_bounds__(gv_warps<TG>() * 32, 1) linear_gemv_kernel(con
         if constexpr (kS32) {
             reinterpret_cast<int32_t *>(out)[(int64_t)m * N + n] = s;
         } else {
-            float v = __fmaf_rn(__int2float_rn(s), __ldg(sw + n), __ldg(bfold + n));
+            const float scale = __ldg(sw + n);
+            const float sc = s_tok ? __fmul_rn(__ldg(s_tok + m), scale) : scale;  // per-token path (Eq. 3)
+            float v = __fmaf_rn(__int2float_rn(s), sc, __ldg(bfold + n));
             if (relu) v = fmaxf(v, 0.f);
             reinterpret_cast<__half *>(out)[(int64_t)m * ldy + n] = __float2half_rn(v);
         }
@@ -205,7 +208,7 @@ cudaError_t run_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     const int grid = (int)((a.N + kGvRows - 1) / kGvRows);
     linear_gemv_kernel<TG, kS32><<<grid, gv_warps<TG>() * 32, 0, st>>>(
         reinterpret_cast<const __half *>(a.q), a.qw, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy,
-        kcb, a.relu);
+        kcb, a.relu, a.s_tok);
     return cudaGetLastError();
 }
 

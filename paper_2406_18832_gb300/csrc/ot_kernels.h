@@ -17,6 +17,11 @@ cudaError_t launch_fold(const void *w, const void *b, int64_t N, int64_t K, cons
                         int bits_w, int8_t *qw, float *sw, float *bfold, cudaStream_t st);
 cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
                             int bits, void *q, int fmt, cudaStream_t st);
+cudaError_t launch_quantize_tokens(const void *x, int64_t M, int64_t K, int64_t ldx, int bits, void *q, int fmt,
+                                   float *s_tok, cudaStream_t st);
+// per-output-channel weight codes without activation scales (s = 1)
+cudaError_t launch_quantize_weights(const void *w, int64_t N, int64_t K, int bits_w, int8_t *qw, float *sw,
+                                    cudaStream_t st);
 
 struct LinearArgs {
     const void *q;        // fp16 codes [M, K]
@@ -29,6 +34,7 @@ struct LinearArgs {
     bool out_s32;
     void *workspace;          // stream-K partial sums (zero-filled before first use) or null
     size_t workspace_bytes;
+    const float *s_tok;       // per-token path: token scales [M] (y uses s_tok[m] * sw[n]); null otherwise
 };
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();

@@ -90,7 +90,78 @@ __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict_
     }
 }
 
+// Per-token dynamic quantization (Eq. 3; Eq. 1 with zero point 0 and one
+// scale per row): one CTA per row; pass 1 takes amax = max |x| (fp16 max is
+// exact; __hmax2 returns the non-NaN operand), pass 2 re-reads the row (L2 /
+// L1 hit) and writes round(x * r) with r = qmax / amax.
+template <bool kF16Out>
+__global__ void __launch_bounds__(256) quantize_tokens_kernel(const __half *__restrict__ x, int64_t K, int64_t ldx,
+                                                              int qmax, void *q, float *s_tok) {
+    __shared__ float red[8];
+    const int64_t m = blockIdx.x;
+    const __half *row = x + m * ldx;
+    const int64_t nv = K / 8;
+    __half2 hm = __float2half2_rn(0.f);
+    for (int64_t v = threadIdx.x; v < nv; v += 256) {
+        const uint4 d = __ldg(reinterpret_cast<const uint4 *>(row + v * 8));
+        const __half2 *h = reinterpret_cast<const __half2 *>(&d);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) hm = __hmax2(hm, __habs2(h[j]));
+    }
+    float a = fmaxf(__low2float(hm), __high2float(hm));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
+    __syncthreads();
+    float amax = red[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) amax = fmaxf(amax, red[w]);
+    float s = 0.f, r = 0.f;
+    if (amax > 0.f && isfinite(amax)) {
+        s = __fdiv_rn(amax, (float)qmax);
+        r = __fdiv_rn((float)qmax, amax);
+    }
+    if (threadIdx.x == 0) s_tok[m] = s;
+    for (int64_t v = threadIdx.x; v < nv; v += 256) {
+        const uint4 d = __ldg(reinterpret_cast<const uint4 *>(row + v * 8));
+        const __half2 *h = reinterpret_cast<const __half2 *>(&d);
+        int c[8];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 f = __half22float2(h[j]);
+            c[2 * j] = max(-qmax, min(qmax, __float2int_rn(__fmul_rn(f.x, r))));
+            c[2 * j + 1] = max(-qmax, min(qmax, __float2int_rn(__fmul_rn(f.y, r))));
+        }
+        if (kF16Out) {
+            uint4 o;
+            o.x = pack_f16_codes(c[0], c[1]);
+            o.y = pack_f16_codes(c[2], c[3]);
+            o.z = pack_f16_codes(c[4], c[5]);
+            o.w = pack_f16_codes(c[6], c[7]);
+            *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + m * K + v * 8) = o;
+        } else {
+            uint2 o;
+            o.x = pack_i8_codes(c[0], c[1], c[2], c[3]);
+            o.y = pack_i8_codes(c[4], c[5], c[6], c[7]);
+            *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + m * K + v * 8) = o;
+        }
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_quantize_tokens(const void *x, int64_t M, int64_t K, int64_t ldx, int bits, void *q, int fmt,
+                                   float *s_tok, cudaStream_t st) {
+    if (M == 0) return cudaSuccess;
+    const int qmax = (1 << (bits - 1)) - 1;
+    if (fmt == OT_CODE_F16)
+        quantize_tokens_kernel<true><<<(unsigned)M, 256, 0, st>>>(reinterpret_cast<const __half *>(x), K, ldx, qmax,
+                                                                  q, s_tok);
+    else
+        quantize_tokens_kernel<false><<<(unsigned)M, 256, 0, st>>>(reinterpret_cast<const __half *>(x), K, ldx,
+                                                                   qmax, q, s_tok);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
                             int bits, void *q, int fmt, cudaStream_t st) {
