@@ -222,6 +222,12 @@ def run_ours(args):
         step()
     torch.cuda.synchronize()
 
+    if args.profile_decode:
+        bench_decode(dev, peaks, reps=args.steps)
+        torch.cuda.synchronize()
+        if rank == 0:
+            print(json.dumps({"profile_run": "decode", "steps": args.steps}), flush=True)
+        return
     if args.profile:
         # small, short run for profilers: the steps only, nothing else
         for _ in range(args.steps):
@@ -338,6 +344,7 @@ def run_ours(args):
     d2h = sum(y.numel() * 2 for y in ybufs)
 
     block = None if args.no_block else bench_block(dev)
+    decode = bench_decode(dev, peaks)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -379,12 +386,50 @@ def run_ours(args):
         "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
                    "ratio": round(weights_fp16 / weights_int8, 3)},
         "block": block,
+        "decode": decode,
         "cpu_baseline": cpu,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def bench_decode(dev, peaks, reps: int = 50):
+    """Decode-sized linears of the OPT-13B shapes (Int6; 1 and 16 tokens): the
+    product is bound by streaming the int8 weights from HBM, so the roofline is
+    weight bytes / time against the HBM peak."""
+    import torch
+
+    from paper_2406_18832_gb300 import binding, synth
+    c = synth.CONFIGS[3]
+    res = []
+    for li in (0, 3):
+        layer = c.layers[li]
+        qm = 31
+        g = torch.Generator(device=dev).manual_seed(3000 + li)
+        qw = torch.randint(-qm, qm + 1, (layer.N, layer.K), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+        sw = torch.rand(layer.N, generator=g, device=dev) * 1e-3
+        bf = torch.zeros(layer.N, device=dev)
+        for M in (1, 16):
+            q = torch.randint(-qm, qm + 1, (M, layer.K), generator=g, device=dev, dtype=torch.int32).half()
+            y = torch.empty(M, layer.N, dtype=torch.float16, device=dev)
+            for _ in range(3):
+                binding.ot_linear(q, qw, sw, bf, 6, 6, y)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                binding.ot_linear(q, qw, sw, bf, 6, 6, y)
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / reps
+            gbs = layer.N * layer.K / (ms * 1e-3) / 1e9
+            res.append({"layer": layer.name, "K": layer.K, "N": layer.N, "tokens": M, "us": round(ms * 1e3, 2),
+                        "weight_gbs": round(gbs, 1), "frac_hbm": round(gbs / peaks["hbm"], 4)})
+        del qw
+    return {"workload": "opt-13b decode-sized linears, Int6", "kernel": "linear_gemv_kernel (mma.sync)",
+            "bound": "hbm", "per_shape": res}
 
 
 def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):
@@ -538,6 +583,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-block", action="store_true", help="skip the OPT-30B block stage")
+    ap.add_argument("--profile-decode", action="store_true",
+                    help="profiler run of the decode-sized linears only (after the setup)")
     ap.add_argument("--profile", action="store_true",
                     help="profiler run: 8192 calibration tokens, the timed steps only, no report")
     args = ap.parse_args()
