@@ -223,10 +223,10 @@ def run_ours(args):
     torch.cuda.synchronize()
 
     if args.profile_decode:
-        bench_decode(dev, peaks, reps=args.steps)
+        dec = bench_decode(dev, peaks, reps=args.steps)
         torch.cuda.synchronize()
         if rank == 0:
-            print(json.dumps({"profile_run": "decode", "steps": args.steps}), flush=True)
+            print(json.dumps({"profile_run": "decode", "steps": args.steps, "decode": dec}), flush=True)
         return
     if args.profile:
         # small, short run for profilers: the steps only, nothing else
@@ -408,28 +408,33 @@ def bench_decode(dev, peaks, reps: int = 50):
         layer = c.layers[li]
         qm = 31
         g = torch.Generator(device=dev).manual_seed(3000 + li)
-        qw = torch.randint(-qm, qm + 1, (layer.N, layer.K), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+        # as many weight copies (successive layers of the model) as keep the
+        # weights read by consecutive calls above 3x the 129 MB L2
+        copies = max(2, -(-3 * 129 * 2 ** 20 // (layer.N * layer.K)))
+        qws = [torch.randint(-qm, qm + 1, (layer.N, layer.K), generator=g, device=dev,
+                             dtype=torch.int32).to(torch.int8) for _ in range(copies)]
         sw = torch.rand(layer.N, generator=g, device=dev) * 1e-3
         bf = torch.zeros(layer.N, device=dev)
         for M in (1, 16):
             q = torch.randint(-qm, qm + 1, (M, layer.K), generator=g, device=dev, dtype=torch.int32).half()
             y = torch.empty(M, layer.N, dtype=torch.float16, device=dev)
-            for _ in range(3):
-                binding.ot_linear(q, qw, sw, bf, 6, 6, y)
+            for i in range(max(3, copies)):
+                binding.ot_linear(q, qws[i % copies], sw, bf, 6, 6, y)
             torch.cuda.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
-            for _ in range(reps):
-                binding.ot_linear(q, qw, sw, bf, 6, 6, y)
+            for i in range(reps):
+                binding.ot_linear(q, qws[i % copies], sw, bf, 6, 6, y)
             e1.record()
             torch.cuda.synchronize()
             ms = e0.elapsed_time(e1) / reps
             gbs = layer.N * layer.K / (ms * 1e-3) / 1e9
             res.append({"layer": layer.name, "K": layer.K, "N": layer.N, "tokens": M, "us": round(ms * 1e3, 2),
                         "weight_gbs": round(gbs, 1), "frac_hbm": round(gbs / peaks["hbm"], 4)})
-        del qw
+        del qws
     return {"workload": "opt-13b decode-sized linears, Int6", "kernel": "linear_gemv_kernel (mma.sync)",
-            "bound": "hbm", "per_shape": res}
+            "bound": "hbm", "l2": "consecutive calls read different weight copies, > 3x L2 in all",
+            "per_shape": res}
 
 
 def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):

@@ -816,6 +816,11 @@ cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
 
 }  // namespace
 
+bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
+                   uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz) {
+    return make_tmap_2d(tm, dt, base, inner, rows, row_bytes, box_inner, box_rows, swz);
+}
+
 // Token counts up to this go to the mma.sync weight-streaming kernel (gemv.cu).
 constexpr int64_t kGemvMaxTokens = 32;
 
@@ -828,7 +833,23 @@ int exact_chunk_kblocks(int bits_a, int bits_w) {
     return kc < 1 ? 1 : (int)kc;
 }
 
-size_t linear_workspace_bytes() { return pair_workspace_bytes(pair_max_clusters()); }
+// Workspace layout: the stream-K region of the prefill kernel, then the
+// split-tile region of the decode kernel.
+size_t linear_workspace_bytes() { return pair_workspace_bytes(pair_max_clusters()) + gemv_workspace_bytes(); }
+
+int *device_status_word() {
+    static std::mutex mu;
+    static int *addr[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<int *>(p);
+    }
+    return addr[dev];
+}
 
 // Scratch of ot_linear_noalloc: the stream-K workspace lives in this
 // file-scope device array, so that entry point never allocates.  Every GPU
@@ -867,7 +888,14 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
     const int nkb = (int)((a.K + kBK - 1) / kBK);
     int kcb = exact_chunk_kblocks(a.bits_a, a.bits_w);
     if (kcb > nkb) kcb = nkb;
-    if (a.M <= kGemvMaxTokens) return launch_linear_gemv(a, kcb, st);
+    if (a.M <= kGemvMaxTokens) {
+        LinearArgs d = a;
+        const size_t off = pair_workspace_bytes(pair_max_clusters());
+        const bool room = a.workspace != nullptr && a.workspace_bytes >= off + gemv_workspace_bytes();
+        d.workspace = room ? static_cast<unsigned char *>(a.workspace) + off : nullptr;
+        d.workspace_bytes = room ? a.workspace_bytes - off : 0;
+        return launch_linear_gemv(d, kcb, st);
+    }
     return a.out_s32 ? dispatch_bn<true>(a, kcb, st) : dispatch_bn<false>(a, kcb, st);
 }
 

@@ -5,24 +5,41 @@
 // A 128-row tcgen05 MMA costs about 118 cycles whatever its token count, which
 // caps weight consumption at ~17 bytes per clock per SM (~5 TB/s on GB300),
 // below the HBM rate.  Warp-level mma.sync m16n8k16 (f16 in, f32 accumulate)
-// has throughput to spare at M <= 32 (600 TFLOPS measured), so here:
-//   - a CTA of 16 (one token group) or 8 (two) warps owns 32 weight rows
-//     (4 groups of 8 = the MMA's n8) and all tokens (groups of 16 = the MMA's
-//     m16); the warps split K in interleaved 64-wide windows, issue the loads
-//     of two windows before computing either (bytes in flight to cover HBM
-//     latency), and reduce their int32 partial sums in shared memory at the
-//     end (no global scratch);
-//   - lane l of a warp loads 16 contiguous int8 weights of row (8g + l/4) at
-//     K offset 16 (l % 4) of the window, widens them to fp16 in registers
-//     (exact), and uses them as the MMA's B fragment under a fixed
-//     permutation of K (the dot product does not depend on the order of k,
-//     only on A and B using the same one): logical k {2t, 2t+1, 2t+8, 2t+9}
-//     of lane-quad position t = l % 4 is actual K {16t+4j .. 16t+4j+3} in
-//     sub-step j; the fp16 activation codes are read as the A fragment under
-//     the same permutation;
+// has throughput to spare at M <= 32, so the kernel is a weight stream:
+//   - work units are (tile of 128 weight rows, 256-wide K slice); one
+//     persistent CTA per SM takes a contiguous range of units, an equal share
+//     of all of them (stream-K), so every SM streams the same number of bytes;
+//   - each unit arrives in a ring of shared-memory stages as two TMA boxes:
+//     128 weight rows x 256 int8 (32 KB, evict-first: read once) and M tokens
+//     x 256 fp16 codes (evict-last: every tile reads them again).  The tensor
+//     maps zero-fill rows past N and K past the end, so ragged tails need no
+//     special case.  Measured on GB300, the TMA unit of an SM completes about
+//     one box per 176 ns whatever its size up to 8 KB, so boxes must be large:
+//     8 KB boxes held the stream near 2.5 TB/s, 32 KB boxes reach ~7 TB/s;
+//   - the ring has no producer warp: the first S units are issued at start,
+//     and the last of the 16 warps to finish with a slot (a shared counter)
+//     refills it with the unit S places later;
+//   - the weights are the MMA's m16 operand and the tokens its n8 operand
+//     (ceil(M / 8) token groups): warp w takes the 64-wide window w % 4 of
+//     every stage and weight rows 32 (w / 4) .. + 31 (two m16 groups).  Lane l
+//     reads 16 int8 weights of rows 16g + l/4 and 16g + l/4 + 8 at window
+//     offset 16 (l % 4) and widens them to fp16 (exact) straight into A
+//     fragment order, under a fixed permutation of K (the dot product does not
+//     depend on the order of k, only on A and B using the same one): logical k
+//     {2t, 2t+1, 2t+8, 2t+9} of lane-quad position t = l % 4 is actual K
+//     {16t+4j .. 16t+4j+3} in sub-step j; the token codes, read under the same
+//     permutation, are already the B fragment (two consecutive words);
 //   - fp32 partial sums stay exact below 2^24 (chunks of kcb windows, as in
-//     the tensor-memory kernels) and are added in int32.
+//     the tensor-memory kernels) and are added, as int32, into the tile's
+//     totals in shared memory (atomics);
+//   - a tile split between CTAs adds its int32 partials into a workspace slot
+//     with integer atomics (order-free, so exact); the CTA whose unit count
+//     completes the tile's counter applies the epilogue and zeroes the slot
+//     and counter again.  Nothing waits on another CTA.
+// Without a workspace the ranges are whole tiles (no split, less even).
 #include <cuda_fp16.h>
+
+#include <mutex>
 
 #include "ot_common.cuh"
 #include "ot_kernels.h"
@@ -31,12 +48,31 @@ namespace ot {
 
 namespace {
 
-constexpr int kGvRows = 32;   // weight rows per CTA
-constexpr int kGvWin = 64;    // K per window
-constexpr int kGvUnroll = 2;  // windows whose loads a warp issues before computing
-// warps per CTA: 16 for one token group, 8 for two (register budget)
-template <int TG>
-__host__ __device__ constexpr int gv_warps() { return TG == 1 ? 16 : 8; }
+constexpr int kGvRows = 128;                      // weight rows per tile (16 MMA n8 groups)
+constexpr int kGvKS = 256;                        // K per unit / stage (= the TMA box width)
+constexpr int kGvWin = 64;                        // K per MMA window
+constexpr int kGvWindows = kGvKS / kGvWin;        // windows per stage (4)
+constexpr int kGvWarps = 16;
+constexpr int kGvThreads = kGvWarps * 32;
+constexpr int kGvWBytes = kGvRows * kGvKS;        // weight box (rows of 256 bytes)
+constexpr int kGvMaxStages = 8;
+constexpr int kGvSmemBudget = 224 * 1024;
+constexpr int kGvHeader = 256;                    // barriers, counters, flags
+constexpr int kGvSlotInts = kGvRows * 32;         // workspace ints per split tile (32 tokens x 128 rows)
+
+struct GvParams {
+    const float *sw, *bfold, *s_tok;
+    void *out;
+    int32_t *part;      // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
+    unsigned *count;    // [grid] units added to each slot so far
+    int *status;        // device status word
+    int M, N, K, ldy, kcb, relu;
+    int nks;            // units per tile
+    int stages, stage_bytes, red_bytes;
+    int64_t ntiles, units;
+    int grid;
+    int whole;          // ranges of whole tiles (no workspace)
+};
 
 __device__ __forceinline__ void i8x4_to_f16x4_gv(uint32_t w, uint32_t &lo, uint32_t &hi) {
     const uint32_t u = w ^ 0x80808080u;
@@ -57,166 +93,327 @@ __device__ __forceinline__ void mma_16816(float (&c)[4], const uint32_t (&a)[4],
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-template <int TG, bool kS32>
-__global__ void __launch_bounds__(gv_warps<TG>() * 32, 1) linear_gemv_kernel(const __half *__restrict__ q,
-                                                                    const int8_t *__restrict__ qw,
-                                                                    const float *__restrict__ sw,
-                                                                    const float *__restrict__ bfold,
-                                                                    void *__restrict__ out, int M, int N, int K,
-                                                                    int ldy, int kcb, int relu,
-                                                                    const float *__restrict__ s_tok) {
-    constexpr int kGvWarps = gv_warps<TG>();
-    __shared__ int32_t red[kGvWarps][TG * 16][kGvRows + 1];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * kGvRows;
-    const int t = lane & 3, r = lane >> 2;
-    const int nwin = (K + kGvWin - 1) / kGvWin;
+// First unit of CTA c's range.
+__device__ __forceinline__ int64_t unit_begin(int64_t c, const GvParams &p) {
+    if (p.whole) return c * p.ntiles / p.grid * p.nks;
+    return c * p.units / p.grid;
+}
 
-    // weight rows of this lane (one per group of 8), clamped for the N tail
-    const int8_t *wrow[4];
-    bool wok[4];
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-        const int n = n0 + 8 * g + r;
-        wok[g] = n < N;
-        wrow[g] = qw + (int64_t)(wok[g] ? n : 0) * K;
-    }
-    // token rows of this lane: r and r + 8 of each token group
-    const __half *qrow[TG][2];
-    bool qok[TG][2];
-#pragma unroll
-    for (int tg = 0; tg < TG; ++tg)
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int m = tg * 16 + r + 8 * h;
-            qok[tg][h] = m < M;
-            qrow[tg][h] = q + (int64_t)(qok[tg][h] ? m : 0) * K;
-        }
+// The CTA whose range holds unit x (ranges begin at floor(c * units / grid)):
+// the largest c with c * units < (x + 1) * grid.  It names the workspace slot
+// of a split tile (the CTA holding the tile's first unit): a CTA starts at
+// most one tile that continues past its range, so the slots are distinct.
+__device__ __forceinline__ int owner_of_unit(int64_t x, const GvParams &p) {
+    return (int)(((x + 1) * p.grid + p.units - 1) / p.units - 1);
+}
 
-    int32_t tot[TG][4][4];
-    float acc[TG][4][4];
-#pragma unroll
-    for (int tg = 0; tg < TG; ++tg)
-#pragma unroll
-        for (int g = 0; g < 4; ++g)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                tot[tg][g][i] = 0;
-                acc[tg][g][i] = 0.f;
-            }
-
-    int in_chunk = 0;
-    for (int win0 = warp; win0 < nwin; win0 += kGvUnroll * kGvWarps) {
-        uint4 wv[kGvUnroll][4];
-        uint4 qv[kGvUnroll][TG][2][2];
-        bool vok[kGvUnroll];
-#pragma unroll
-        for (int u = 0; u < kGvUnroll; ++u) {
-            const int win = win0 + u * kGvWarps;
-            const int k0 = win * kGvWin + 16 * t;  // this lane's 16 K of the window
-            vok[u] = win < nwin;
-            const bool kok = vok[u] && k0 < K;     // K % 16 == 0: a segment is whole or absent
-#pragma unroll
-            for (int g = 0; g < 4; ++g)
-                wv[u][g] = (kok && wok[g]) ? __ldcs(reinterpret_cast<const uint4 *>(wrow[g] + k0))
-                                           : make_uint4(0, 0, 0, 0);
-#pragma unroll
-            for (int tg = 0; tg < TG; ++tg)
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int p = 0; p < 2; ++p)
-                        qv[u][tg][h][p] = (kok && qok[tg][h])
-                                              ? __ldg(reinterpret_cast<const uint4 *>(qrow[tg][h] + k0 + 8 * p))
-                                              : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int u = 0; u < kGvUnroll; ++u) {
-            if (!vok[u]) break;
-#pragma unroll
-            for (int g = 0; g < 4; ++g) {
-                uint32_t b[8];
-                i8x4_to_f16x4_gv(wv[u][g].x, b[0], b[1]);
-                i8x4_to_f16x4_gv(wv[u][g].y, b[2], b[3]);
-                i8x4_to_f16x4_gv(wv[u][g].z, b[4], b[5]);
-                i8x4_to_f16x4_gv(wv[u][g].w, b[6], b[7]);
-#pragma unroll
-                for (int tg = 0; tg < TG; ++tg) {
-                    const uint32_t *x0 = reinterpret_cast<const uint32_t *>(&qv[u][tg][0][0]);  // token r
-                    const uint32_t *x1 = reinterpret_cast<const uint32_t *>(&qv[u][tg][1][0]);  // token r + 8
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        // sub-step j covers actual K 16t + 4j .. 16t + 4j + 3 of the window
-                        const uint32_t a[4] = {x0[2 * j], x1[2 * j], x0[2 * j + 1], x1[2 * j + 1]};
-                        mma_16816(acc[tg][g], a, b[2 * j], b[2 * j + 1]);
-                    }
-                }
-            }
-            if (++in_chunk == kcb) {
-                in_chunk = 0;
-#pragma unroll
-                for (int tg = 0; tg < TG; ++tg)
-#pragma unroll
-                    for (int g = 0; g < 4; ++g)
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            tot[tg][g][i] += __float2int_rn(acc[tg][g][i]);
-                            acc[tg][g][i] = 0.f;
-                        }
-            }
-        }
-    }
-#pragma unroll
-    for (int tg = 0; tg < TG; ++tg)
-#pragma unroll
-        for (int g = 0; g < 4; ++g)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) tot[tg][g][i] += __float2int_rn(acc[tg][g][i]);
-
-    // accumulator fragment: c0 = (token r, row 2t), c1 = (r, 2t+1), c2 = (r+8, 2t), c3 = (r+8, 2t+1)
-#pragma unroll
-    for (int tg = 0; tg < TG; ++tg)
-#pragma unroll
-        for (int g = 0; g < 4; ++g) {
-            red[warp][tg * 16 + r][8 * g + 2 * t] = tot[tg][g][0];
-            red[warp][tg * 16 + r][8 * g + 2 * t + 1] = tot[tg][g][1];
-            red[warp][tg * 16 + r + 8][8 * g + 2 * t] = tot[tg][g][2];
-            red[warp][tg * 16 + r + 8][8 * g + 2 * t + 1] = tot[tg][g][3];
-        }
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < TG * 16 * kGvRows; idx += kGvWarps * 32) {
-        const int m = idx / kGvRows, c = idx % kGvRows;
-        const int n = n0 + c;
-        if (m >= M || n >= N) continue;
-        int32_t s = 0;
-#pragma unroll
-        for (int w = 0; w < kGvWarps; ++w) s += red[w][m][c];
-        if constexpr (kS32) {
-            reinterpret_cast<int32_t *>(out)[(int64_t)m * N + n] = s;
-        } else {
-            const float scale = __ldg(sw + n);
-            const float sc = s_tok ? __fmul_rn(__ldg(s_tok + m), scale) : scale;  // per-token path (Eq. 3)
-            float v = __fmaf_rn(__int2float_rn(s), sc, __ldg(bfold + n));
-            if (relu) v = fmaxf(v, 0.f);
-            reinterpret_cast<__half *>(out)[(int64_t)m * ldy + n] = __float2half_rn(v);
-        }
+template <bool kS32>
+__device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32_t s) {
+    if constexpr (kS32) {
+        reinterpret_cast<int32_t *>(p.out)[(int64_t)m * p.N + n] = s;
+    } else {
+        const float scale = __ldg(p.sw + n);
+        const float sc = p.s_tok ? __fmul_rn(__ldg(p.s_tok + m), scale) : scale;  // per-token path (Eq. 3)
+        float v = __fmaf_rn(__int2float_rn(s), sc, __ldg(p.bfold + n));
+        if (p.relu) v = fmaxf(v, 0.f);
+        reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = __float2half_rn(v);
     }
 }
 
-template <int TG, bool kS32>
-cudaError_t run_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
-    const int grid = (int)((a.N + kGvRows - 1) / kGvRows);
-    linear_gemv_kernel<TG, kS32><<<grid, gv_warps<TG>() * 32, 0, st>>>(
-        reinterpret_cast<const __half *>(a.q), a.qw, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy,
-        kcb, a.relu, a.s_tok);
+// TN token groups of 8 (the MMA's n8).
+template <int TN, bool kS32>
+__global__ void __launch_bounds__(kGvThreads, 1)
+    linear_gemv_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_a,
+                       const GvParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    uint64_t *full = reinterpret_cast<uint64_t *>(base);
+    unsigned *done = reinterpret_cast<unsigned *>(full + kGvMaxStages);  // warps finished with a slot, ever
+    unsigned *loads = done + kGvMaxStages;                                // units loaded into a slot, ever
+    volatile int *abort = reinterpret_cast<volatile int *>(loads + kGvMaxStages);
+    volatile int *last = abort + 1;
+    int32_t(*red)[kGvRows + 1] = reinterpret_cast<int32_t(*)[kGvRows + 1]>(base + kGvHeader);  // [TN*8]
+    uint8_t *ring = base + kGvHeader + p.red_bytes;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int S = p.stages;
+    const int64_t u_begin = unit_begin(blockIdx.x, p), u_end = unit_begin(blockIdx.x + 1, p);
+    const int M = p.M, N = p.N, K = p.K, nks = p.nks;
+    const int64_t tile0 = u_begin / nks;
+    const int ks0 = (int)(u_begin - tile0 * nks);
+    const uint32_t abytes = (uint32_t)M * kGvKS * 2;  // activation box
+    uint64_t pol_w = 0, pol_a = 0;
+
+    // Load unit (tile, ks) into `slot`, completing on full[slot].
+    auto load_unit = [&](int slot, int64_t tile, int ks) {
+        const uint32_t bar = smem_u32(&full[slot]);
+        mbar_arrive_expect_tx(bar, kGvWBytes + abytes);
+        const uint32_t st = smem_u32(ring + (size_t)slot * p.stage_bytes);
+        tma_load_2d_hint(st, &tm_w, bar, ks * kGvKS, (int32_t)(tile * kGvRows), pol_w);
+        tma_load_2d_hint(st + kGvWBytes, &tm_a, bar, ks * kGvKS, 0, pol_a);
+        loads[slot] += 1;
+    };
+
+    if (lane == 0) {
+        pol_w = l2_policy_evict_first();
+        pol_a = l2_policy_evict_last();
+    }
+    for (int i = threadIdx.x; i < TN * 8 * (kGvRows + 1); i += kGvThreads) (&red[0][0])[i] = 0;
+    if (threadIdx.x == 0) {
+        tma_prefetch_desc(&tm_w);
+        tma_prefetch_desc(&tm_a);
+        for (int s = 0; s < S; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            done[s] = 0;
+            loads[s] = 0;
+        }
+        *abort = 0;
+        *last = 0;
+        fence_barrier_init();
+        int64_t tile = tile0;
+        int ks = ks0;
+        for (int s = 0; s < S && u_begin + s < u_end; ++s) {
+            load_unit(s, tile, ks);
+            if (++ks == nks) {
+                ks = 0;
+                ++tile;
+            }
+        }
+    }
+    __syncthreads();
+
+    const int t = lane & 3, r = lane >> 2;
+    const int win = warp % kGvWindows, rp = warp / kGvWindows;  // window; rows 32 rp .. 32 rp + 31
+    const int kw = win * kGvWin;
+    bool tok[TN];  // this lane's token (8 tn + r) exists
+    bool tgv[TN];  // some lane's does (warp-uniform)
+#pragma unroll
+    for (int tn = 0; tn < TN; ++tn) {
+        tok[tn] = tn * 8 + r < M;
+        tgv[tn] = tn * 8 < M;
+    }
+    // byte offsets inside a stage: this lane's weight row 32 rp + r and token row r
+    const int w_off = (32 * rp + r) * kGvKS + kw + 16 * t;
+    const int a_off = kGvWBytes + r * (2 * kGvKS) + 2 * (kw + 16 * t);
+
+    float acc[2][TN][4];
+#pragma unroll
+    for (int g = 0; g < 2; ++g)
+#pragma unroll
+        for (int tn = 0; tn < TN; ++tn)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[g][tn][i] = 0.f;
+    // Add the exact fp32 chunk sums into the tile's int32 totals in shared
+    // memory.  Accumulator fragment: c0 = (row r, token 2t), c1 = (r, 2t+1),
+    // c2 = (r+8, 2t), c3 = (r+8, 2t+1).
+    auto flush = [&]() {
+#pragma unroll
+        for (int g = 0; g < 2; ++g)
+#pragma unroll
+            for (int tn = 0; tn < TN; ++tn)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int m = tn * 8 + 2 * t + (i & 1);
+                    if (m < M) atomicAdd(&red[m][32 * rp + 16 * g + r + 8 * (i >> 1)], __float2int_rn(acc[g][tn][i]));
+                    acc[g][tn][i] = 0.f;
+                }
+    };
+
+    int slot = 0;
+    uint32_t phase = 0;
+    int in_chunk = 0;
+    int64_t tile = tile0;
+    int ks = ks0;
+    int64_t u = u_begin;
+    while (u < u_end) {
+        const int64_t seg_end = min(u_end, u + (nks - ks));
+        const int mine = (int)(seg_end - u);
+        for (; u < seg_end; ++u, ++ks) {
+            const bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[slot]), phase, abort, p.status));
+            // past K the boxes hold zeros; skip windows that lie wholly past it
+            if (ok && kw < K - ks * kGvKS) {
+                if (in_chunk == p.kcb) {
+                    in_chunk = 0;
+                    flush();
+                }
+                ++in_chunk;
+                const uint8_t *st = ring + (size_t)slot * p.stage_bytes;
+                uint4 wv[2][2];  // [group][row r / r + 8]
+#pragma unroll
+                for (int g = 0; g < 2; ++g)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+                        wv[g][h] = *reinterpret_cast<const uint4 *>(st + w_off + (16 * g + 8 * h) * kGvKS);
+                uint32_t x[TN][8];  // token 8 tn + r, actual K 16t .. 16t + 15 of the window (fp16 pairs)
+#pragma unroll
+                for (int tn = 0; tn < TN; ++tn) {
+                    uint4 lo = make_uint4(0, 0, 0, 0), hi = make_uint4(0, 0, 0, 0);
+                    if (tgv[tn] && tok[tn]) {
+                        lo = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * (2 * kGvKS));
+                        hi = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * (2 * kGvKS) + 16);
+                    }
+                    x[tn][0] = lo.x; x[tn][1] = lo.y; x[tn][2] = lo.z; x[tn][3] = lo.w;
+                    x[tn][4] = hi.x; x[tn][5] = hi.y; x[tn][6] = hi.z; x[tn][7] = hi.w;
+                }
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                    // A fragment of sub-step j: {row r: k pair 0, row r+8: k pair 0, row r: pair 1, row r+8: pair 1}
+                    uint32_t a[4][4];
+                    const uint32_t w0[4] = {wv[g][0].x, wv[g][0].y, wv[g][0].z, wv[g][0].w};
+                    const uint32_t w1[4] = {wv[g][1].x, wv[g][1].y, wv[g][1].z, wv[g][1].w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        i8x4_to_f16x4_gv(w0[j], a[j][0], a[j][2]);
+                        i8x4_to_f16x4_gv(w1[j], a[j][1], a[j][3]);
+                    }
+#pragma unroll
+                    for (int tn = 0; tn < TN; ++tn) {
+                        if (!tgv[tn]) continue;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) mma_16816(acc[g][tn], a[j], x[tn][2 * j], x[tn][2 * j + 1]);
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) {
+                // the last warp done with this slot refills it with the unit S places on
+                __threadfence_block();
+                if (atomicAdd(&done[slot], 1u) % kGvWarps == kGvWarps - 1 && u + S < u_end && !*abort) {
+                    __threadfence_block();
+                    int64_t tile2 = tile;
+                    int ks2 = ks + S;
+                    while (ks2 >= nks) {
+                        ks2 -= nks;
+                        ++tile2;
+                    }
+                    load_unit(slot, tile2, ks2);
+                }
+            }
+            if (++slot == S) {
+                slot = 0;
+                phase ^= 1;
+            }
+        }
+
+        // ---- end of this CTA's part of the tile: add the warps' totals ----
+        in_chunk = 0;
+        flush();
+        __syncthreads();
+        const int n0 = (int)(tile * kGvRows);
+        if (mine == nks) {
+            for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
+                const int m = idx / kGvRows, c = idx % kGvRows;
+                const int32_t s = red[m][c];
+                red[m][c] = 0;
+                if (n0 + c < N) store_out<kS32>(p, m, n0 + c, s);
+            }
+        } else {
+            const int owner = owner_of_unit(tile * nks, p);
+            int32_t *part = p.part + (size_t)owner * kGvSlotInts;
+            for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
+                const int m = idx / kGvRows, c = idx % kGvRows;
+                const int32_t s = red[m][c];
+                red[m][c] = 0;
+                if (n0 + c < N) atomicAdd(part + idx, s);
+            }
+            __threadfence();
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                const unsigned before = atomicAdd(p.count + owner, (unsigned)mine);
+                *last = (before + (unsigned)mine == (unsigned)nks) ? 1 : 0;
+            }
+            __syncthreads();
+            if (*last) {
+                // every other part of the tile is in the slot: finish it and leave the slot zeroed
+                __threadfence();
+                for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
+                    const int m = idx / kGvRows, c = idx % kGvRows;
+                    if (n0 + c >= N) continue;
+                    store_out<kS32>(p, m, n0 + c, __ldcg(part + idx));
+                    __stcg(part + idx, 0);
+                }
+                if (threadIdx.x == 0) p.count[owner] = 0;
+            }
+        }
+        __syncthreads();  // red and the flag are reused by the next tile
+        ks = 0;
+        ++tile;
+    }
+    // teardown (only matters after a timeout): every copy issued must land
+    // before the CTA's shared memory goes away
+    if (threadIdx.x == 0)
+        for (int s = 0; s < S; ++s)
+            if (loads[s] > 0) wait_teardown_status(smem_u32(&full[s]), (loads[s] - 1) & 1, p.status);
+}
+
+template <int TN, bool kS32>
+cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvParams &base, cudaStream_t st) {
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(linear_gemv_kernel<TN, kS32>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kGvSmemBudget);
+    });
+    if (attr_err != cudaSuccess) return attr_err;
+    GvParams p = base;
+    p.red_bytes = (TN * 8 * (kGvRows + 1) * 4 + 127) / 128 * 128;
+    p.stage_bytes = kGvWBytes + p.M * kGvKS * 2;  // a multiple of 512
+    const int room = kGvSmemBudget - 128 - kGvHeader - p.red_bytes;
+    p.stages = room / p.stage_bytes;
+    if (p.stages > kGvMaxStages) p.stages = kGvMaxStages;
+    if (p.stages < 2) return cudaErrorInvalidConfiguration;
+    const size_t smem = 128 + kGvHeader + (size_t)p.red_bytes + (size_t)p.stages * p.stage_bytes;
+    linear_gemv_kernel<TN, kS32><<<p.grid, kGvThreads, smem, st>>>(tm_w, tm_a, p);
     return cudaGetLastError();
 }
 
 }  // namespace
 
+size_t gemv_workspace_bytes() {
+    const size_t g = (size_t)num_sms();
+    return g * kGvSlotInts * sizeof(int32_t) + (g * sizeof(unsigned) + 15) / 16 * 16;
+}
+
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
-    if (a.M <= 16) return a.out_s32 ? run_gemv<1, true>(a, kcb, st) : run_gemv<1, false>(a, kcb, st);
-    return a.out_s32 ? run_gemv<2, true>(a, kcb, st) : run_gemv<2, false>(a, kcb, st);
+    // weights: boxes of 128 rows x 256 int8; codes: boxes of all M tokens x 256
+    // fp16 (no swizzle; both zero-filled outside the arrays)
+    CUtensorMap tm_w, tm_a;
+    if (!tensor_map_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
+                       kGvKS, kGvRows, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !tensor_map_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
+                       (uint64_t)a.K * 2, kGvKS, (uint32_t)a.M, CU_TENSOR_MAP_SWIZZLE_NONE))
+        return cudaErrorInvalidValue;
+    GvParams p{};
+    p.sw = a.sw;
+    p.bfold = a.bfold;
+    p.s_tok = a.s_tok;
+    p.out = a.out;
+    p.status = device_status_word();
+    if (!p.status) return cudaErrorUnknown;
+    p.M = (int)a.M;
+    p.N = (int)a.N;
+    p.K = (int)a.K;
+    p.ldy = (int)a.ldy;
+    p.kcb = kcb;
+    p.relu = a.relu;
+    p.nks = (int)((a.K + kGvKS - 1) / kGvKS);
+    p.ntiles = (a.N + kGvRows - 1) / kGvRows;
+    p.units = p.ntiles * p.nks;
+    const int sms = num_sms();
+    // a.workspace here is the decode region of the caller's workspace
+    const bool split = a.workspace != nullptr && a.workspace_bytes >= gemv_workspace_bytes();
+    if (split) {
+        p.whole = 0;
+        p.grid = (int)(p.units < sms ? p.units : sms);
+        p.part = reinterpret_cast<int32_t *>(a.workspace);
+        p.count = reinterpret_cast<unsigned *>(p.part + (size_t)sms * kGvSlotInts);
+    } else {
+        p.whole = 1;
+        p.grid = (int)(p.ntiles < sms ? p.ntiles : sms);
+    }
+    if (a.M <= 8) return a.out_s32 ? run_gemv<1, true>(tm_w, tm_a, p, st) : run_gemv<1, false>(tm_w, tm_a, p, st);
+    if (a.M <= 16) return a.out_s32 ? run_gemv<2, true>(tm_w, tm_a, p, st) : run_gemv<2, false>(tm_w, tm_a, p, st);
+    return a.out_s32 ? run_gemv<4, true>(tm_w, tm_a, p, st) : run_gemv<4, false>(tm_w, tm_a, p, st);
 }
 
 }  // namespace ot

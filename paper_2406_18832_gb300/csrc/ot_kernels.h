@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace ot {
@@ -42,8 +43,17 @@ size_t linear_workspace_bytes();
 constexpr size_t kNoAllocScratchBytes = (size_t)24 << 20;
 cudaError_t noalloc_scratch(void **ptr, cudaStream_t st);
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
-// decode-sized token counts (M <= 32); kcb as in launch_linear
+// decode-sized token counts (M <= 32); kcb as in launch_linear; a.workspace is
+// the decode region of the caller's workspace (or null)
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st);
+// bytes of the decode region (split-tile partial sums and counters)
+size_t gemv_workspace_bytes();
+// device address of the status word that bounded waits write on timeout
+int *device_status_word();
+// 2-D tiled tensor map of a row-major [rows, inner] array (false if the
+// driver's encoder is missing or rejects the arguments)
+bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
+                   uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz);
 
 int num_sms();
 int exact_chunk_kblocks(int bits_a, int bits_w);
