@@ -816,6 +816,8 @@ cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
 
 }  // namespace
 
+uint64_t next_launch_epoch() { return next_epoch(); }
+
 bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz) {
     return make_tmap_2d(tm, dt, base, inner, rows, row_bytes, box_inner, box_rows, swz);

@@ -9,9 +9,10 @@
 //   - work units are (tile of 128 weight rows, 256-wide K slice); one
 //     persistent CTA per SM takes a contiguous range of units, an equal share
 //     of all of them (stream-K), so every SM streams the same number of bytes;
-//   - each unit arrives in a ring of shared-memory stages as two TMA boxes:
-//     128 weight rows x 256 int8 (32 KB, evict-first: read once) and M tokens
-//     x 256 fp16 codes (evict-last: every tile reads them again).  The tensor
+//   - each unit arrives in a ring of shared-memory stages as three TMA boxes:
+//     two of 128 weight rows x 128 int8 (16 KB each, 128-byte swizzle,
+//     evict-first: read once) and one of M tokens x 256 fp16 codes
+//     (evict-last: every tile reads them again).  The tensor
 //     maps zero-fill rows past N and K past the end, so ragged tails need no
 //     special case.  Measured on GB300, the TMA unit of an SM completes about
 //     one box per 176 ns whatever its size up to 8 KB, so boxes must be large:
@@ -32,10 +33,14 @@
 //   - fp32 partial sums stay exact below 2^24 (chunks of kcb windows, as in
 //     the tensor-memory kernels) and are added, as int32, into the tile's
 //     totals in shared memory (atomics);
-//   - a tile split between CTAs adds its int32 partials into a workspace slot
-//     with integer atomics (order-free, so exact); the CTA whose unit count
-//     completes the tile's counter applies the epilogue and zeroes the slot
-//     and counter again.  Nothing waits on another CTA.
+//   - a tile split between CTAs is finished by the CTA holding its first
+//     unit, which works on it last (at the end of its range); the others work
+//     on it first (at the start of theirs), store their int32 partials in a
+//     workspace slot of their own and publish it with a launch-epoch flag
+//     (release).  The finisher adds the slots (acquire; normally published
+//     long before) and applies the epilogue.  The epochs grow from launch to
+//     launch, so a flag left by an earlier launch never matches and nothing
+//     has to be cleared.
 // Without a workspace the ranges are whole tiles (no split, less even).
 #include <cuda_fp16.h>
 
@@ -54,7 +59,8 @@ constexpr int kGvWin = 64;                        // K per MMA window
 constexpr int kGvWindows = kGvKS / kGvWin;        // windows per stage (4)
 constexpr int kGvWarps = 16;
 constexpr int kGvThreads = kGvWarps * 32;
-constexpr int kGvWBytes = kGvRows * kGvKS;        // weight box (rows of 256 bytes)
+constexpr int kGvWBox = kGvRows * 128;           // weight box: 128 rows x 128 bytes, 128-byte swizzle
+constexpr int kGvWBytes = 2 * kGvWBox;            // weights of a stage (two boxes)
 constexpr int kGvMaxStages = 8;
 constexpr int kGvSmemBudget = 224 * 1024;
 constexpr int kGvHeader = 256;                    // barriers, counters, flags
@@ -63,8 +69,9 @@ constexpr int kGvSlotInts = kGvRows * 32;         // workspace ints per split ti
 struct GvParams {
     const float *sw, *bfold, *s_tok;
     void *out;
-    int32_t *part;      // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
-    unsigned *count;    // [grid] units added to each slot so far
+    int32_t *part;                 // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
+    unsigned long long *flags;     // [grid] launch epoch once a CTA's slot is complete
+    uint64_t epoch;
     int *status;        // device status word
     int M, N, K, ldy, kcb, relu;
     int nks;            // units per tile
@@ -100,11 +107,15 @@ __device__ __forceinline__ int64_t unit_begin(int64_t c, const GvParams &p) {
 }
 
 // The CTA whose range holds unit x (ranges begin at floor(c * units / grid)):
-// the largest c with c * units < (x + 1) * grid.  It names the workspace slot
-// of a split tile (the CTA holding the tile's first unit): a CTA starts at
-// most one tile that continues past its range, so the slots are distinct.
-__device__ __forceinline__ int owner_of_unit(int64_t x, const GvParams &p) {
+// the largest c with c * units < (x + 1) * grid.
+__device__ __forceinline__ int cta_of_unit(int64_t x, const GvParams &p) {
     return (int)(((x + 1) * p.grid + p.units - 1) / p.units - 1);
+}
+
+__device__ __forceinline__ uint64_t ld_acquire_flag(const unsigned long long *f) {
+    uint64_t v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(f) : "memory");
+    return v;
 }
 
 template <bool kS32>
@@ -126,14 +137,14 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     linear_gemv_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_a,
                        const GvParams p) {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    // 1024-byte alignment: the swizzle pattern of a TMA box repeats every 1024 bytes
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(base);
     unsigned *done = reinterpret_cast<unsigned *>(full + kGvMaxStages);  // warps finished with a slot, ever
     unsigned *loads = done + kGvMaxStages;                                // units loaded into a slot, ever
     volatile int *abort = reinterpret_cast<volatile int *>(loads + kGvMaxStages);
-    volatile int *last = abort + 1;
     int32_t(*red)[kGvRows + 1] = reinterpret_cast<int32_t(*)[kGvRows + 1]>(base + kGvHeader);  // [TN*8]
-    uint8_t *ring = base + kGvHeader + p.red_bytes;
+    uint8_t *ring = base + ((kGvHeader + p.red_bytes + 1023) & ~1023);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int S = p.stages;
@@ -150,6 +161,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         mbar_arrive_expect_tx(bar, kGvWBytes + abytes);
         const uint32_t st = smem_u32(ring + (size_t)slot * p.stage_bytes);
         tma_load_2d_hint(st, &tm_w, bar, ks * kGvKS, (int32_t)(tile * kGvRows), pol_w);
+        tma_load_2d_hint(st + kGvWBox, &tm_w, bar, ks * kGvKS + 128, (int32_t)(tile * kGvRows), pol_w);
         tma_load_2d_hint(st + kGvWBytes, &tm_a, bar, ks * kGvKS, 0, pol_a);
         loads[slot] += 1;
     };
@@ -168,7 +180,6 @@ __global__ void __launch_bounds__(kGvThreads, 1)
             loads[s] = 0;
         }
         *abort = 0;
-        *last = 0;
         fence_barrier_init();
         int64_t tile = tile0;
         int ks = ks0;
@@ -193,7 +204,12 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         tgv[tn] = tn * 8 < M;
     }
     // byte offsets inside a stage: this lane's weight row 32 rp + r and token row r
-    const int w_off = (32 * rp + r) * kGvKS + kw + 16 * t;
+    // Lane r holds the A fragment rows r and r + 8 of each m16 group; logical row
+    // r is the group's physical row sg = r/2 + 4 (r % 2), so that the two rows of
+    // a quarter-warp (r = 2q, 2q + 1) sit 4 rows apart and their 128-byte
+    // swizzles (16-byte chunk c stored at c ^ (row % 8)) fall in different bank halves.
+    const int sg = (r >> 1) + 4 * (r & 1);
+    const int w_off = (kw >> 7) * kGvWBox + (32 * rp + sg) * 128 + ((((kw & 127) >> 4) + t) ^ sg) * 16;
     const int a_off = kGvWBytes + r * (2 * kGvKS) + 2 * (kw + 16 * t);
 
     float acc[2][TN][4];
@@ -214,7 +230,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int m = tn * 8 + 2 * t + (i & 1);
-                    if (m < M) atomicAdd(&red[m][32 * rp + 16 * g + r + 8 * (i >> 1)], __float2int_rn(acc[g][tn][i]));
+                    if (m < M) atomicAdd(&red[m][32 * rp + 16 * g + sg + 8 * (i >> 1)], __float2int_rn(acc[g][tn][i]));
                     acc[g][tn][i] = 0.f;
                 }
     };
@@ -226,7 +242,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     int ks = ks0;
     int64_t u = u_begin;
     while (u < u_end) {
-        const int64_t seg_end = min(u_end, u + (nks - ks));
+        const int64_t seg_begin = u, seg_end = min(u_end, u + (nks - ks));
         const int mine = (int)(seg_end - u);
         for (; u < seg_end; ++u, ++ks) {
             const bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[slot]), phase, abort, p.status));
@@ -243,7 +259,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 for (int g = 0; g < 2; ++g)
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
-                        wv[g][h] = *reinterpret_cast<const uint4 *>(st + w_off + (16 * g + 8 * h) * kGvKS);
+                        wv[g][h] = *reinterpret_cast<const uint4 *>(st + w_off + (16 * g + 8 * h) * 128);
                 uint32_t x[TN][8];  // token 8 tn + r, actual K 16t .. 16t + 15 of the window (fp16 pairs)
 #pragma unroll
                 for (int tn = 0; tn < TN; ++tn) {
@@ -307,35 +323,46 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 red[m][c] = 0;
                 if (n0 + c < N) store_out<kS32>(p, m, n0 + c, s);
             }
-        } else {
-            const int owner = owner_of_unit(tile * nks, p);
-            int32_t *part = p.part + (size_t)owner * kGvSlotInts;
+        } else if (seg_begin != tile * nks) {
+            // a later part of a tile that an earlier CTA finishes: publish it
+            int32_t *part = p.part + (size_t)blockIdx.x * kGvSlotInts;
             for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
                 const int m = idx / kGvRows, c = idx % kGvRows;
-                const int32_t s = red[m][c];
+                __stcg(part + idx, red[m][c]);
                 red[m][c] = 0;
-                if (n0 + c < N) atomicAdd(part + idx, s);
             }
             __threadfence();
             __syncthreads();
             if (threadIdx.x == 0) {
-                const unsigned before = atomicAdd(p.count + owner, (unsigned)mine);
-                *last = (before + (unsigned)mine == (unsigned)nks) ? 1 : 0;
+                __threadfence();
+                atomicExch(p.flags + blockIdx.x, (unsigned long long)p.epoch);
+            }
+        } else {
+            // the first part: add the later parts (CTAs blockIdx.x + 1 .. last) and finish the tile
+            const int c_last = cta_of_unit((tile + 1) * nks - 1, p);
+            const int nc = c_last - (int)blockIdx.x;
+            if (threadIdx.x < nc) {
+                const unsigned long long *f = p.flags + blockIdx.x + 1 + threadIdx.x;
+                const uint64_t t0 = globaltimer_ns();
+                while (ld_acquire_flag(f) != p.epoch) {
+                    if (*abort) break;
+                    if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                        atomicExch(p.status, (int)OT_ERR_TIMEOUT);
+                        *abort = 1;
+                        break;
+                    }
+                }
             }
             __syncthreads();
-            if (*last) {
-                // every other part of the tile is in the slot: finish it and leave the slot zeroed
-                __threadfence();
-                for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
-                    const int m = idx / kGvRows, c = idx % kGvRows;
-                    if (n0 + c >= N) continue;
-                    store_out<kS32>(p, m, n0 + c, __ldcg(part + idx));
-                    __stcg(part + idx, 0);
-                }
-                if (threadIdx.x == 0) p.count[owner] = 0;
+            for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
+                const int m = idx / kGvRows, c = idx % kGvRows;
+                int32_t s = red[m][c];
+                red[m][c] = 0;
+                for (int j = 1; j <= nc; ++j) s += __ldcg(p.part + (size_t)(blockIdx.x + j) * kGvSlotInts + idx);
+                if (n0 + c < N) store_out<kS32>(p, m, n0 + c, s);
             }
         }
-        __syncthreads();  // red and the flag are reused by the next tile
+        __syncthreads();  // red is reused by the next tile
         ks = 0;
         ++tile;
     }
@@ -357,12 +384,13 @@ cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvP
     if (attr_err != cudaSuccess) return attr_err;
     GvParams p = base;
     p.red_bytes = (TN * 8 * (kGvRows + 1) * 4 + 127) / 128 * 128;
-    p.stage_bytes = kGvWBytes + p.M * kGvKS * 2;  // a multiple of 512
-    const int room = kGvSmemBudget - 128 - kGvHeader - p.red_bytes;
+    p.stage_bytes = (kGvWBytes + p.M * kGvKS * 2 + 1023) & ~1023;
+    const int ring_off = (kGvHeader + p.red_bytes + 1023) & ~1023;
+    const int room = kGvSmemBudget - 1024 - ring_off;
     p.stages = room / p.stage_bytes;
     if (p.stages > kGvMaxStages) p.stages = kGvMaxStages;
     if (p.stages < 2) return cudaErrorInvalidConfiguration;
-    const size_t smem = 128 + kGvHeader + (size_t)p.red_bytes + (size_t)p.stages * p.stage_bytes;
+    const size_t smem = 1024 + ring_off + (size_t)p.stages * p.stage_bytes;
     linear_gemv_kernel<TN, kS32><<<p.grid, kGvThreads, smem, st>>>(tm_w, tm_a, p);
     return cudaGetLastError();
 }
@@ -371,15 +399,15 @@ cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvP
 
 size_t gemv_workspace_bytes() {
     const size_t g = (size_t)num_sms();
-    return g * kGvSlotInts * sizeof(int32_t) + (g * sizeof(unsigned) + 15) / 16 * 16;
+    return g * kGvSlotInts * sizeof(int32_t) + g * sizeof(unsigned long long);
 }
 
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
-    // weights: boxes of 128 rows x 256 int8; codes: boxes of all M tokens x 256
-    // fp16 (no swizzle; both zero-filled outside the arrays)
+    // weights: boxes of 128 rows x 128 int8 (128-byte swizzle); codes: boxes of
+    // all M tokens x 256 fp16 (no swizzle); both zero-filled outside the arrays
     CUtensorMap tm_w, tm_a;
     if (!tensor_map_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
-                       kGvKS, kGvRows, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+                       128, kGvRows, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !tensor_map_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
                        (uint64_t)a.K * 2, kGvKS, (uint32_t)a.M, CU_TENSOR_MAP_SWIZZLE_NONE))
         return cudaErrorInvalidValue;
@@ -406,7 +434,8 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
         p.whole = 0;
         p.grid = (int)(p.units < sms ? p.units : sms);
         p.part = reinterpret_cast<int32_t *>(a.workspace);
-        p.count = reinterpret_cast<unsigned *>(p.part + (size_t)sms * kGvSlotInts);
+        p.flags = reinterpret_cast<unsigned long long *>(p.part + (size_t)sms * kGvSlotInts);
+        p.epoch = next_launch_epoch();
     } else {
         p.whole = 1;
         p.grid = (int)(p.ntiles < sms ? p.ntiles : sms);

@@ -48,6 +48,8 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st);
 // bytes of the decode region (split-tile partial sums and counters)
 size_t gemv_workspace_bytes();
+// strictly increasing per call (stream-K flags of both linear kernels)
+uint64_t next_launch_epoch();
 // device address of the status word that bounded waits write on timeout
 int *device_status_word();
 // 2-D tiled tensor map of a row-major [rows, inner] array (false if the
