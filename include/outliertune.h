@@ -135,11 +135,12 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  *   workspace, workspace_bytes  optional device scratch (16-byte aligned) of
  *           at least ot_linear_workspace_size() bytes, ZERO-FILLED before its
  *           first use; the kernel leaves it valid for the next call.  With it,
- *           prefill-sized calls (M > 128) share the (tile, k-block) work
- *           evenly over the SMs and exchange exact int32 partial sums through
- *           it (stream-K); with NULL / too small, whole tiles are dealt out.
- *           Calls that overlap on the GPU must not share a workspace.  The
- *           result is bit-identical either way.
+ *           prefill-sized calls (M > 128) and decode-sized calls (M <= 32) may
+ *           share the (tile, K-slice) work evenly over the SMs and exchange
+ *           exact int32 partial sums through it (stream-K); with NULL / too
+ *           small, whole tiles are dealt out.  Calls that overlap on the GPU
+ *           must not share a workspace.  The result is bit-identical either
+ *           way.
  * Exactness: the tensor cores accumulate in fp32, which holds integers
  * exactly up to 2^24; the kernel therefore sums K in chunks short enough
  * that no partial sum can pass 2^24 for the promised bits, and adds the
@@ -153,8 +154,8 @@ ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
 
 /*
  * ot_linear_workspace_size -- bytes of scratch that let ot_linear /
- * ot_linear_s32 balance prefill-sized calls over all SMs on the current
- * device (about 20 MB on a 152-SM GB300).  Host-only query.
+ * ot_linear_s32 balance prefill- and decode-sized calls over all SMs on the
+ * current device (about 22.4 MB on a 152-SM GB300).  Host-only query.
  */
 ot_status ot_linear_workspace_size(size_t *bytes);
 
@@ -216,7 +217,7 @@ ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int
  *     calls that overlap on the GPU (on different streams, or from several
  *     threads) race and may corrupt each other's results: serialize them.
  *   - Returns OT_ERR_UNSUPPORTED if the device would need more scratch than
- *     the array holds (more than 96 CTA pairs, i.e. more than 192 SMs).
+ *     the array holds (more than 170 SMs; a 152-SM GB300 needs ~22.4 MB).
  */
 ot_status ot_linear_noalloc(const void *q_f16, int64_t M, int64_t K,
                             const int8_t *qw, const float *sw,

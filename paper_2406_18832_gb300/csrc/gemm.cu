@@ -856,8 +856,8 @@ int *device_status_word() {
 // Scratch of ot_linear_noalloc: the stream-K workspace lives in this
 // file-scope device array, so that entry point never allocates.  Every GPU
 // that loads the library holds it until the process exits.  24 MiB covers
-// the partial-sum slots and flags of up to 96 CTA pairs (a 152-SM GB300 uses
-// 76 pairs, about 20 MB).
+// the prefill and decode partial-sum slots and flags of devices with up to
+// 170 SMs (a 152-SM GB300 needs about 22.4 MB).
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 // Device address of g_noalloc_scratch on the current device.  In host code

@@ -428,8 +428,18 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     p.ntiles = (a.N + kGvRows - 1) / kGvRows;
     p.units = p.ntiles * p.nks;
     const int sms = num_sms();
-    // a.workspace here is the decode region of the caller's workspace
-    const bool split = a.workspace != nullptr && a.workspace_bytes >= gemv_workspace_bytes();
+    // a.workspace here is the decode region of the caller's workspace.  Split
+    // tiles even out the per-SM work but add the partial-sum exchange, and the
+    // weight stream saturates HBM once about 60% of the SMs take part; so whole
+    // tiles are kept when they already occupy that many SMs and the busiest
+    // CTA gets at most 25% more units than an even split would give it
+    // (measured on GB300: OPT-13B QKV and 16384 x 4096 at one token run 8-15%
+    // faster on whole tiles, fc2 and 4096 x 4096 2-2.5x faster split).
+    const int64_t active = p.ntiles < sms ? p.ntiles : sms;
+    const int64_t whole_units = (p.ntiles + sms - 1) / sms * p.nks;
+    const int64_t even_units = (p.units + sms - 1) / sms;
+    const bool whole_ok = 10 * active >= 6 * (int64_t)sms && 4 * whole_units <= 5 * even_units;
+    const bool split = !whole_ok && a.workspace != nullptr && a.workspace_bytes >= gemv_workspace_bytes();
     if (split) {
         p.whole = 0;
         p.grid = (int)(p.units < sms ? p.units : sms);
