@@ -18,6 +18,10 @@ and the per-token path of Eq. 3 (the paper's out / fc2 linears):
   quantize_tokens   - dynamic per-token scale s_m = max|x[m,:]| / qmax and codes
   quantize_weights  - per-output-channel codes of W without activation scales
   epilogue_tokens   - fp16(fma((float)acc, s_m * sw_n, b_n))
+and the asymmetric weights ("Int8": per-output-channel zero points, Eq. 1):
+  fold_codes_asym   - codes of W_s over [min(0, min), max(0, max)] with a zero point
+  rowsum            - sum_k q[m,k] (exact)
+  epilogue_asym     - fp16(fma((float)(acc - zc_n rs_m), sw_n, b'_n))
 """
 from __future__ import annotations
 
@@ -67,8 +71,12 @@ def _load():
             lib.oracle_epilogue.argtypes = [P, I64, I64, P, P, I, P]
             lib.oracle_quantize_tokens.argtypes = [P, I64, I64, I64, I, P, P]
             lib.oracle_epilogue_tokens.argtypes = [P, I64, I64, P, P, P, I, P]
+            lib.oracle_fold_codes_asym.argtypes = [P, I64, I64, P, I, P, P, P]
+            lib.oracle_rowsum.argtypes = [P, I64, I64, P]
+            lib.oracle_epilogue_asym.argtypes = [P, P, P, I64, I64, P, P, I, P]
             for f in ("oracle_calibrate", "oracle_params", "oracle_fold", "oracle_quantize",
-                      "oracle_matmul", "oracle_epilogue", "oracle_quantize_tokens", "oracle_epilogue_tokens"):
+                      "oracle_matmul", "oracle_epilogue", "oracle_quantize_tokens", "oracle_epilogue_tokens",
+                      "oracle_fold_codes_asym", "oracle_rowsum", "oracle_epilogue_asym"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -205,4 +213,40 @@ def epilogue_tokens(acc: np.ndarray, s_tok: np.ndarray, sw: np.ndarray, bias: np
     y = np.empty((M, N), np.uint16)
     _load().oracle_epilogue_tokens(_ptr(acc), M, N, _ptr(_f32(s_tok)), _ptr(_f32(sw)), _ptr(_f32(bias)),
                                    1 if relu else 0, _ptr(y))
+    return y.view(np.float16)
+
+
+def fold_codes_asym(w: np.ndarray, s: np.ndarray | None, bits_w: int):
+    """Asymmetric per-output-channel codes of W_s = W (.) s (R9; s None: s = 1).
+    Returns (qw int8 [N, K] stored as u - 2^(b-1), sw fp32 [N], zc int32 [N])."""
+    w = _f16(w)
+    N, K = w.shape
+    ss = None if s is None else _f32(s)
+    qw = np.empty((N, K), np.int8)
+    sw = np.empty(N, np.float32)
+    zc = np.empty(N, np.int32)
+    _load().oracle_fold_codes_asym(_ptr(w), N, K, None if ss is None else _ptr(ss), bits_w, _ptr(qw), _ptr(sw),
+                                   _ptr(zc))
+    return qw, sw, zc
+
+
+def rowsum(q: np.ndarray) -> np.ndarray:
+    """int64 rs[m] = sum_k q[m, k]."""
+    q = np.ascontiguousarray(q, dtype=np.int8)
+    M, K = q.shape
+    rs = np.empty(M, np.int64)
+    _load().oracle_rowsum(_ptr(q), M, K, _ptr(rs))
+    return rs
+
+
+def epilogue_asym(acc: np.ndarray, rs: np.ndarray, zc: np.ndarray, sw: np.ndarray, bfold: np.ndarray,
+                  relu: bool = False) -> np.ndarray:
+    """fp16 Y[M, N] = fp16(fma((float)(acc - zc_n rs_m), sw_n, b'_n)), optional ReLU."""
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
+    rs = np.ascontiguousarray(rs, dtype=np.int64)
+    zc = np.ascontiguousarray(zc, dtype=np.int32)
+    M, N = acc.shape
+    y = np.empty((M, N), np.uint16)
+    _load().oracle_epilogue_asym(_ptr(acc), _ptr(rs), _ptr(zc), M, N, _ptr(_f32(sw)), _ptr(_f32(bfold)),
+                                 1 if relu else 0, _ptr(y))
     return y.view(np.float16)

@@ -39,6 +39,14 @@
  *                fp32 fused multiply-add (one rounding), the result is
  *                rounded once to fp16 (half to even, overflow to +-inf);
  *                optional ReLU before the fp16 rounding.
+ *   R9 Int8      the asymmetric weights ("Int8", Section 4 / Appendix A:
+ *                zero points for the weights, min-max calibration) apply
+ *                Eq. 1 to each row of W_s over the range [min(0, min),
+ *                max(0, max)] (so 0 is exactly representable), with
+ *                s = range / (2^b - 1), zero point round(-min * r) and codes
+ *                clip(round(w * r) + zp, 0, 2^b - 1); NaN codes to the zero
+ *                point.  Codes and zero points are stored shifted by
+ *                -2^(b-1) so they fit int8.
  *
  * Floating point: compile with -ffp-contract=off and no fast-math, so every
  * fp32 expression below rounds once per operation as written.
@@ -304,6 +312,95 @@ void oracle_epilogue_tokens(const int64_t *acc, int64_t M, int64_t N, const floa
             float a = (float)acc[m * N + n];
             float scale = s_tok[m] * sw[n];
             float v = fmaf(a, scale, bias[n]);
+            if (relu && !(v > 0.0f)) v = 0.0f;
+            y[m * N + n] = ot_double_to_half((double)v);
+        }
+}
+
+/* ---------------------------------------------------------------------------
+ * Asymmetric per-output-channel weights ("Int8", R9; Eq. 1 with z != 0).
+ *
+ * Step A3': Eq. 1 on each row of W_s = W (.) s^X (Eq. 5):
+ *   lo_n = min(0, min_k W_s[n,k]),  hi_n = max(0, max_k W_s[n,k])
+ *   sw_n = (hi_n - lo_n) / (2^b - 1),  rw_n = (2^b - 1) / (hi_n - lo_n)   (R2)
+ *   zp_n = clip(round(-lo_n * rw_n), 0, 2^b - 1)
+ *   u[n,k] = clip(round(W_s[n,k] * rw_n) + zp_n, 0, 2^b - 1)
+ * so that W_s[n,k] ~ (u[n,k] - zp_n) * sw_n.  Stored shifted by -2^(b-1):
+ *   qw[n,k] = u[n,k] - 2^(b-1),  zc_n = zp_n - 2^(b-1),  W_s ~ (qw - zc) sw.
+ * A row whose range is 0 or not finite gets sw = 0 and every code equal to
+ * its zero point (dequantizing to 0).  s may be NULL (s_k = 1).
+ * ------------------------------------------------------------------------- */
+static int asym_code(float u, int zp, int umax)
+{
+    int c;
+    if (u != u) {
+        c = 0;                                /* NaN: the zero point */
+    } else {
+        float r = nearbyintf(u);              /* R1 */
+        if (r > (float)umax) c = umax;        /* the clip below decides */
+        else if (r < -(float)umax) c = -umax;
+        else c = (int)r;
+    }
+    c += zp;
+    return c < 0 ? 0 : (c > umax ? umax : c);
+}
+
+void oracle_fold_codes_asym(const uint16_t *w, int64_t N, int64_t K, const float *s,
+                            int bits_w, int8_t *qw, float *sw, int32_t *zc)
+{
+    const int umax = (1 << bits_w) - 1;
+    const int shift = 1 << (bits_w - 1);
+    for (int64_t n = 0; n < N; ++n) {
+        const uint16_t *wrow = w + n * K;
+        float lo = 0.0f, hi = 0.0f;
+        for (int64_t k = 0; k < K; ++k) {
+            float ws = ot_half_to_float(wrow[k]) * (s ? s[k] : 1.0f);
+            if (ws < lo) lo = ws;               /* NaN compares false */
+            if (ws > hi) hi = ws;
+        }
+        float range = hi - lo;
+        float swn = 0.0f, rwn = 0.0f;
+        int zp = 0;
+        if (range > 0.0f && isfinite(range)) {
+            swn = range / (float)umax;
+            rwn = (float)umax / range;
+            zp = asym_code(-lo * rwn, 0, umax);
+        }
+        sw[n] = swn;
+        zc[n] = zp - shift;
+        for (int64_t k = 0; k < K; ++k) {
+            float ws = ot_half_to_float(wrow[k]) * (s ? s[k] : 1.0f);
+            qw[n * K + k] = (int8_t)(asym_code(ws * rwn, zp, umax) - shift);
+        }
+    }
+}
+
+/* Sum of each row's activation codes, rs[m] = sum_k q[m,k] (exact). */
+void oracle_rowsum(const int8_t *q, int64_t M, int64_t K, int64_t *rs)
+{
+    for (int64_t m = 0; m < M; ++m) {
+        int64_t t = 0;
+        for (int64_t k = 0; k < K; ++k) t += q[m * K + k];
+        rs[m] = t;
+    }
+}
+
+/* ---------------------------------------------------------------------------
+ * Step A6': external scaling with the weight zero point.  With
+ * acc[m,n] = sum_k q[m,k] qw[n,k] (Eq. 6 on the stored codes),
+ *   sum_k q[m,k] (qw[n,k] - zc_n) = acc[m,n] - zc_n * rs[m]   (exact, int64)
+ *   y[m,n] = fp16( fma((float)(acc[m,n] - zc_n rs[m]), sw_n, b'_n) )
+ * (R8 otherwise; ReLU before the fp16 rounding).
+ * ------------------------------------------------------------------------- */
+void oracle_epilogue_asym(const int64_t *acc, const int64_t *rs, const int32_t *zc,
+                          int64_t M, int64_t N, const float *sw, const float *bfold,
+                          int relu, uint16_t *y)
+{
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t n = 0; n < N; ++n) {
+            int64_t t = acc[m * N + n] - (int64_t)zc[n] * rs[m];
+            float a = (float)t;                    /* round to nearest even */
+            float v = fmaf(a, sw[n], bfold[n]);    /* one rounding */
             if (relu && !(v > 0.0f)) v = 0.0f;
             y[m * N + n] = ot_double_to_half((double)v);
         }
