@@ -201,6 +201,55 @@ ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int
                               void *stream);
 
 /*
+ * Asymmetric per-output-channel weights: the paper's "Int8" (Section 4,
+ * Appendix A: zero points for the weights, min-max calibration), which trades
+ * a little speed for accuracy against the symmetric "Int8*" of ot_fold_weights.
+ *
+ * ot_fold_weights_asym -- as ot_fold_weights (Eq. 5 fold, Eq. 7 bias), but each
+ * row of W_s = W (.) s is quantized with Eq. 1 and a zero point over the range
+ * [lo, hi] = [min(0, min_k W_s), max(0, max_k W_s)]:
+ *   sw_n = (hi - lo) / (2^b - 1),  rw_n = (2^b - 1) / (hi - lo)
+ *   zp_n = clip(round(-lo * rw_n), 0, 2^b - 1)
+ *   u = clip(round(W_s * rw_n) + zp_n, 0, 2^b - 1),   W_s ~ (u - zp_n) sw_n
+ * stored shifted so the codes fit int8:  qw = u - 2^(b-1),  zc_n = zp_n - 2^(b-1).
+ * A row whose range is 0 or not finite gets sw = 0 and codes equal to zc.
+ * Arguments as ot_fold_weights plus zc int32 [N] out (4-byte aligned).
+ */
+ot_status ot_fold_weights_asym(const float *ch_min, const float *ch_max, int bits_a,
+                               int symmetrize, const void *w_f16, const void *b_f16,
+                               int64_t N, int64_t K, int bits_w, float *z, float *s,
+                               float *r, int8_t *qw, float *sw, int32_t *zc,
+                               float *b_fold, void *stream);
+
+/*
+ * ot_quantize_act_rowsum -- ot_quantize_act plus the sum of each row's codes,
+ *   rowsum[m] = sum_k q[m,k]   (int32 [M], exact; 4-byte aligned),
+ * which the asymmetric-weight epilogue needs.  rowsum is cleared on `stream`
+ * before the codes are added (integer atomics, so the result is exact and
+ * independent of order).  K * qmax(bits_a) must be < 2^31.
+ */
+ot_status ot_quantize_act_rowsum(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
+                                 const float *z, const float *r, int bits_a, void *q,
+                                 int q_format, int32_t *rowsum, void *stream);
+
+/*
+ * ot_linear_asym -- the quantized linear with asymmetric weights:
+ *   acc[m,n] = sum_k q[m,k] * qw[n,k]                       exact integer
+ *   y[m,n]   = fp16( fma((float)(acc[m,n] - zc_n * rowsum[m]), sw_n, b'_n) )
+ * where acc - zc_n * rowsum_m = sum_k q[m,k] (qw[n,k] - zc_n) is formed exactly
+ * in 64-bit integers and rounded once to fp32; ReLU before the fp16 rounding.
+ * Arguments as ot_linear plus zc int32 [N] (from ot_fold_weights_asym) and
+ * rowsum int32 [M] (from ot_quantize_act_rowsum).  The stored codes reach
+ * -2^(bits_w-1), so K * qmax(bits_a) * 2^(bits_w-1) must be < 2^31 (K <= 132,104
+ * for 8-bit codes).
+ */
+ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
+                         const float *sw, const int32_t *zc, const int32_t *rowsum,
+                         const float *b_fold, int64_t N, int bits_a, int bits_w,
+                         void *y_f16, int64_t ldy, int relu, void *workspace,
+                         size_t workspace_bytes, void *stream);
+
+/*
  * ot_linear_noalloc -- ot_linear for callers that cannot allocate device
  * memory: for example a server or plugin that owns all GPU memory through
  * its own pool and forbids further cudaMalloc calls, or code that must not

@@ -38,6 +38,10 @@ _SIGNATURES = {
     "ot_quantize_weights": ([_P, _I64, _I64, _I, _P, _P, _P], _I),
     "ot_linear_per_token": ([_P, _I64, _I64, _P, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P],
                             _I),
+    "ot_fold_weights_asym": ([_P, _P, _I, _I, _P, _P, _I64, _I64, _I, _P, _P, _P, _P, _P, _P, _P, _P], _I),
+    "ot_quantize_act_rowsum": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _I, _P, _P], _I),
+    "ot_linear_asym": ([_P, _I64, _I64, _P, _P, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P],
+                       _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -151,6 +155,53 @@ def ot_quantize_act(x, z, r, bits_a: int, q, q_format: int = OT_CODE_F16, stream
                                   _dev(r, "r", torch.float32), bits_a, _dev(q, "q", want), q_format,
                                   _stream(stream)),
            "ot_quantize_act")
+
+
+def ot_fold_weights_asym(ch_min, ch_max, bits_a: int, w, b, bits_w: int, z, s, r, qw, sw, zc, b_fold,
+                         symmetrize: bool = True, stream=None):
+    """ot_fold_weights with asymmetric per-output-channel codes (the paper's "Int8"):
+    qw int8 [N, K] stored as u - 2^(b-1), zero points zc int32 [N]."""
+    _dense(w, "w")
+    N, K = w.shape
+    pb = None if b is None else _dev(b, "b", torch.float16)
+    _check(load().ot_fold_weights_asym(_dev(ch_min, "ch_min", torch.float32),
+                                       _dev(ch_max, "ch_max", torch.float32), bits_a, 1 if symmetrize else 0,
+                                       _dev(w, "w", torch.float16), pb, N, K, bits_w, _dev(z, "z", torch.float32),
+                                       _dev(s, "s", torch.float32), _dev(r, "r", torch.float32),
+                                       _dev(qw, "qw", torch.int8), _dev(sw, "sw", torch.float32),
+                                       _dev(zc, "zc", torch.int32), _dev(b_fold, "b_fold", torch.float32),
+                                       _stream(stream)),
+           "ot_fold_weights_asym")
+
+
+def ot_quantize_act_rowsum(x, z, r, bits_a: int, q, rowsum, q_format: int = OT_CODE_F16, stream=None):
+    """ot_quantize_act plus rowsum[m] = sum_k q[m, k] (int32 [M])."""
+    M, K, ldx = _rows(x, "x")
+    _dense(q, "q")
+    want = torch.float16 if q_format == OT_CODE_F16 else torch.int8
+    _check(load().ot_quantize_act_rowsum(_dev(x, "x", torch.float16), M, K, ldx, _dev(z, "z", torch.float32),
+                                         _dev(r, "r", torch.float32), bits_a, _dev(q, "q", want), q_format,
+                                         _dev(rowsum, "rowsum", torch.int32), _stream(stream)),
+           "ot_quantize_act_rowsum")
+
+
+def ot_linear_asym(q, qw, sw, zc, rowsum, b_fold, bits_a: int, bits_w: int, y, relu: bool = False,
+                   workspace=None, stream=None):
+    """y = fp16(fma((float)(acc - zc_n rowsum_m), sw_n, b'_n)) with asymmetric weight codes."""
+    _dense(q, "q")
+    _dense(qw, "qw")
+    M, K = q.shape
+    N = qw.shape[0]
+    ym, yn, ldy = _rows(y, "y")
+    if ym != M or yn != N:
+        raise ValueError("y must be [M, N]")
+    wp, wb = _ws_args(workspace, q.device, stream)
+    _check(load().ot_linear_asym(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8),
+                                 _dev(sw, "sw", torch.float32), _dev(zc, "zc", torch.int32),
+                                 _dev(rowsum, "rowsum", torch.int32), _dev(b_fold, "b_fold", torch.float32), N,
+                                 bits_a, bits_w, _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb,
+                                 _stream(stream)),
+           "ot_linear_asym")
 
 
 def ot_linear_workspace_size() -> int:

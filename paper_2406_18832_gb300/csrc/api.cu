@@ -81,6 +81,34 @@ ot_status ot_fold_weights(const float *ch_min, const float *ch_max, int bits_a, 
     return from_cuda(ot::launch_fold(w_f16, b_f16, N, K, z, s, bits_w, qw, sw, b_fold, st));
 }
 
+ot_status ot_fold_weights_asym(const float *ch_min, const float *ch_max, int bits_a, int symmetrize,
+                               const void *w_f16, const void *b_f16, int64_t N, int64_t K, int bits_w, float *z,
+                               float *s, float *r, int8_t *qw, float *sw, int32_t *zc, float *b_fold, void *stream) {
+    if (N < 0 || K <= 0 || K % 16 != 0 || !bits_ok(bits_a) || !bits_ok(bits_w)) return OT_ERR_INVALID_ARG;
+    if (!ch_min || !ch_max || !z || !s || !r || !sw || !b_fold) return OT_ERR_INVALID_ARG;
+    if (N > 0 && (!w_f16 || !qw || !zc || !aligned(w_f16, 16) || !aligned(qw, 16) || !aligned(zc, 4)))
+        return OT_ERR_INVALID_ARG;
+    if (b_f16 && !aligned(b_f16, 2)) return OT_ERR_INVALID_ARG;
+    cudaStream_t st = as_stream(stream);
+    cudaError_t e = ot::launch_params(ch_min, ch_max, K, bits_a, symmetrize, z, s, r, st);
+    if (e != cudaSuccess) return OT_ERR_CUDA;
+    return from_cuda(ot::launch_fold_asym(w_f16, b_f16, N, K, z, s, bits_w, qw, sw, zc, b_fold, st));
+}
+
+ot_status ot_quantize_act_rowsum(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z,
+                                 const float *r, int bits_a, void *q, int q_format, int32_t *rowsum,
+                                 void *stream) {
+    if (M < 0 || K <= 0 || K % 8 != 0 || ldx < K || ldx % 8 != 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;
+    if (q_format != OT_CODE_I8 && q_format != OT_CODE_F16) return OT_ERR_INVALID_ARG;
+    if (!z || !r || !aligned(z, 16) || !aligned(r, 16)) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!x_f16 || !q || !rowsum || !aligned(x_f16, 16) || !aligned(q, 16) || !aligned(rowsum, 4)))
+        return OT_ERR_INVALID_ARG;
+    if ((M + 63) / 64 > 65535) return OT_ERR_UNSUPPORTED;
+    if (K * qmax_of(bits_a) > kIntMax) return OT_ERR_UNSUPPORTED;  // int32 row sums
+    return from_cuda(
+        ot::launch_quantize(x_f16, M, K, ldx, z, r, bits_a, q, q_format, as_stream(stream), rowsum));
+}
+
 ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
                           int bits_a, void *q, int q_format, void *stream) {
     if (M < 0 || K <= 0 || K % 8 != 0 || ldx < K || ldx % 8 != 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;
@@ -149,6 +177,24 @@ ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int
     if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
     ot::LinearArgs a{q_f16, qw, sw, bias, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
                      workspace, workspace ? workspace_bytes : 0, s_tok};
+    return from_cuda(ot::launch_linear(a, as_stream(stream)));
+}
+
+ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw,
+                         const int32_t *zc, const int32_t *rowsum, const float *b_fold, int64_t N, int bits_a,
+                         int bits_w, void *y_f16, int64_t ldy, int relu, void *workspace, size_t workspace_bytes,
+                         void *stream) {
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
+    if (v != OT_OK) return v;
+    if (!sw || !b_fold || !zc || !aligned(zc, 4) || ldy < N || (y_f16 && !aligned(y_f16, 2)))
+        return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!rowsum || !aligned(rowsum, 4))) return OT_ERR_INVALID_ARG;
+    if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
+    if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
+    // the stored asymmetric codes reach -2^(bits_w - 1)
+    if (K * qmax_of(bits_a) * (qmax_of(bits_w) + 1) > kIntMax) return OT_ERR_UNSUPPORTED;
+    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+                     workspace, workspace ? workspace_bytes : 0, nullptr, zc, rowsum};
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 

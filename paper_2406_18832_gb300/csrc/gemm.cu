@@ -94,11 +94,12 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     hi = *reinterpret_cast<const uint32_t *>(&hb);
 }
 
-template <int BN, bool kS32>
+template <int BN, bool kS32, bool kAsym>
 __global__ void __launch_bounds__(kThreads, 1)
     linear_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                   const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
-                  int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok) {
+                  int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok,
+                  const int32_t *__restrict__ zc, const int32_t *__restrict__ rowsum) {
     extern __shared__ uint8_t smem_raw[];
     Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -269,13 +270,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
+                    const long long zn = kAsym ? (long long)__ldg(zc + n) : 0;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
                     for (int j = 0; j < CPW; ++j) {
                         const int m = m0 + col0 + j;
+                        const int mc = m < M ? m : M - 1;
                         // per-token path (Eq. 3): one fp32 product s_m * sw_n
-                        const float sc = s_tok ? __fmul_rn(__ldg(s_tok + (m < M ? m : M - 1)), scale) : scale;
-                        float v = __fmaf_rn(__int2float_rn(tot[j]), sc, bias);
+                        const float sc = s_tok ? __fmul_rn(__ldg(s_tok + mc), scale) : scale;
+                        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m, exact in int64
+                        const float a = kAsym ? __ll2float_rn((long long)tot[j] - zn * __ldg(rowsum + mc))
+                                           : __int2float_rn(tot[j]);
+                        float v = __fmaf_rn(a, sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
                         if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
                     }
@@ -410,12 +416,13 @@ __device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) 
     return v;
 }
 
-template <bool kS32>
+template <bool kS32, bool kAsym>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
                        int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws, uint64_t epoch,
-                       const float *__restrict__ s_tok) {
+                       const float *__restrict__ s_tok, const int32_t *__restrict__ zc,
+                       const int32_t *__restrict__ rowsum) {
     extern __shared__ uint8_t smem_raw[];
     SmemPair &S = *reinterpret_cast<SmemPair *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -645,13 +652,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     }
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
+                    const long long zn = kAsym ? (long long)__ldg(zc + n) : 0;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
                     for (int j = 0; j < 128; ++j) {
                         const int m = m0 + col0 + j;
+                        const int mc = m < M ? m : M - 1;
                         // per-token path (Eq. 3): one fp32 product s_m * sw_n
-                        const float sc = s_tok ? __fmul_rn(__ldg(s_tok + (m < M ? m : M - 1)), scale) : scale;
-                        float v = __fmaf_rn(__int2float_rn(tot[j]), sc, bias);
+                        const float sc = s_tok ? __fmul_rn(__ldg(s_tok + mc), scale) : scale;
+                        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m, exact in int64
+                        const float a = kAsym ? __ll2float_rn((long long)tot[j] - zn * __ldg(rowsum + mc))
+                                           : __int2float_rn(tot[j]);
+                        float v = __fmaf_rn(a, sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
                         if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
                     }
@@ -712,7 +724,7 @@ bool make_tmap_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uin
     return r == CUDA_SUCCESS;
 }
 
-template <int BN, bool kS32>
+template <int BN, bool kS32, bool kAsym>
 cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
     if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
@@ -725,14 +737,15 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32, kAsym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
-    linear_kernel<BN, kS32><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
-                                                         (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok);
+    linear_kernel<BN, kS32, kAsym><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
+                                                         (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
+                                                         a.rowsum);
     return cudaGetLastError();
 }
 
@@ -746,7 +759,7 @@ int pair_max_clusters() {
     if (dev_cached == dev) return value;
     const size_t smem = sizeof(SmemPair) + 1024;
     int n = 0;
-    if (cudaFuncSetAttribute(linear_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+    if (cudaFuncSetAttribute(linear_pair_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
         cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 256);
@@ -759,7 +772,7 @@ int pair_max_clusters() {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<false>, &cfg) != cudaSuccess) n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<false, false>, &cfg) != cudaSuccess) n = 0;
     }
     cudaGetLastError();
     if (n <= 0) n = num_sms() / 2;
@@ -768,7 +781,7 @@ int pair_max_clusters() {
     return n;
 }
 
-template <bool kS32>
+template <bool kS32, bool kAsym>
 cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
     if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
@@ -780,7 +793,7 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32, kAsym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
@@ -799,19 +812,18 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
     const uint64_t epoch = streamk ? next_epoch() : 0;
-    linear_pair_kernel<kS32><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
+    linear_pair_kernel<kS32, kAsym><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
                                                                 (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
-                                                                epoch, a.s_tok);
+                                                                epoch, a.s_tok, a.zc, a.rowsum);
     return cudaGetLastError();
 }
 
-template <bool kS32>
+// M <= 32 goes to the decode kernel (gemv.cu) before this dispatch.
+template <bool kS32, bool kAsym>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
-    if (a.M <= 16) return run_linear<16, kS32>(a, kcb, st);
-    if (a.M <= 32) return run_linear<32, kS32>(a, kcb, st);
-    if (a.M <= 64) return run_linear<64, kS32>(a, kcb, st);
-    if (a.M <= 128) return run_linear<128, kS32>(a, kcb, st);
-    return run_linear_pair<kS32>(a, kcb, st);
+    if (a.M <= 64) return run_linear<64, kS32, kAsym>(a, kcb, st);
+    if (a.M <= 128) return run_linear<128, kS32, kAsym>(a, kcb, st);
+    return run_linear_pair<kS32, kAsym>(a, kcb, st);
 }
 
 }  // namespace
@@ -828,8 +840,9 @@ constexpr int64_t kGemvMaxTokens = 32;
 
 // Largest number of 64-wide k-blocks whose fp32 partial sums stay exact:
 // kcb * 64 * qmax_a * qmax_w <= 2^24.
-int exact_chunk_kblocks(int bits_a, int bits_w) {
-    const int64_t qa = (1 << (bits_a - 1)) - 1, qw = (1 << (bits_w - 1)) - 1;
+int exact_chunk_kblocks(int bits_a, int bits_w, bool asym_w) {
+    // asymmetric weight codes are stored as u - 2^(b-1): |qw| <= 2^(b-1)
+    const int64_t qa = (1 << (bits_a - 1)) - 1, qw = (1 << (bits_w - 1)) - (asym_w ? 0 : 1);
     int64_t kc = ((int64_t)1 << 24) / (qa * qw);
     kc /= kBK;
     return kc < 1 ? 1 : (int)kc;
@@ -888,7 +901,7 @@ cudaError_t noalloc_scratch(void **ptr, cudaStream_t st) {
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
     if (a.M == 0 || a.N == 0) return cudaSuccess;
     const int nkb = (int)((a.K + kBK - 1) / kBK);
-    int kcb = exact_chunk_kblocks(a.bits_a, a.bits_w);
+    int kcb = exact_chunk_kblocks(a.bits_a, a.bits_w, a.zc != nullptr);
     if (kcb > nkb) kcb = nkb;
     if (a.M <= kGemvMaxTokens) {
         LinearArgs d = a;
@@ -898,7 +911,8 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
         d.workspace_bytes = room ? a.workspace_bytes - off : 0;
         return launch_linear_gemv(d, kcb, st);
     }
-    return a.out_s32 ? dispatch_bn<true>(a, kcb, st) : dispatch_bn<false>(a, kcb, st);
+    if (a.out_s32) return dispatch_bn<true, false>(a, kcb, st);
+    return a.zc ? dispatch_bn<false, true>(a, kcb, st) : dispatch_bn<false, false>(a, kcb, st);
 }
 
 }  // namespace ot

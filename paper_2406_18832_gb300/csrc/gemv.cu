@@ -68,6 +68,7 @@ constexpr int kGvSlotInts = kGvRows * 32;         // workspace ints per split ti
 
 struct GvParams {
     const float *sw, *bfold, *s_tok;
+    const int32_t *zc, *rowsum;    // asymmetric weights: zero points [N], code row sums [M] (or null)
     void *out;
     int32_t *part;                 // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
     unsigned long long *flags;     // [grid] launch epoch once a CTA's slot is complete
@@ -125,7 +126,10 @@ __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32
     } else {
         const float scale = __ldg(p.sw + n);
         const float sc = p.s_tok ? __fmul_rn(__ldg(p.s_tok + m), scale) : scale;  // per-token path (Eq. 3)
-        float v = __fmaf_rn(__int2float_rn(s), sc, __ldg(p.bfold + n));
+        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m, exact in int64
+        const float a = p.zc ? __ll2float_rn((long long)s - (long long)__ldg(p.zc + n) * __ldg(p.rowsum + m))
+                             : __int2float_rn(s);
+        float v = __fmaf_rn(a, sc, __ldg(p.bfold + n));
         if (p.relu) v = fmaxf(v, 0.f);
         reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = __float2half_rn(v);
     }
@@ -415,6 +419,8 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     p.sw = a.sw;
     p.bfold = a.bfold;
     p.s_tok = a.s_tok;
+    p.zc = a.zc;
+    p.rowsum = a.rowsum;
     p.out = a.out;
     p.status = device_status_word();
     if (!p.status) return cudaErrorUnknown;

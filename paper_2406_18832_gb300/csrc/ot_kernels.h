@@ -16,10 +16,14 @@ cudaError_t launch_params(const float *mn, const float *mx, int64_t K, int bits,
                           float *s, float *r, cudaStream_t st);
 cudaError_t launch_fold(const void *w, const void *b, int64_t N, int64_t K, const float *z, const float *s,
                         int bits_w, int8_t *qw, float *sw, float *bfold, cudaStream_t st);
+// rowsum (optional, int32 [M]): sum_k q[m,k], for the asymmetric-weight epilogue
 cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
-                            int bits, void *q, int fmt, cudaStream_t st);
+                            int bits, void *q, int fmt, cudaStream_t st, int32_t *rowsum = nullptr);
 cudaError_t launch_quantize_tokens(const void *x, int64_t M, int64_t K, int64_t ldx, int bits, void *q, int fmt,
                                    float *s_tok, cudaStream_t st);
+// asymmetric per-output-channel codes of W_s (zero points zc) and b'
+cudaError_t launch_fold_asym(const void *w, const void *b, int64_t N, int64_t K, const float *z, const float *s,
+                             int bits_w, int8_t *qw, float *sw, int32_t *zc, float *bfold, cudaStream_t st);
 // per-output-channel weight codes without activation scales (s = 1)
 cudaError_t launch_quantize_weights(const void *w, int64_t N, int64_t K, int bits_w, int8_t *qw, float *sw,
                                     cudaStream_t st);
@@ -36,6 +40,8 @@ struct LinearArgs {
     void *workspace;          // stream-K partial sums (zero-filled before first use) or null
     size_t workspace_bytes;
     const float *s_tok;       // per-token path: token scales [M] (y uses s_tok[m] * sw[n]); null otherwise
+    const int32_t *zc;        // asymmetric weights: zero points [N] (stored codes' scale), or null
+    const int32_t *rowsum;    // with zc: sum_k q[m,k] [M]
 };
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();
@@ -58,7 +64,7 @@ bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, ui
                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz);
 
 int num_sms();
-int exact_chunk_kblocks(int bits_a, int bits_w);
+int exact_chunk_kblocks(int bits_a, int bits_w, bool asym_w);
 cudaError_t read_clear_status(int *value, cudaStream_t st);
 cudaError_t launch_wait_timeout(int64_t limit_ns, cudaStream_t st);
 

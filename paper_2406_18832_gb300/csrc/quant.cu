@@ -39,16 +39,20 @@ __device__ __forceinline__ uint32_t pack_i8_codes(int c0, int c1, int c2, int c3
 
 // Block 32 x 8: threadIdx.x owns 8 consecutive channels of a 256-channel
 // strip (blockIdx.x) and keeps their z, r in registers while it walks
-// kQRowsPerThread rows of the block's row range (blockIdx.y).
-template <bool kF16Out>
+// kQRowsPerThread rows of the block's row range (blockIdx.y).  With kRowSum
+// the warp also adds its 256 codes of each row and one lane adds that into
+// rowsum[m] (integer atomics: exact, order-free; rowsum starts at 0).
+template <bool kF16Out, bool kRowSum>
 __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict__ x, int64_t M, int64_t K,
                                                        int64_t ldx, const float *__restrict__ z,
-                                                       const float *__restrict__ r, int qmax, void *q) {
+                                                       const float *__restrict__ r, int qmax, void *q,
+                                                       int32_t *rowsum) {
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int64_t c0 = (int64_t)blockIdx.x * 256 + tx * 8;
-    if (c0 >= K) return;
-    float zz[8], rr[8];
-    {
+    const bool active = c0 < K;  // K % 8 == 0: a lane's 8 channels are whole or absent
+    if (!kRowSum && !active) return;
+    float zz[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f}, rr[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (active) {
         const float4 *zp = reinterpret_cast<const float4 *>(z + c0);
         const float4 *rp = reinterpret_cast<const float4 *>(r + c0);
         float4 a = __ldg(zp), b = __ldg(zp + 1), c = __ldg(rp), d = __ldg(rp + 1);
@@ -60,12 +64,13 @@ __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict_
 #pragma unroll
     for (int u = 0; u < kQRowsPerThread; ++u) {
         const int64_t m = row0 + 8 * u;
-        if (m < M) v[u] = __ldcs(reinterpret_cast<const uint4 *>(x + m * ldx + c0));
+        v[u] = make_uint4(0, 0, 0, 0);
+        if (m < M && active) v[u] = __ldcs(reinterpret_cast<const uint4 *>(x + m * ldx + c0));
     }
 #pragma unroll
     for (int u = 0; u < kQRowsPerThread; ++u) {
         const int64_t m = row0 + 8 * u;
-        if (m >= M) break;
+        if (m >= M) break;  // uniform over the warp
         const __half2 *h = reinterpret_cast<const __half2 *>(&v[u]);
         int c[8];
 #pragma unroll
@@ -74,6 +79,15 @@ __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict_
             c[2 * j] = code_of(f.x, zz[2 * j], rr[2 * j], qmax);
             c[2 * j + 1] = code_of(f.y, zz[2 * j + 1], rr[2 * j + 1], qmax);
         }
+        if (kRowSum) {
+            int t = 0;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) t += c[j];  // inactive lanes: codes of 0 * 0 = 0
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            if (tx == 0) atomicAdd(rowsum + m, t);
+        }
+        if (!active) continue;
         if (kF16Out) {
             uint4 o;
             o.x = pack_f16_codes(c[0], c[1]);
@@ -164,14 +178,23 @@ cudaError_t launch_quantize_tokens(const void *x, int64_t M, int64_t K, int64_t 
 }
 
 cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
-                            int bits, void *q, int fmt, cudaStream_t st) {
+                            int bits, void *q, int fmt, cudaStream_t st, int32_t *rowsum) {
     if (M == 0) return cudaSuccess;
     const int qmax = (1 << (bits - 1)) - 1;
     dim3 grid((unsigned)((K + 255) / 256), (unsigned)((M + kQRowsPerBlock - 1) / kQRowsPerBlock));
-    if (fmt == OT_CODE_F16)
-        quantize_kernel<true><<<grid, 256, 0, st>>>(reinterpret_cast<const __half *>(x), M, K, ldx, z, r, qmax, q);
-    else
-        quantize_kernel<false><<<grid, 256, 0, st>>>(reinterpret_cast<const __half *>(x), M, K, ldx, z, r, qmax, q);
+    const __half *xh = reinterpret_cast<const __half *>(x);
+    if (rowsum) {
+        cudaError_t e = cudaMemsetAsync(rowsum, 0, (size_t)M * sizeof(int32_t), st);
+        if (e != cudaSuccess) return e;
+        if (fmt == OT_CODE_F16)
+            quantize_kernel<true, true><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, rowsum);
+        else
+            quantize_kernel<false, true><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, rowsum);
+    } else if (fmt == OT_CODE_F16) {
+        quantize_kernel<true, false><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, nullptr);
+    } else {
+        quantize_kernel<false, false><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, nullptr);
+    }
     return cudaGetLastError();
 }
 
