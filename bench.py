@@ -345,6 +345,7 @@ def run_ours(args):
 
     block = None if args.no_block else bench_block(dev)
     decode = bench_decode(dev, peaks)
+    asym = bench_asym(dev, layers, xs, ops_step, ms_per_step)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -387,12 +388,66 @@ def run_ours(args):
                    "ratio": round(weights_fp16 / weights_int8, 3)},
         "block": block,
         "decode": decode,
+        "asym_weights": asym,
         "cpu_baseline": cpu,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 8192):
+    """The same OPT-6.7B prefill step with the paper's "Int8" weights
+    (per-output-channel zero points): quantize with code row sums, then the
+    linear whose epilogue subtracts zc_n * rowsum_m.  Calibrated on 8192
+    tokens of the same synthetic stream as the main line."""
+    import torch
+
+    from paper_2406_18832_gb300 import QuantizedLinear, synth
+    cfg = synth.CONFIGS[WORKLOAD_CFG]
+    qls = []
+    for li, (layer, (ql_sym, w, b)) in enumerate(zip(cfg.layers, layers)):
+        ql = QuantizedLinear(layer.K, layer.N, ql_sym.bits_a, ql_sym.bits_w, relu=layer.relu_out, device=dev,
+                             weights="asym")
+        ql.calibrate(synth.activations(WORKLOAD_CFG, li, layer, t_cal, 3, device=dev)).fold(w, b)
+        qls.append(ql)
+    qb = [torch.empty(TOKENS, ql.K, dtype=torch.float16, device=dev) for ql in qls]
+    rb = [torch.empty(TOKENS, dtype=torch.int32, device=dev) for _ in qls]
+    yb = [torch.empty(TOKENS, ql.N, dtype=torch.float16, device=dev) for ql in qls]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in qls]
+    gemm_ms = [0.0] * len(qls)
+
+    def step(timed=False):
+        for i, ql in enumerate(qls):
+            if timed:
+                evs[i][0].record()
+            ql.quantize_with_rowsum(xs[i], qb[i], rb[i])
+            if timed:
+                evs[i][1].record()
+            ql.linear(qb[i], yb[i], rowsum=rb[i])
+            if timed:
+                evs[i][2].record()
+
+    for _ in range(5):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    for _ in range(20):
+        step(timed=True)
+        torch.cuda.synchronize()
+        for i in range(len(qls)):
+            gemm_ms[i] += evs[i][1].elapsed_time(evs[i][2]) / 20
+    return {"workload": "opt-6.7b-linears-prefill, Int8 weights with zero points", "tokens": TOKENS,
+            "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
+            "over_symmetric_step": round(ms / ms_sym, 4),
+            "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
 
 
 def bench_decode(dev, peaks, reps: int = 50):

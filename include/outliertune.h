@@ -236,12 +236,12 @@ ot_status ot_quantize_act_rowsum(const void *x_f16, int64_t M, int64_t K, int64_
  * ot_linear_asym -- the quantized linear with asymmetric weights:
  *   acc[m,n] = sum_k q[m,k] * qw[n,k]                       exact integer
  *   y[m,n]   = fp16( fma((float)(acc[m,n] - zc_n * rowsum[m]), sw_n, b'_n) )
- * where acc - zc_n * rowsum_m = sum_k q[m,k] (qw[n,k] - zc_n) is formed exactly
- * in 64-bit integers and rounded once to fp32; ReLU before the fp16 rounding.
+ where acc - zc_n * rowsum_m = sum_k q[m,k] (qw[n,k] - zc_n) is formed exactly
+ * in integers and rounded once to fp32; ReLU before the fp16 rounding.
  * Arguments as ot_linear plus zc int32 [N] (from ot_fold_weights_asym) and
- * rowsum int32 [M] (from ot_quantize_act_rowsum).  The stored codes reach
- * -2^(bits_w-1), so K * qmax(bits_a) * 2^(bits_w-1) must be < 2^31 (K <= 132,104
- * for 8-bit codes).
+ * rowsum int32 [M] (from ot_quantize_act_rowsum).  |qw - zc| reaches
+ * 2^bits_w - 1, so K * qmax(bits_a) * (2^bits_w - 1) must be < 2^31 (K <= 66,313
+ * for W8A8; OT_ERR_UNSUPPORTED beyond).
  */
 ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
                          const float *sw, const int32_t *zc, const int32_t *rowsum,

@@ -191,8 +191,9 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
     if (M > 0 && (!rowsum || !aligned(rowsum, 4))) return OT_ERR_INVALID_ARG;
     if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
     if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
-    // the stored asymmetric codes reach -2^(bits_w - 1)
-    if (K * qmax_of(bits_a) * (qmax_of(bits_w) + 1) > kIntMax) return OT_ERR_UNSUPPORTED;
+    // the corrected sum, sum_k q (qw - zc) with |qw - zc| <= 2^bits_w - 1, must fit int32
+    // (it bounds the stored codes' sum too: |qw| <= 2^(bits_w - 1))
+    if (K * qmax_of(bits_a) * (2 * qmax_of(bits_w) + 1) > kIntMax) return OT_ERR_UNSUPPORTED;
     ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
                      workspace, workspace ? workspace_bytes : 0, nullptr, zc, rowsum};
     return from_cuda(ot::launch_linear(a, as_stream(stream)));

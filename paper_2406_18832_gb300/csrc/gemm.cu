@@ -270,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
-                    const long long zn = kAsym ? (long long)__ldg(zc + n) : 0;
+                    const int32_t zn = kAsym ? __ldg(zc + n) : 0;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
                     for (int j = 0; j < CPW; ++j) {
@@ -278,9 +278,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int mc = m < M ? m : M - 1;
                         // per-token path (Eq. 3): one fp32 product s_m * sw_n
                         const float sc = s_tok ? __fmul_rn(__ldg(s_tok + mc), scale) : scale;
-                        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m, exact in int64
-                        const float a = kAsym ? __ll2float_rn((long long)tot[j] - zn * __ldg(rowsum + mc))
-                                           : __int2float_rn(tot[j]);
+                        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m; the
+                        // entry point bounds it below 2^31, so int32 arithmetic (wrapping in between)
+                        // gives it exactly
+                        const float a = __int2float_rn(kAsym ? (int32_t)((uint32_t)tot[j] -
+                                                                          (uint32_t)zn * (uint32_t)__ldg(rowsum + mc))
+                                                             : tot[j]);
                         float v = __fmaf_rn(a, sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
                         if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
@@ -652,7 +655,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     }
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
-                    const long long zn = kAsym ? (long long)__ldg(zc + n) : 0;
+                    const int32_t zn = kAsym ? __ldg(zc + n) : 0;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
                     for (int j = 0; j < 128; ++j) {
@@ -660,9 +663,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         const int mc = m < M ? m : M - 1;
                         // per-token path (Eq. 3): one fp32 product s_m * sw_n
                         const float sc = s_tok ? __fmul_rn(__ldg(s_tok + mc), scale) : scale;
-                        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m, exact in int64
-                        const float a = kAsym ? __ll2float_rn((long long)tot[j] - zn * __ldg(rowsum + mc))
-                                           : __int2float_rn(tot[j]);
+                        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m; the
+                        // entry point bounds it below 2^31, so int32 arithmetic (wrapping in between)
+                        // gives it exactly
+                        const float a = __int2float_rn(kAsym ? (int32_t)((uint32_t)tot[j] -
+                                                                          (uint32_t)zn * (uint32_t)__ldg(rowsum + mc))
+                                                             : tot[j]);
                         float v = __fmaf_rn(a, sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
                         if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);

@@ -126,9 +126,10 @@ __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32
     } else {
         const float scale = __ldg(p.sw + n);
         const float sc = p.s_tok ? __fmul_rn(__ldg(p.s_tok + m), scale) : scale;  // per-token path (Eq. 3)
-        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m, exact in int64
-        const float a = p.zc ? __ll2float_rn((long long)s - (long long)__ldg(p.zc + n) * __ldg(p.rowsum + m))
-                             : __int2float_rn(s);
+        // asymmetric weights: sum_k q (qw - zc_n) = acc - zc_n * rowsum_m; the entry point
+        // bounds it below 2^31, so int32 arithmetic (wrapping in between) gives it exactly
+        const float a = __int2float_rn(
+            p.zc ? (int32_t)((uint32_t)s - (uint32_t)__ldg(p.zc + n) * (uint32_t)__ldg(p.rowsum + m)) : s);
         float v = __fmaf_rn(a, sc, __ldg(p.bfold + n));
         if (p.relu) v = fmaxf(v, 0.f);
         reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = __float2half_rn(v);

@@ -7,6 +7,11 @@ Offline (Section 3.2 "predetermined offline"; Appendix A):
 Online (Eq. 6, Eq. 7):
     forward(x) = ot_linear(ot_quantize_act(x))
 
+weights="asym" selects the paper's "Int8" weights (per-output-channel zero
+points; Section 4, Appendix A): the fold also yields zero points zc, the
+quantize step also yields each token's code sum, and the linear subtracts
+zc_n * rowsum_m before the external scaling.
+
 Every step is one call through the C ABI (binding.py); this class only owns
 the device tensors and the stream order.
 """
@@ -19,10 +24,13 @@ from . import binding as B
 
 class QuantizedLinear:
     def __init__(self, in_features: int, out_features: int, bits_a: int = 8, bits_w: int = 8,
-                 symmetrize: bool = True, relu: bool = False, device="cuda"):
+                 symmetrize: bool = True, relu: bool = False, device="cuda", weights: str = "sym"):
+        if weights not in ("sym", "asym"):
+            raise ValueError("weights must be 'sym' (Int8*) or 'asym' (Int8 with zero points)")
         self.K, self.N = in_features, out_features
         self.bits_a, self.bits_w = bits_a, bits_w
         self.symmetrize, self.relu = symmetrize, relu
+        self.asym = weights == "asym"
         dev = torch.device(device)
         f32 = dict(dtype=torch.float32, device=dev)
         self.ch_min = torch.empty(self.K, **f32)
@@ -33,6 +41,7 @@ class QuantizedLinear:
         self.qw = torch.empty(self.N, self.K, dtype=torch.int8, device=dev)
         self.sw = torch.empty(self.N, **f32)
         self.b_fold = torch.empty(self.N, **f32)
+        self.zc = torch.empty(self.N, dtype=torch.int32, device=dev) if self.asym else None
         self._calibrated = False
 
     # ---- offline --------------------------------------------------------
@@ -46,8 +55,13 @@ class QuantizedLinear:
         """Derive z, s, r from the calibration and fold them into W and b."""
         if not self._calibrated:
             raise RuntimeError("calibrate() before fold()")
-        B.ot_fold_weights(self.ch_min, self.ch_max, self.bits_a, w, b, self.bits_w, self.z, self.s, self.r,
-                          self.qw, self.sw, self.b_fold, symmetrize=self.symmetrize, stream=stream)
+        if self.asym:
+            B.ot_fold_weights_asym(self.ch_min, self.ch_max, self.bits_a, w, b, self.bits_w, self.z, self.s,
+                                   self.r, self.qw, self.sw, self.zc, self.b_fold, symmetrize=self.symmetrize,
+                                   stream=stream)
+        else:
+            B.ot_fold_weights(self.ch_min, self.ch_max, self.bits_a, w, b, self.bits_w, self.z, self.s, self.r,
+                              self.qw, self.sw, self.b_fold, symmetrize=self.symmetrize, stream=stream)
         return self
 
     # ---- online ---------------------------------------------------------
@@ -57,22 +71,43 @@ class QuantizedLinear:
         B.ot_quantize_act(x, self.z, self.r, self.bits_a, out, B.OT_CODE_F16, stream=stream)
         return out
 
-    def linear(self, q: torch.Tensor, out: torch.Tensor | None = None, stream=None):
+    def quantize_with_rowsum(self, x: torch.Tensor, out: torch.Tensor | None = None,
+                             rowsum: torch.Tensor | None = None, stream=None):
+        """Codes and each token's code sum (int32 [M]), for the asymmetric weights."""
+        if out is None:
+            out = torch.empty(x.shape[0], self.K, dtype=torch.float16, device=x.device)
+        if rowsum is None:
+            rowsum = torch.empty(x.shape[0], dtype=torch.int32, device=x.device)
+        B.ot_quantize_act_rowsum(x, self.z, self.r, self.bits_a, out, rowsum, B.OT_CODE_F16, stream=stream)
+        return out, rowsum
+
+    def linear(self, q: torch.Tensor, out: torch.Tensor | None = None, stream=None,
+               rowsum: torch.Tensor | None = None):
         if out is None:
             out = torch.empty(q.shape[0], self.N, dtype=torch.float16, device=q.device)
-        B.ot_linear(q, self.qw, self.sw, self.b_fold, self.bits_a, self.bits_w, out, relu=self.relu,
-                    stream=stream)
+        if self.asym:
+            if rowsum is None:
+                raise ValueError("asymmetric weights need the codes' row sums (quantize_with_rowsum)")
+            B.ot_linear_asym(q, self.qw, self.sw, self.zc, rowsum, self.b_fold, self.bits_a, self.bits_w, out,
+                             relu=self.relu, stream=stream)
+        else:
+            B.ot_linear(q, self.qw, self.sw, self.b_fold, self.bits_a, self.bits_w, out, relu=self.relu,
+                        stream=stream)
         return out
 
     def forward(self, x: torch.Tensor, q_buf: torch.Tensor | None = None, out: torch.Tensor | None = None,
                 stream=None):
+        if self.asym:
+            q, rs = self.quantize_with_rowsum(x, q_buf, stream=stream)
+            return self.linear(q, out, stream, rowsum=rs)
         return self.linear(self.quantize(x, q_buf, stream), out, stream)
 
     __call__ = forward
 
     def state_dict(self):
         """The per-layer artefact, as plain tensors (saved with torch.save)."""
-        return {k: getattr(self, k) for k in ("ch_min", "ch_max", "z", "s", "r", "qw", "sw", "b_fold")}
+        keys = ("ch_min", "ch_max", "z", "s", "r", "qw", "sw", "b_fold") + (("zc",) if self.asym else ())
+        return {k: getattr(self, k) for k in keys}
 
     def load_state_dict(self, sd):
         for k, v in sd.items():
@@ -81,7 +116,7 @@ class QuantizedLinear:
         return self
 
     def weight_bytes(self) -> int:
-        return self.qw.numel() + 4 * (self.sw.numel() + self.b_fold.numel())
+        return self.qw.numel() + 4 * (self.sw.numel() + self.b_fold.numel() + (self.N if self.asym else 0))
 
 
 class QuantizedBlockLinears:

@@ -66,6 +66,9 @@ def _linear_args(handle):
     handle.ot_calibrate.argtypes = [P, I64, I64, I64, P, P, I, P]
     handle.ot_fold_weights.argtypes = [P, P, I, I, P, P, I64, I64, I, P, P, P, P, P, P, P]
     handle.ot_selftest_wait_timeout.argtypes = [I64, P]
+    handle.ot_linear_asym.argtypes = [P, I64, I64, P, P, P, P, P, I64, I, I, P, I64, I, P, S, P]
+    handle.ot_quantize_act_rowsum.argtypes = [P, I64, I64, I64, P, P, I, P, I, P, P]
+    handle.ot_fold_weights_asym.argtypes = [P, P, I, I, P, P, I64, I64, I, P, P, P, P, P, P, P, P]
 
 
 # Fake, 256-byte-aligned addresses: every call below must be rejected on the
@@ -107,6 +110,16 @@ def test_validation_rejects_bad_arguments_before_launch(lib):
     assert handle.ot_fold_weights(A, A, 8, 1, A + 2, None, 16, 64, 8, A, A, A, A2, A, A, None) == INV
     # self-test limit outside [1 ms, 2 s]
     assert handle.ot_selftest_wait_timeout(10, None) == INV
+    # asymmetric weights: null zero points / row sums, unaligned zero points
+    assert handle.ot_linear_asym(A, 4, 64, A2, A, None, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear_asym(A, 4, 64, A2, A, A, None, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear_asym(A, 4, 64, A2, A, A + 2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    # the corrected sum K * 127 * 255 must fit int32: K = 66,320 is refused, 66,304 is not
+    assert handle.ot_linear_asym(A, 4, 66320, A2, A, A, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == UNS
+    assert 127 * 255 * 66304 < 2 ** 31
+    assert handle.ot_quantize_act_rowsum(A, 4, 64, 64, A, A, 8, A2, 1, None, None) == INV
+    assert handle.ot_quantize_act_rowsum(A, 4, 64, 64, A, A, 8, A2, 1, A + 2, None) == INV
+    assert handle.ot_fold_weights_asym(A, A, 8, 1, A, None, 16, 64, 8, A, A, A, A2, A, None, A, None) == INV
 
 
 def test_binding_refuses_host_tensors():

@@ -181,3 +181,23 @@ def test_asym_layer_end_to_end_and_accuracy():
     err_asym = np.abs(got.astype(np.float64) - exact).mean()
     err_sym = np.abs(ref_sym.astype(np.float64) - exact).mean()
     assert err_asym < err_sym
+
+
+def test_quantized_linear_asym_layer_matches_oracle():
+    """QuantizedLinear(weights="asym"): calibrate, fold, forward == the oracle chain."""
+    from paper_2406_18832_gb300 import QuantizedLinear
+    M, N, K = 40, 320, 768
+    cal, x = _acts(512, K, 60), _acts(M, K, 61)
+    w = _weights(N, K, 62)
+    b = (torch.randn(N, generator=_gen(63)) * 0.01).half()
+    ql = QuantizedLinear(K, N, 8, 8, relu=True, device=DEV, weights="asym")
+    ql.calibrate(cal[:256].to(DEV)).calibrate(cal[256:].to(DEV)).fold(w.to(DEV), b.to(DEV))
+    y = ql(x.to(DEV)).cpu().numpy()
+    mn, mx = oracle.calibrate(cal.numpy())
+    z, s, r = oracle.params(mn, mx, 8)
+    qw, sw, zc = oracle.fold_codes_asym(w.numpy(), s, 8)
+    _, _, bf = oracle.fold(w.numpy(), b.numpy(), z, s, 8)
+    q = oracle.quantize(x.numpy(), z, r, 8)
+    ref = oracle.epilogue_asym(oracle.matmul(q, qw), oracle.rowsum(q), zc, sw, bf, relu=True)
+    assert np.array_equal(y.view(np.uint16), ref.view(np.uint16))
+    assert set(ql.state_dict()) >= {"zc", "qw", "sw", "b_fold"}
