@@ -22,6 +22,9 @@ and the asymmetric weights ("Int8": per-output-channel zero points, Eq. 1):
   fold_codes_asym   - codes of W_s over [min(0, min), max(0, max)] with a zero point
   rowsum            - sum_k q[m,k] (exact)
   epilogue_asym     - fp16(fma((float)(acc - zc_n rs_m), sw_n, b'_n))
+and the LayerNorm fused with the symmetrization and quantization (Section 3.2):
+  fold_layernorm       - gamma * r and (beta - z) * r
+  layernorm_quantize   - exact row statistics, codes of LN(h) - z scaled by r
 """
 from __future__ import annotations
 
@@ -74,9 +77,12 @@ def _load():
             lib.oracle_fold_codes_asym.argtypes = [P, I64, I64, P, I, P, P, P]
             lib.oracle_rowsum.argtypes = [P, I64, I64, P]
             lib.oracle_epilogue_asym.argtypes = [P, P, P, I64, I64, P, P, I, P]
+            lib.oracle_fold_layernorm.argtypes = [P, P, P, P, I64, P, P]
+            lib.oracle_layernorm_quantize.argtypes = [P, I64, I64, I64, P, P, ctypes.c_float, I, P, P, P, P]
             for f in ("oracle_calibrate", "oracle_params", "oracle_fold", "oracle_quantize",
                       "oracle_matmul", "oracle_epilogue", "oracle_quantize_tokens", "oracle_epilogue_tokens",
-                      "oracle_fold_codes_asym", "oracle_rowsum", "oracle_epilogue_asym"):
+                      "oracle_fold_codes_asym", "oracle_rowsum", "oracle_epilogue_asym",
+                      "oracle_fold_layernorm", "oracle_layernorm_quantize"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -250,3 +256,25 @@ def epilogue_asym(acc: np.ndarray, rs: np.ndarray, zc: np.ndarray, sw: np.ndarra
     _load().oracle_epilogue_asym(_ptr(acc), _ptr(rs), _ptr(zc), M, N, _ptr(_f32(sw)), _ptr(_f32(bfold)),
                                  1 if relu else 0, _ptr(y))
     return y.view(np.float16)
+
+
+def fold_layernorm(gamma: np.ndarray, beta: np.ndarray, z: np.ndarray, r: np.ndarray):
+    """(gamma_r, beta_r) fp32 [K]: gamma * r and (beta - z) * r (gamma, beta fp16)."""
+    gamma, beta = _f16(gamma), _f16(beta)
+    K = gamma.shape[0]
+    gr, br = np.empty(K, np.float32), np.empty(K, np.float32)
+    _load().oracle_fold_layernorm(_ptr(gamma), _ptr(beta), _ptr(_f32(z)), _ptr(_f32(r)), K, _ptr(gr), _ptr(br))
+    return gr, br
+
+
+def layernorm_quantize(h: np.ndarray, gamma_r: np.ndarray, beta_r: np.ndarray, eps: float, bits: int):
+    """(codes int8 [M, K], rowsum int64 [M], mean fp32 [M], rstd fp32 [M]) of the
+    LayerNorm of fp16 h [M, K] fused with the per-channel quantization."""
+    h = _f16(h)
+    M, K = h.shape
+    q = np.empty((M, K), np.int8)
+    rs = np.empty(M, np.int64)
+    mean, rstd = np.empty(M, np.float32), np.empty(M, np.float32)
+    _load().oracle_layernorm_quantize(_ptr(h), M, K, K, _ptr(_f32(gamma_r)), _ptr(_f32(beta_r)), float(eps), bits,
+                                      _ptr(q), _ptr(rs), _ptr(mean), _ptr(rstd))
+    return q, rs, mean, rstd

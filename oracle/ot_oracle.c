@@ -47,6 +47,15 @@
  *                clip(round(w * r) + zp, 0, 2^b - 1); NaN codes to the zero
  *                point.  Codes and zero points are stored shifted by
  *                -2^(b-1) so they fit int8.
+ *   R10 LN fusion the paper fuses the per-channel quantization into the
+ *                LayerNorm before the linear (Section 3.2) without fixing the
+ *                arithmetic.  Here the row statistics are exact: h * 2^24 is
+ *                an integer for every fp16 h, so sum(h) and sum(h^2) are
+ *                exact integer sums; mean and 1/sqrt(var + eps) (biased
+ *                variance) follow by a fixed sequence of IEEE fp64
+ *                operations, and the codes by one fp32 fma with the folded
+ *                gamma * r and (beta - z) * r.  A row holding a non-finite
+ *                value codes to 0 throughout.
  *
  * Floating point: compile with -ffp-contract=off and no fast-math, so every
  * fp32 expression below rounds once per operation as written.
@@ -404,4 +413,84 @@ void oracle_epilogue_asym(const int64_t *acc, const int64_t *rs, const int32_t *
             if (relu && !(v > 0.0f)) v = 0.0f;
             y[m * N + n] = ot_double_to_half((double)v);
         }
+}
+
+/* ---------------------------------------------------------------------------
+ * LayerNorm fused with the symmetrization and the per-channel quantization
+ * (Section 3.2, R10): LN(h) = (h - mean) / sqrt(var + eps) * gamma + beta, and
+ * the codes round((LN(h) - z) * r) = round(n * gamma * r + (beta - z) * r)
+ * with n = (h - mean) / sqrt(var + eps).
+ *
+ * Step L0 (offline, with the fold): gamma_r[k] = gamma[k] * r[k] and
+ * beta_r[k] = (beta[k] - z[k]) * r[k] in fp32 (gamma, beta fp16).
+ * ------------------------------------------------------------------------- */
+void oracle_fold_layernorm(const uint16_t *gamma, const uint16_t *beta, const float *z,
+                           const float *r, int64_t K, float *gamma_r, float *beta_r)
+{
+    for (int64_t k = 0; k < K; ++k) {
+        gamma_r[k] = ot_half_to_float(gamma[k]) * r[k];
+        beta_r[k] = (ot_half_to_float(beta[k]) - z[k]) * r[k];
+    }
+}
+
+/* A non-negative 128-bit integer as hi * 2^64 + lo, each part converted to
+ * double and added (round to nearest at each step). */
+static double u128_to_double(unsigned __int128 v)
+{
+    const uint64_t hi = (uint64_t)(v >> 64), lo = (uint64_t)v;
+    return (double)hi * 18446744073709551616.0 + (double)lo;
+}
+
+/* ---------------------------------------------------------------------------
+ * Step L1: per row m of the hidden state h [M, K] (fp16, row stride ldh):
+ *   H_k  = h_k * 2^24 (integer),  S1 = sum_k H_k,  S2 = sum_k H_k^2   (exact)
+ *   mean = float( ((double)S1 / K) * 2^-24 )
+ *   V    = K * S2 - S1^2  (exact, >= 0),  var = (double(V) / K / K) * 2^-48
+ *   rstd = float( 1 / sqrt(var + (double)eps) )
+ *   u_k  = fma((h_k - mean) * rstd, gamma_r[k], beta_r[k])   (fp32 roundings)
+ *   q_k  = round_half_even(u_k) in [-qmax, qmax]
+ * q is [M, K] int8; rowsum[m] = sum_k q[m,k] if rowsum is not NULL; mean and
+ * rstd per row are returned for the tests (NULL to skip).
+ * ------------------------------------------------------------------------- */
+void oracle_layernorm_quantize(const uint16_t *h, int64_t M, int64_t K, int64_t ldh,
+                               const float *gamma_r, const float *beta_r, float eps,
+                               int bits, int8_t *q, int64_t *rowsum, float *mean_out,
+                               float *rstd_out)
+{
+    const int qmax = qmax_of(bits);
+    for (int64_t m = 0; m < M; ++m) {
+        const uint16_t *row = h + m * ldh;
+        int64_t s1 = 0;
+        unsigned __int128 s2 = 0;
+        int finite = 1;
+        for (int64_t k = 0; k < K; ++k) {
+            const float v = ot_half_to_float(row[k]);
+            if (!isfinite(v)) { finite = 0; break; }
+            const int64_t hk = (int64_t)(v * 16777216.0f);   /* exact: an fp16 times 2^24 */
+            s1 += hk;
+            const uint64_t a = (uint64_t)(hk < 0 ? -hk : hk);
+            s2 += (unsigned __int128)a * a;
+        }
+        float mean = 0.0f, rstd = 0.0f;
+        if (finite) {
+            mean = (float)(((double)s1 / (double)K) * 0x1p-24);
+            const __int128 s1s = (__int128)s1;
+            const unsigned __int128 v = (unsigned __int128)K * s2 - (unsigned __int128)(s1s * s1s);
+            const double var = ((u128_to_double(v) / (double)K) / (double)K) * 0x1p-48;
+            rstd = (float)(1.0 / sqrt(var + (double)eps));
+        }
+        if (mean_out) mean_out[m] = mean;
+        if (rstd_out) rstd_out[m] = rstd;
+        int64_t rs = 0;
+        for (int64_t k = 0; k < K; ++k) {
+            int c = 0;
+            if (finite) {
+                const float n = (ot_half_to_float(row[k]) - mean) * rstd;
+                c = quantize_code(fmaf(n, gamma_r[k], beta_r[k]), qmax);
+            }
+            q[m * K + k] = (int8_t)c;
+            rs += c;
+        }
+        if (rowsum) rowsum[m] = rs;
+    }
 }
