@@ -346,6 +346,7 @@ def run_ours(args):
     block = None if args.no_block else bench_block(dev)
     decode = bench_decode(dev, peaks)
     asym = bench_asym(dev, layers, xs, ops_step, ms_per_step)
+    lnq = bench_layernorm(dev, peaks)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -389,6 +390,7 @@ def run_ours(args):
         "block": block,
         "decode": decode,
         "asym_weights": asym,
+        "layernorm_quantize": lnq,
         "cpu_baseline": cpu,
     }
     if rank == 0:
@@ -448,6 +450,64 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
             "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
             "over_symmetric_step": round(ms / ms_sym, 4),
             "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
+
+
+def bench_layernorm(dev, peaks, reps: int = 200):
+    """The LayerNorm before QKV / fc1 fused with the symmetrization and the
+    per-channel quantization (Section 3.2), OPT-6.7B at 2048 tokens (hidden
+    4096): one kernel reads h and writes the codes, against the unfused pair
+    (a LayerNorm writing fp16, here torch's, then the quantize kernel).
+    Consecutive calls rotate over input copies larger than the L2 and are
+    timed as CUDA-graph replays."""
+    import torch
+    import torch.nn.functional as F
+
+    from paper_2406_18832_gb300 import binding
+    M, K, eps = TOKENS, 4096, 1e-5
+    g = torch.Generator(device=dev).manual_seed(77)
+    copies = -(-3 * L2_BYTES // (M * K * 2))
+    hs = [torch.randn(M, K, generator=g, device=dev).half() for _ in range(copies)]
+    gamma = (1 + 0.1 * torch.randn(K, generator=g, device=dev)).half()
+    beta = (0.1 * torch.randn(K, generator=g, device=dev)).half()
+    z = 0.1 * torch.randn(K, generator=g, device=dev)
+    r = torch.full((K,), 30.0, device=dev)
+    gr, br = torch.empty(K, device=dev), torch.empty(K, device=dev)
+    binding.ot_fold_layernorm(gamma, beta, z, r, gr, br)
+    q = torch.empty(M, K, dtype=torch.float16, device=dev)
+
+    def timed(fn):
+        # CUDA-graph replay of `reps` consecutive calls (kernel time, not the
+        # Python call overhead of eager launches)
+        for i in range(copies):
+            fn(hs[i])
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for i in range(reps):
+                fn(hs[i % copies])
+        graph.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(3):
+            graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / (3 * reps)
+
+    fused_ms = timed(lambda h: binding.ot_layernorm_quantize(h, gr, br, eps, 8, q))
+
+    def unfused(h):
+        binding.ot_quantize_act(F.layer_norm(h, (K,), gamma, beta, eps), z, r, 8, q)
+
+    unfused_ms = timed(unfused)
+    bytes_fused = 4 * M * K + 8 * K
+    gbs = bytes_fused / (fused_ms * 1e-3) / 1e9
+    return {"workload": "opt-6.7b LayerNorm -> QKV / fc1 input, 2048 tokens x 4096", "kernel": "layernorm_quantize",
+            "us": round(fused_ms * 1e3, 2), "gbs": round(gbs, 1), "frac_hbm": round(gbs / peaks["hbm"], 4),
+            "bytes": bytes_fused, "note": "fp16 h in + fp16 codes out; statistics exact (integer sums)",
+            "unfused_us": round(unfused_ms * 1e3, 2),
+            "unfused": "torch layer_norm (fp16 out) + quantize_kernel"}
 
 
 def bench_decode(dev, peaks, reps: int = 50):

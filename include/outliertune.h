@@ -201,6 +201,44 @@ ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int
                               void *stream);
 
 /*
+ * LayerNorm fused with the symmetrization and the per-channel quantization
+ * (Section 3.2: the codes of Eq. 7 come out of the LayerNorm before the linear,
+ * whose gamma and beta absorb the scale r and the shift z).  For the linears
+ * that follow a LayerNorm, h is the residual-stream input of that LayerNorm.
+ *
+ * ot_fold_layernorm -- offline, after calibration (z, r from ot_derive_params
+ * or ot_fold_weights on the LayerNorm's outputs):
+ *   gamma_r[k] = gamma[k] * r[k],   beta_r[k] = (beta[k] - z[k]) * r[k]   (fp32)
+ *   gamma_f16, beta_f16  fp16 [K] (the LayerNorm's affine parameters)
+ */
+ot_status ot_fold_layernorm(const void *gamma_f16, const void *beta_f16, const float *z,
+                            const float *r, int64_t K, float *gamma_r, float *beta_r,
+                            void *stream);
+
+/*
+ * ot_layernorm_quantize -- codes of the symmetrized LayerNorm output:
+ *   mean = sum_k h / K,  var = sum_k h^2 / K - mean^2 (biased),
+ *   q[m,k] = round_half_even( ((h - mean) * rstd) * gamma_r[k] + beta_r[k] )
+ * clipped to [-qmax, qmax], with rstd = 1 / sqrt(var + eps).  The statistics are
+ * exact: h * 2^24 is an integer for every fp16 h, its sum S1 and the sum of
+ * its squares S2 are exact integers, mean and rstd are formed from them by a
+ * fixed sequence of IEEE fp32 operations (mean = (float(S1) / K) * 2^-24,
+ * var = (float(K S2 - S1^2) / K / K) * 2^-48 with the 128-bit integer taken
+ * as float(hi) 2^64 + float(lo), rstd = 1 / sqrt(var + eps)), then
+ * (h - mean) * rstd and one fp32 fma, so the codes do not depend on the order
+ * of any reduction.  A row holding a non-finite value codes to 0 throughout.
+ *   h_f16   fp16 [M, K], row stride ldh (16-byte aligned; K, ldh % 8 == 0; K <= 2^22)
+ *   gamma_r, beta_r  fp32 [K] from ot_fold_layernorm (16-byte aligned)
+ *   eps     finite, >= 0
+ *   q       [M, K] dense codes, int8 or fp16 (ot_code_format), 16-byte aligned
+ *   rowsum  optional int32 [M]: sum_k q[m,k] (for ot_linear_asym), or NULL
+ */
+ot_status ot_layernorm_quantize(const void *h_f16, int64_t M, int64_t K, int64_t ldh,
+                                const float *gamma_r, const float *beta_r, float eps,
+                                int bits_a, void *q, int q_format, int32_t *rowsum,
+                                void *stream);
+
+/*
  * Asymmetric per-output-channel weights: the paper's "Int8" (Section 4,
  * Appendix A: zero points for the weights, min-max calibration), which trades
  * a little speed for accuracy against the symmetric "Int8*" of ot_fold_weights.

@@ -52,7 +52,7 @@
  *                arithmetic.  Here the row statistics are exact: h * 2^24 is
  *                an integer for every fp16 h, so sum(h) and sum(h^2) are
  *                exact integer sums; mean and 1/sqrt(var + eps) (biased
- *                variance) follow by a fixed sequence of IEEE fp64
+ *                variance) follow by a fixed sequence of IEEE fp32
  *                operations, and the codes by one fp32 fma with the folded
  *                gamma * r and (beta - z) * r.  A row holding a non-finite
  *                value codes to 0 throughout.
@@ -434,19 +434,19 @@ void oracle_fold_layernorm(const uint16_t *gamma, const uint16_t *beta, const fl
 }
 
 /* A non-negative 128-bit integer as hi * 2^64 + lo, each part converted to
- * double and added (round to nearest at each step). */
-static double u128_to_double(unsigned __int128 v)
+ * float and added (round to nearest at each step; the scaling is exact). */
+static float u128_to_float(unsigned __int128 v)
 {
     const uint64_t hi = (uint64_t)(v >> 64), lo = (uint64_t)v;
-    return (double)hi * 18446744073709551616.0 + (double)lo;
+    return (float)hi * 18446744073709551616.0f + (float)lo;
 }
 
 /* ---------------------------------------------------------------------------
  * Step L1: per row m of the hidden state h [M, K] (fp16, row stride ldh):
  *   H_k  = h_k * 2^24 (integer),  S1 = sum_k H_k,  S2 = sum_k H_k^2   (exact)
- *   mean = float( ((double)S1 / K) * 2^-24 )
- *   V    = K * S2 - S1^2  (exact, >= 0),  var = (double(V) / K / K) * 2^-48
- *   rstd = float( 1 / sqrt(var + (double)eps) )
+ *   mean = ((float)S1 / K) * 2^-24                              (fp32)
+ *   V    = K * S2 - S1^2  (exact, >= 0),  var = (float(V) / K / K) * 2^-48
+ *   rstd = 1 / sqrt(var + eps)                                   (fp32, IEEE)
  *   u_k  = fma((h_k - mean) * rstd, gamma_r[k], beta_r[k])   (fp32 roundings)
  *   q_k  = round_half_even(u_k) in [-qmax, qmax]
  * q is [M, K] int8; rowsum[m] = sum_k q[m,k] if rowsum is not NULL; mean and
@@ -473,11 +473,12 @@ void oracle_layernorm_quantize(const uint16_t *h, int64_t M, int64_t K, int64_t 
         }
         float mean = 0.0f, rstd = 0.0f;
         if (finite) {
-            mean = (float)(((double)s1 / (double)K) * 0x1p-24);
+            const float kf = (float)K;
+            mean = ((float)s1 / kf) * 0x1p-24f;
             const __int128 s1s = (__int128)s1;
             const unsigned __int128 v = (unsigned __int128)K * s2 - (unsigned __int128)(s1s * s1s);
-            const double var = ((u128_to_double(v) / (double)K) / (double)K) * 0x1p-48;
-            rstd = (float)(1.0 / sqrt(var + (double)eps));
+            const float var = ((u128_to_float(v) / kf) / kf) * 0x1p-48f;
+            rstd = 1.0f / sqrtf(var + eps);
         }
         if (mean_out) mean_out[m] = mean;
         if (rstd_out) rstd_out[m] = rstd;

@@ -42,6 +42,8 @@ _SIGNATURES = {
     "ot_quantize_act_rowsum": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _I, _P, _P], _I),
     "ot_linear_asym": ([_P, _I64, _I64, _P, _P, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P],
                        _I),
+    "ot_fold_layernorm": ([_P, _P, _P, _P, _I64, _P, _P, _P], _I),
+    "ot_layernorm_quantize": ([_P, _I64, _I64, _I64, _P, _P, _F, _I, _P, _I, _P, _P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -202,6 +204,29 @@ def ot_linear_asym(q, qw, sw, zc, rowsum, b_fold, bits_a: int, bits_w: int, y, r
                                  bits_a, bits_w, _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb,
                                  _stream(stream)),
            "ot_linear_asym")
+
+
+def ot_fold_layernorm(gamma, beta, z, r, gamma_r, beta_r, stream=None):
+    """gamma_r = gamma * r, beta_r = (beta - z) * r (fp32 [K]) from the LayerNorm's fp16 gamma, beta."""
+    K = gamma.numel()
+    _check(load().ot_fold_layernorm(_dev(gamma, "gamma", torch.float16), _dev(beta, "beta", torch.float16),
+                                    _dev(z, "z", torch.float32), _dev(r, "r", torch.float32), K,
+                                    _dev(gamma_r, "gamma_r", torch.float32), _dev(beta_r, "beta_r", torch.float32),
+                                    _stream(stream)),
+           "ot_fold_layernorm")
+
+
+def ot_layernorm_quantize(h, gamma_r, beta_r, eps: float, bits_a: int, q, q_format: int = OT_CODE_F16,
+                          rowsum=None, stream=None):
+    """Codes of the symmetrized LayerNorm output of fp16 h [M, K] (optionally their row sums)."""
+    M, K, ldh = _rows(h, "h")
+    _dense(q, "q")
+    want = torch.float16 if q_format == OT_CODE_F16 else torch.int8
+    prs = None if rowsum is None else _dev(rowsum, "rowsum", torch.int32)
+    _check(load().ot_layernorm_quantize(_dev(h, "h", torch.float16), M, K, ldh, _dev(gamma_r, "gamma_r", torch.float32),
+                                        _dev(beta_r, "beta_r", torch.float32), float(eps), bits_a,
+                                        _dev(q, "q", want), q_format, prs, _stream(stream)),
+           "ot_layernorm_quantize")
 
 
 def ot_linear_workspace_size() -> int:

@@ -109,6 +109,30 @@ ot_status ot_quantize_act_rowsum(const void *x_f16, int64_t M, int64_t K, int64_
         ot::launch_quantize(x_f16, M, K, ldx, z, r, bits_a, q, q_format, as_stream(stream), rowsum));
 }
 
+ot_status ot_fold_layernorm(const void *gamma_f16, const void *beta_f16, const float *z, const float *r, int64_t K,
+                            float *gamma_r, float *beta_r, void *stream) {
+    if (K <= 0 || !gamma_f16 || !beta_f16 || !z || !r || !gamma_r || !beta_r) return OT_ERR_INVALID_ARG;
+    if (!aligned(gamma_f16, 2) || !aligned(beta_f16, 2) || !aligned(z, 4) || !aligned(r, 4) ||
+        !aligned(gamma_r, 4) || !aligned(beta_r, 4))
+        return OT_ERR_INVALID_ARG;
+    if (K > kIntMax) return OT_ERR_UNSUPPORTED;
+    return from_cuda(ot::launch_fold_layernorm(gamma_f16, beta_f16, z, r, K, gamma_r, beta_r, as_stream(stream)));
+}
+
+ot_status ot_layernorm_quantize(const void *h_f16, int64_t M, int64_t K, int64_t ldh, const float *gamma_r,
+                                const float *beta_r, float eps, int bits_a, void *q, int q_format,
+                                int32_t *rowsum, void *stream) {
+    if (M < 0 || K <= 0 || K % 8 != 0 || ldh < K || ldh % 8 != 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;
+    if (q_format != OT_CODE_I8 && q_format != OT_CODE_F16) return OT_ERR_INVALID_ARG;
+    if (!(eps >= 0.0f) || !(eps < 3.0e38f)) return OT_ERR_INVALID_ARG;  // finite, non-negative (rejects NaN)
+    if (!gamma_r || !beta_r || !aligned(gamma_r, 16) || !aligned(beta_r, 16)) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!h_f16 || !q || !aligned(h_f16, 16) || !aligned(q, 16))) return OT_ERR_INVALID_ARG;
+    if (rowsum && !aligned(rowsum, 4)) return OT_ERR_INVALID_ARG;
+    if (K > ((int64_t)1 << 22)) return OT_ERR_UNSUPPORTED;  // exact 64-bit partial sums of the squares
+    return from_cuda(ot::launch_layernorm_quantize(h_f16, M, K, ldh, gamma_r, beta_r, eps, bits_a, q, q_format,
+                                                   rowsum, as_stream(stream)));
+}
+
 ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
                           int bits_a, void *q, int q_format, void *stream) {
     if (M < 0 || K <= 0 || K % 8 != 0 || ldx < K || ldx % 8 != 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;

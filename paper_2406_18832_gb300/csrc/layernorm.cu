@@ -1,0 +1,270 @@
+// layernorm.cu -- the LayerNorm before a per-channel quantized linear, fused
+// with the symmetrization and the activation quantization (Section 3.2: the
+// codes round(X_hat / s) "through the kernel fusion with its previous
+// LayerNorm"; LN's gamma and beta absorb r and z):
+//   q = round(((h - mean) * rstd) * gamma_r + beta_r),
+//   gamma_r = gamma * r,  beta_r = (beta - z) * r   (folded once, offline).
+// The row statistics are exact so the codes do not depend on a reduction
+// order: h * 2^24 is an integer H for every fp16 h (|H| < 2^40), sum H is an
+// exact int64 and sum H^2 is kept as three exact 64-bit partial sums of
+// 20-bit halves (H = a 2^20 + b:  H^2 = a^2 2^40 + 2ab 2^20 + b^2), combined in
+// 128 bits once per row.  Mean and 1/sqrt(var + eps) then follow by a fixed
+// sequence of IEEE fp32 operations (one lane per row) and the codes by one
+// fp32 fma per element.
+// HBM-bound: one warp per row, no block barriers; rows up to 8192 wide are
+// held in registers (one HBM read with the whole row in flight), longer ones
+// are streamed and read again from L2 for the codes.
+#include <cuda_fp16.h>
+
+#include "ot_common.cuh"
+#include "ot_kernels.h"
+
+namespace ot {
+
+namespace {
+
+constexpr int kLnThreads = 256;
+constexpr int kLnWarps = kLnThreads / 32;  // rows per CTA
+
+__global__ void __launch_bounds__(256) fold_layernorm_kernel(const __half *__restrict__ gamma,
+                                                             const __half *__restrict__ beta,
+                                                             const float *__restrict__ z,
+                                                             const float *__restrict__ r, int64_t K,
+                                                             float *gamma_r, float *beta_r) {
+    const int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (k >= K) return;
+    const float rk = __ldg(r + k);
+    gamma_r[k] = __fmul_rn(__half2float(gamma[k]), rk);
+    beta_r[k] = __fmul_rn(__fsub_rn(__half2float(beta[k]), __ldg(z + k)), rk);
+}
+
+struct LnSums {
+    long long sh, sl;             // sum of the signed 20-bit halves of H: S1 = sh 2^20 + sl
+    unsigned long long a, b, c;   // sum hi^2, sum hi*lo, sum lo^2 of the 20-bit halves of |H|
+    int bad;                      // non-finite values seen
+};
+
+// One fp16 value (bits u) into the sums, in 32-bit integer arithmetic: for
+// exponent field e and fraction f, |H| = h 2^24 = mant << sh with mant =
+// f | 1024 (f for e = 0) and sh = max(e - 1, 0) <= 29; its 20-bit halves are
+// hi = |H| >> 20 and lo = |H| & (2^20 - 1).  The caller's chunk of 8 values
+// keeps the signed half sums in int32 (|sum| < 2^23).
+__device__ __forceinline__ void ln_add_bits(uint32_t u, int &chi, int &clo, LnSums &s) {
+    const uint32_t e = (u >> 10) & 31u, f = u & 1023u;
+    s.bad |= (e == 31u);
+    const uint32_t nz = e != 0u;
+    const uint32_t mant = f | (nz << 10);
+    const uint32_t sh = e - nz;
+    const uint32_t t = mant << (sh < 20u ? sh : 0u);                 // < 2^31 when sh < 20
+    const uint32_t hi = sh >= 20u ? mant << (sh - 20u) : t >> 20;
+    const uint32_t lo = sh >= 20u ? 0u : t & 0xFFFFFu;
+    const bool neg = (u & 0x8000u) != 0u;
+    chi += neg ? -(int)hi : (int)hi;
+    clo += neg ? -(int)lo : (int)lo;
+    s.a += (unsigned long long)hi * hi;
+    s.b += (unsigned long long)hi * lo;
+    s.c += (unsigned long long)lo * lo;
+}
+
+// Codes of 8 elements (one 16-byte chunk of the row) from mean, rstd and the
+// folded affine; returns their sum.
+template <bool kF16Out>
+__device__ __forceinline__ int ln_codes8(const uint4 &d, int64_t k, float mean, float rstd,
+                                         const float *__restrict__ gamma_r, const float *__restrict__ beta_r,
+                                         int qmax, void *q, int64_t qoff, bool bad) {
+    int c[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (!bad) {
+        const __half2 *hv = reinterpret_cast<const __half2 *>(&d);
+        const float4 g0 = __ldg(reinterpret_cast<const float4 *>(gamma_r + k));
+        const float4 g1 = __ldg(reinterpret_cast<const float4 *>(gamma_r + k + 4));
+        const float4 b0 = __ldg(reinterpret_cast<const float4 *>(beta_r + k));
+        const float4 b1 = __ldg(reinterpret_cast<const float4 *>(beta_r + k + 4));
+        const float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+        const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 f = __half22float2(hv[j]);
+            const float n0 = __fmul_rn(__fsub_rn(f.x, mean), rstd);
+            const float n1 = __fmul_rn(__fsub_rn(f.y, mean), rstd);
+            // cvt.rni maps NaN to 0 and saturates; then the symmetric range
+            c[2 * j] = max(-qmax, min(qmax, __float2int_rn(__fmaf_rn(n0, g[2 * j], bb[2 * j]))));
+            c[2 * j + 1] = max(-qmax, min(qmax, __float2int_rn(__fmaf_rn(n1, g[2 * j + 1], bb[2 * j + 1]))));
+        }
+    }
+    int rs = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) rs += c[j];
+    if (kF16Out) {
+        // fp16 holding the integer c: the pattern 0x6400 | (c + 128), minus 1152 (exact)
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t bits = (uint32_t)(0x6480 + c[2 * j]) | ((uint32_t)(0x6480 + c[2 * j + 1]) << 16);
+            const __half2 v = __hsub2(*reinterpret_cast<const __half2 *>(&bits),
+                                      __half2half2(__ushort_as_half(0x6480)));
+            w[j] = *reinterpret_cast<const uint32_t *>(&v);
+        }
+        *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + qoff) = make_uint4(w[0], w[1], w[2], w[3]);
+    } else {
+        uint2 o;
+        o.x = __byte_perm(__byte_perm((uint32_t)c[0], (uint32_t)c[1], 0x0040),
+                          __byte_perm((uint32_t)c[2], (uint32_t)c[3], 0x0040), 0x5410);
+        o.y = __byte_perm(__byte_perm((uint32_t)c[4], (uint32_t)c[5], 0x0040),
+                          __byte_perm((uint32_t)c[6], (uint32_t)c[7], 0x0040), 0x5410);
+        *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + qoff) = o;
+    }
+    return rs;
+}
+
+__device__ __forceinline__ void ln_add8(LnSums &s, const uint4 &d) {
+    int chi = 0, clo = 0;
+    const uint32_t w[4] = {d.x, d.y, d.z, d.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        ln_add_bits(w[j] & 0xFFFFu, chi, clo, s);
+        ln_add_bits(w[j] >> 16, chi, clo, s);
+    }
+    s.sh += chi;
+    s.sl += clo;
+}
+
+// mean and rstd of the row from the warp's exact sums (lane 0; IEEE fp32 in
+// the order documented above), broadcast to the warp.
+__device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        s.sh += __shfl_xor_sync(0xffffffffu, s.sh, o);
+        s.sl += __shfl_xor_sync(0xffffffffu, s.sl, o);
+        s.a += __shfl_xor_sync(0xffffffffu, s.a, o);
+        s.b += __shfl_xor_sync(0xffffffffu, s.b, o);
+        s.c += __shfl_xor_sync(0xffffffffu, s.c, o);
+        s.bad |= __shfl_xor_sync(0xffffffffu, s.bad, o);
+    }
+    mean = 0.f;
+    rstd = 0.f;
+    if ((threadIdx.x & 31) == 0 && !s.bad) {
+        const float kf = (float)K;  // exact: K <= 2^22
+        const long long S1 = s.sh * (1LL << 20) + s.sl;  // exact: |S1| < 2^62
+        mean = __fmul_rn(__fdiv_rn(__ll2float_rn(S1), kf), 0x1p-24f);
+        const unsigned __int128 s2 = ((unsigned __int128)s.a << 40) + ((unsigned __int128)s.b << 21) +
+                                     (unsigned __int128)s.c;
+        const __int128 s1 = (__int128)S1;
+        const unsigned __int128 v = (unsigned __int128)K * s2 - (unsigned __int128)(s1 * s1);
+        const float vf = __fadd_rn(__fmul_rn(__ull2float_rn((unsigned long long)(v >> 64)), 18446744073709551616.0f),
+                                   __ull2float_rn((unsigned long long)v));
+        const float var = __fmul_rn(__fdiv_rn(__fdiv_rn(vf, kf), kf), 0x1p-48f);
+        rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, eps)));
+    }
+    mean = __shfl_sync(0xffffffffu, mean, 0);
+    rstd = __shfl_sync(0xffffffffu, rstd, 0);
+}
+
+// One warp per row (kLnWarps rows per CTA, grid-stride).  kCh > 0: the lane
+// holds its kCh 16-byte chunks of the row (K <= 256 kCh) in registers, all
+// loaded before use, so the row is read from HBM once with the whole row in
+// flight.  kCh == 0: longer rows stream in batches of 8 chunks per lane and
+// are read again (from L2) for the codes.
+template <bool kF16Out, int kCh>
+__global__ void __launch_bounds__(kLnThreads) layernorm_quantize_kernel(const __half *__restrict__ h, int64_t M,
+                                                                        int64_t K, int64_t ldh,
+                                                                        const float *__restrict__ gamma_r,
+                                                                        const float *__restrict__ beta_r, float eps,
+                                                                        int qmax, void *q, int32_t *rowsum) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int64_t m = (int64_t)blockIdx.x * kLnWarps + warp; m < M; m += (int64_t)gridDim.x * kLnWarps) {
+        const __half *row = h + m * ldh;
+        LnSums s{0, 0, 0, 0, 0, 0};
+        float mean, rstd;
+        int rs = 0;
+        if constexpr (kCh > 0) {
+            uint4 d[kCh];
+#pragma unroll
+            for (int i = 0; i < kCh; ++i) {
+                const int64_t k = (int64_t)(lane + 32 * i) * 8;
+                d[i] = k < K ? __ldcs(reinterpret_cast<const uint4 *>(row + k)) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int i = 0; i < kCh; ++i)
+                if ((int64_t)(lane + 32 * i) * 8 < K) ln_add8(s, d[i]);
+            ln_stats(s, K, eps, mean, rstd);
+#pragma unroll
+            for (int i = 0; i < kCh; ++i) {
+                const int64_t k = (int64_t)(lane + 32 * i) * 8;
+                if (k < K) rs += ln_codes8<kF16Out>(d[i], k, mean, rstd, gamma_r, beta_r, qmax, q, m * K + k, s.bad);
+            }
+        } else {
+            constexpr int kB = 8;
+            for (int64_t k0 = (int64_t)lane * 8; k0 < K; k0 += 32 * 8 * kB) {
+                uint4 d[kB];
+#pragma unroll
+                for (int i = 0; i < kB; ++i) {
+                    const int64_t k = k0 + (int64_t)i * 32 * 8;
+                    d[i] = k < K ? __ldg(reinterpret_cast<const uint4 *>(row + k)) : make_uint4(0, 0, 0, 0);
+                }
+#pragma unroll
+                for (int i = 0; i < kB; ++i)
+                    if (k0 + (int64_t)i * 32 * 8 < K) ln_add8(s, d[i]);
+            }
+            ln_stats(s, K, eps, mean, rstd);
+            for (int64_t k0 = (int64_t)lane * 8; k0 < K; k0 += 32 * 8 * kB) {
+                uint4 d[kB];
+#pragma unroll
+                for (int i = 0; i < kB; ++i) {
+                    const int64_t k = k0 + (int64_t)i * 32 * 8;
+                    d[i] = k < K ? __ldcs(reinterpret_cast<const uint4 *>(row + k)) : make_uint4(0, 0, 0, 0);
+                }
+#pragma unroll
+                for (int i = 0; i < kB; ++i) {
+                    const int64_t k = k0 + (int64_t)i * 32 * 8;
+                    if (k < K) rs += ln_codes8<kF16Out>(d[i], k, mean, rstd, gamma_r, beta_r, qmax, q, m * K + k, s.bad);
+                }
+            }
+        }
+        if (rowsum) {
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) rs += __shfl_xor_sync(0xffffffffu, rs, o);
+            if (lane == 0) rowsum[m] = rs;
+        }
+    }
+}
+
+template <bool kF16Out>
+cudaError_t run_layernorm_quantize(const __half *h, int64_t M, int64_t K, int64_t ldh, const float *gamma_r,
+                                   const float *beta_r, float eps, int qmax, void *q, int32_t *rowsum,
+                                   cudaStream_t st) {
+    const int64_t ctas = (M + kLnWarps - 1) / kLnWarps;
+    const unsigned grid = (unsigned)(ctas < (1 << 30) ? ctas : (1 << 30));
+    const int64_t ch = (K + 255) / 256;  // 16-byte chunks per lane
+#define OT_LN_LAUNCH(C)                                                                                         \
+    layernorm_quantize_kernel<kF16Out, C><<<grid, kLnThreads, 0, st>>>(h, M, K, ldh, gamma_r, beta_r, eps, qmax, \
+                                                                       q, rowsum)
+    if (ch <= 4) OT_LN_LAUNCH(4);
+    else if (ch <= 8) OT_LN_LAUNCH(8);
+    else if (ch <= 16) OT_LN_LAUNCH(16);
+    else if (ch <= 24) OT_LN_LAUNCH(24);
+    else if (ch <= 32) OT_LN_LAUNCH(32);
+    else OT_LN_LAUNCH(0);
+#undef OT_LN_LAUNCH
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_fold_layernorm(const void *gamma, const void *beta, const float *z, const float *r, int64_t K,
+                                  float *gamma_r, float *beta_r, cudaStream_t st) {
+    fold_layernorm_kernel<<<(unsigned)((K + 255) / 256), 256, 0, st>>>(
+        reinterpret_cast<const __half *>(gamma), reinterpret_cast<const __half *>(beta), z, r, K, gamma_r, beta_r);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm_quantize(const void *h, int64_t M, int64_t K, int64_t ldh, const float *gamma_r,
+                                      const float *beta_r, float eps, int bits, void *q, int fmt,
+                                      int32_t *rowsum, cudaStream_t st) {
+    if (M == 0) return cudaSuccess;
+    const int qmax = (1 << (bits - 1)) - 1;
+    const __half *hh = reinterpret_cast<const __half *>(h);
+    if (fmt == OT_CODE_F16) return run_layernorm_quantize<true>(hh, M, K, ldh, gamma_r, beta_r, eps, qmax, q, rowsum, st);
+    return run_layernorm_quantize<false>(hh, M, K, ldh, gamma_r, beta_r, eps, qmax, q, rowsum, st);
+}
+
+}  // namespace ot

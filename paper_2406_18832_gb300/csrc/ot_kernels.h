@@ -21,6 +21,12 @@ cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, co
                             int bits, void *q, int fmt, cudaStream_t st, int32_t *rowsum = nullptr);
 cudaError_t launch_quantize_tokens(const void *x, int64_t M, int64_t K, int64_t ldx, int bits, void *q, int fmt,
                                    float *s_tok, cudaStream_t st);
+// LayerNorm fused with the symmetrization and quantization (layernorm.cu)
+cudaError_t launch_fold_layernorm(const void *gamma, const void *beta, const float *z, const float *r, int64_t K,
+                                  float *gamma_r, float *beta_r, cudaStream_t st);
+cudaError_t launch_layernorm_quantize(const void *h, int64_t M, int64_t K, int64_t ldh, const float *gamma_r,
+                                      const float *beta_r, float eps, int bits, void *q, int fmt,
+                                      int32_t *rowsum, cudaStream_t st);
 // asymmetric per-output-channel codes of W_s (zero points zc) and b'
 cudaError_t launch_fold_asym(const void *w, const void *b, int64_t N, int64_t K, const float *z, const float *s,
                              int bits_w, int8_t *qw, float *sw, int32_t *zc, float *bfold, cudaStream_t st);

@@ -64,6 +64,24 @@ class QuantizedLinear:
                               self.qw, self.sw, self.b_fold, symmetrize=self.symmetrize, stream=stream)
         return self
 
+    def fold_layernorm(self, gamma: torch.Tensor, beta: torch.Tensor, eps: float = 1e-5, stream=None):
+        """Fuse the LayerNorm in front of this linear into its quantize step
+        (Section 3.2): gamma * r and (beta - z) * r, after fold()."""
+        self.ln_gamma_r = torch.empty(self.K, dtype=torch.float32, device=self.z.device)
+        self.ln_beta_r = torch.empty(self.K, dtype=torch.float32, device=self.z.device)
+        self.ln_eps = float(eps)
+        B.ot_fold_layernorm(gamma, beta, self.z, self.r, self.ln_gamma_r, self.ln_beta_r, stream=stream)
+        return self
+
+    def forward_hidden(self, h: torch.Tensor, out: torch.Tensor | None = None, stream=None):
+        """y = linear(LayerNorm(h)) with the LayerNorm, symmetrization and
+        quantization in one kernel (fold_layernorm() first)."""
+        q = torch.empty(h.shape[0], self.K, dtype=torch.float16, device=h.device)
+        rs = torch.empty(h.shape[0], dtype=torch.int32, device=h.device) if self.asym else None
+        B.ot_layernorm_quantize(h, self.ln_gamma_r, self.ln_beta_r, self.ln_eps, self.bits_a, q, B.OT_CODE_F16,
+                                rowsum=rs, stream=stream)
+        return self.linear(q, out, stream, rowsum=rs)
+
     # ---- online ---------------------------------------------------------
     def quantize(self, x: torch.Tensor, out: torch.Tensor | None = None, stream=None):
         if out is None:

@@ -19,8 +19,9 @@ def _ln_ref(h, gamma, beta, eps):
 
 def test_ln_statistics_match_fp64_library():
     """mean and 1/sqrt(var + eps) from the exact integer sums agree with numpy's
-    fp64 mean / variance to within the final fp32 rounding, over rows with
-    large, small, subnormal and mixed-sign values."""
+    fp64 mean / variance to within the fp32 roundings of their definition
+    (mean: 2 roundings; rstd: at most 7 from the exact variance), over rows
+    with large, small, subnormal and mixed-sign values."""
     rng = np.random.default_rng(1)
     K = 1536
     rows = [rng.standard_normal(K), rng.standard_normal(K) * 1000 + 3000, rng.standard_normal(K) * 1e-3,
@@ -32,9 +33,9 @@ def test_ln_statistics_match_fp64_library():
     eps = 1e-5
     _, mean, rstd = oracle.layernorm_quantize(h, gr, br, eps, 8)[1:]
     _, mu, var = _ln_ref(h, np.ones(K), np.zeros(K), eps)
-    assert np.all(np.abs(mean.astype(np.float64) - mu) <= np.abs(mu) * 2 ** -23 + 1e-45)
+    assert np.all(np.abs(mean.astype(np.float64) - mu) <= np.abs(mu) * 2 * 2 ** -24 * 1.0001)
     want = 1 / np.sqrt(var + np.float64(np.float32(eps)))
-    assert np.all(np.abs(rstd.astype(np.float64) - want) <= want * 2 ** -23)
+    assert np.all(np.abs(rstd.astype(np.float64) - want) <= want * 7 * 2 ** -24)
 
 
 @pytest.mark.parametrize("a,c,eps", [(1.5, 0.25, 1.75), (4.0, -2.0, 0.0), (0.125, 64.0, 0.046875)])
