@@ -25,6 +25,8 @@ and the asymmetric weights ("Int8": per-output-channel zero points, Eq. 1):
 and the LayerNorm fused with the symmetrization and quantization (Section 3.2):
   fold_layernorm       - gamma * r and (beta - z) * r
   layernorm_quantize   - exact row statistics, codes of LN(h) - z scaled by r
+and the token-wise clipping calibration of bias-free models (Appendix D):
+  calibrate_clipped    - per-channel order statistics at quantile alpha
 """
 from __future__ import annotations
 
@@ -79,10 +81,11 @@ def _load():
             lib.oracle_epilogue_asym.argtypes = [P, P, P, I64, I64, P, P, I, P]
             lib.oracle_fold_layernorm.argtypes = [P, P, P, P, I64, P, P]
             lib.oracle_layernorm_quantize.argtypes = [P, I64, I64, I64, P, P, ctypes.c_float, I, P, P, P, P]
+            lib.oracle_calibrate_clipped.argtypes = [P, I64, I64, I64, ctypes.c_double, P, P]
             for f in ("oracle_calibrate", "oracle_params", "oracle_fold", "oracle_quantize",
                       "oracle_matmul", "oracle_epilogue", "oracle_quantize_tokens", "oracle_epilogue_tokens",
                       "oracle_fold_codes_asym", "oracle_rowsum", "oracle_epilogue_asym",
-                      "oracle_fold_layernorm", "oracle_layernorm_quantize"):
+                      "oracle_fold_layernorm", "oracle_layernorm_quantize", "oracle_calibrate_clipped"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -278,3 +281,13 @@ def layernorm_quantize(h: np.ndarray, gamma_r: np.ndarray, beta_r: np.ndarray, e
     _load().oracle_layernorm_quantize(_ptr(h), M, K, K, _ptr(_f32(gamma_r)), _ptr(_f32(beta_r)), float(eps), bits,
                                       _ptr(q), _ptr(rs), _ptr(mean), _ptr(rstd))
     return q, rs, mean, rstd
+
+
+def calibrate_clipped(x: np.ndarray, alpha: float):
+    """(lo, hi) fp32 [K]: per-channel order statistics of fp16 X_cal [T, K] at
+    ascending ranks T' + 1 - ceil(alpha T') and ceil(alpha T') (NaN ignored)."""
+    x = _f16(x)
+    T, K = x.shape
+    lo, hi = np.empty(K, np.float32), np.empty(K, np.float32)
+    _load().oracle_calibrate_clipped(_ptr(x), T, K, K, float(alpha), _ptr(lo), _ptr(hi))
+    return lo, hi

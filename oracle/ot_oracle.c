@@ -56,6 +56,14 @@
  *                operations, and the codes by one fp32 fma with the folded
  *                gamma * r and (beta - z) * r.  A row holding a non-finite
  *                value codes to 0 throughout.
+ *   R11 clipping the token-wise clipping the paper applies to bias-free
+ *                models (Appendix D, after Outlier Suppression) replaces each
+ *                channel's calibration min / max by order statistics over
+ *                the calibration tokens: with T' the non-NaN values of the
+ *                channel and rho = ceil(alpha * T') (fp64), the upper end is
+ *                the value of ascending rank rho and the lower end the value
+ *                of ascending rank T' + 1 - rho (alpha = 1: max and min).
+ *                fp16 values are ordered by value with -0 before +0.
  *
  * Floating point: compile with -ffp-contract=off and no fast-math, so every
  * fp32 expression below rounds once per operation as written.
@@ -63,6 +71,7 @@
 #include <stdint.h>
 #include <stddef.h>
 #include <math.h>
+#include <stdlib.h>
 #include <string.h>
 
 /* ---------------------------------------------------------------------------
@@ -494,4 +503,50 @@ void oracle_layernorm_quantize(const uint16_t *h, int64_t M, int64_t K, int64_t 
         }
         if (rowsum) rowsum[m] = rs;
     }
+}
+
+/* ---------------------------------------------------------------------------
+ * Token-wise clipping calibration (R11; Appendix D): per channel k of
+ * X_cal [T, K] (fp16, row stride ldx), the clipped range [lo_k, hi_k] at
+ * quantile alpha in (0, 1].  A channel without non-NaN values gets
+ * lo = +inf, hi = -inf (as min / max of nothing).
+ * ------------------------------------------------------------------------- */
+static uint16_t order_key(uint16_t h)       /* monotone in the fp16 value */
+{
+    return (h & 0x8000u) ? (uint16_t)~h : (uint16_t)(h | 0x8000u);
+}
+
+static int cmp_u16(const void *a, const void *b)
+{
+    const uint16_t x = *(const uint16_t *)a, y = *(const uint16_t *)b;
+    return (x > y) - (x < y);
+}
+
+void oracle_calibrate_clipped(const uint16_t *x, int64_t T, int64_t K, int64_t ldx, double alpha,
+                              float *lo, float *hi)
+{
+    uint16_t *keys = (uint16_t *)malloc((size_t)(T > 0 ? T : 1) * sizeof(uint16_t));
+    for (int64_t k = 0; k < K; ++k) {
+        int64_t n = 0;
+        for (int64_t t = 0; t < T; ++t) {
+            const uint16_t h = x[t * ldx + k];
+            if ((h & 0x7C00u) == 0x7C00u && (h & 0x03FFu)) continue;   /* NaN */
+            keys[n++] = order_key(h);
+        }
+        if (n == 0) {
+            lo[k] = INFINITY;
+            hi[k] = -INFINITY;
+            continue;
+        }
+        qsort(keys, (size_t)n, sizeof(uint16_t), cmp_u16);
+        int64_t rho = (int64_t)ceil(alpha * (double)n);
+        if (rho < 1) rho = 1;
+        if (rho > n) rho = n;
+        const uint16_t kh = keys[rho - 1], kl = keys[n - rho];
+        const uint16_t bh = (kh & 0x8000u) ? (uint16_t)(kh & 0x7FFFu) : (uint16_t)~kh;
+        const uint16_t bl = (kl & 0x8000u) ? (uint16_t)(kl & 0x7FFFu) : (uint16_t)~kl;
+        hi[k] = ot_half_to_float(bh);
+        lo[k] = ot_half_to_float(bl);
+    }
+    free(keys);
 }
