@@ -201,6 +201,25 @@ ot_status ot_linear_per_token(const void *q_f16, int64_t M, int64_t K, const int
                               void *stream);
 
 /*
+ * ot_calibrate_clipped -- token-wise clipping calibration for models whose
+ * linears have no bias (Appendix D: Llama cannot be symmetrized, and its
+ * static activation scales are calibrated with token-wise clipping).  Per
+ * channel k of X_cal [T, K] (fp16, row stride ldx), with T' the non-NaN
+ * values and rho = ceil(alpha * T') evaluated in fp64:
+ *   ch_hi[k] = the value of ascending rank rho,
+ *   ch_lo[k] = the value of ascending rank T' + 1 - rho
+ * (fp16 ordered by value, -0 before +0; alpha = 1 gives the min / max of
+ * ot_calibrate).  A channel without non-NaN values gets lo = +inf, hi = -inf.
+ * The whole calibration set is one call (order statistics do not accumulate
+ * batch by batch); pass the range to ot_derive_params / ot_fold_weights as
+ * ch_min / ch_max (symmetrize = 0 for bias-free models).
+ *   alpha    in (0, 1], e.g. 0.999 to drop the 0.1 % most extreme tokens per side
+ *   ch_lo, ch_hi  fp32 [K] out
+ */
+ot_status ot_calibrate_clipped(const void *x_f16, int64_t T, int64_t K, int64_t ldx,
+                               double alpha, float *ch_lo, float *ch_hi, void *stream);
+
+/*
  * LayerNorm fused with the symmetrization and the per-channel quantization
  * (Section 3.2: the codes of Eq. 7 come out of the LayerNorm before the linear,
  * whose gamma and beta absorb the scale r and the shift z).  For the linears

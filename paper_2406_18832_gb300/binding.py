@@ -44,6 +44,7 @@ _SIGNATURES = {
                        _I),
     "ot_fold_layernorm": ([_P, _P, _P, _P, _I64, _P, _P, _P], _I),
     "ot_layernorm_quantize": ([_P, _I64, _I64, _I64, _P, _P, _F, _I, _P, _I, _P, _P], _I),
+    "ot_calibrate_clipped": ([_P, _I64, _I64, _I64, ctypes.c_double, _P, _P, _P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -125,6 +126,15 @@ def ot_calibrate(x: torch.Tensor, ch_min: torch.Tensor, ch_max: torch.Tensor, re
     _check(load().ot_calibrate(px, T, K, ldx, _dev(ch_min, "ch_min", torch.float32),
                                _dev(ch_max, "ch_max", torch.float32), 1 if reset else 0, _stream(stream)),
            "ot_calibrate")
+
+
+def ot_calibrate_clipped(x: torch.Tensor, alpha: float, ch_lo: torch.Tensor, ch_hi: torch.Tensor, stream=None):
+    """Token-wise clipped per-channel range of fp16 X_cal [T, K] at quantile alpha (order statistics)."""
+    T, K, ldx = _rows(x, "x")
+    _check(load().ot_calibrate_clipped(_dev(x, "x", torch.float16), T, K, ldx, float(alpha),
+                                       _dev(ch_lo, "ch_lo", torch.float32), _dev(ch_hi, "ch_hi", torch.float32),
+                                       _stream(stream)),
+           "ot_calibrate_clipped")
 
 
 def ot_derive_params(ch_min, ch_max, bits_a: int, z, s, r, symmetrize: bool = True, stream=None):

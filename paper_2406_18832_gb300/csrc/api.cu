@@ -61,6 +61,15 @@ ot_status ot_calibrate(const void *x_f16, int64_t T, int64_t K, int64_t ldx, flo
     return from_cuda(ot::launch_calibrate(x_f16, T, K, ldx, ch_min, ch_max, reset, as_stream(stream)));
 }
 
+ot_status ot_calibrate_clipped(const void *x_f16, int64_t T, int64_t K, int64_t ldx, double alpha, float *ch_lo,
+                               float *ch_hi, void *stream) {
+    if (T < 0 || K <= 0 || ldx < K || !(alpha > 0.0) || !(alpha <= 1.0)) return OT_ERR_INVALID_ARG;
+    if (!ch_lo || !ch_hi || !aligned(ch_lo, 4) || !aligned(ch_hi, 4)) return OT_ERR_INVALID_ARG;
+    if (T > 0 && (!x_f16 || !aligned(x_f16, 2))) return OT_ERR_INVALID_ARG;
+    if (T > kIntMax) return OT_ERR_UNSUPPORTED;  // 32-bit histogram counts
+    return from_cuda(ot::launch_calibrate_clipped(x_f16, T, K, ldx, alpha, ch_lo, ch_hi, as_stream(stream)));
+}
+
 ot_status ot_derive_params(const float *ch_min, const float *ch_max, int64_t K, int bits_a, int symmetrize,
                            float *z, float *s, float *r, void *stream) {
     if (K <= 0 || !bits_ok(bits_a)) return OT_ERR_INVALID_ARG;

@@ -21,6 +21,9 @@ cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, co
                             int bits, void *q, int fmt, cudaStream_t st, int32_t *rowsum = nullptr);
 cudaError_t launch_quantize_tokens(const void *x, int64_t M, int64_t K, int64_t ldx, int bits, void *q, int fmt,
                                    float *s_tok, cudaStream_t st);
+// token-wise clipping calibration: per-channel order statistics (clip.cu)
+cudaError_t launch_calibrate_clipped(const void *x, int64_t T, int64_t K, int64_t ldx, double alpha, float *lo,
+                                     float *hi, cudaStream_t st);
 // LayerNorm fused with the symmetrization and quantization (layernorm.cu)
 cudaError_t launch_fold_layernorm(const void *gamma, const void *beta, const float *z, const float *r, int64_t K,
                                   float *gamma_r, float *beta_r, cudaStream_t st);

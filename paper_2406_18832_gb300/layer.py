@@ -51,6 +51,13 @@ class QuantizedLinear:
         self._calibrated = True
         return self
 
+    def calibrate_clipped(self, x_cal: torch.Tensor, alpha: float = 0.999, stream=None):
+        """Token-wise clipping calibration (Appendix D, for bias-free models;
+        use symmetrize=False): the whole calibration set [T, K] in one call."""
+        B.ot_calibrate_clipped(x_cal, alpha, self.ch_min, self.ch_max, stream=stream)
+        self._calibrated = True
+        return self
+
     def fold(self, w: torch.Tensor, b: torch.Tensor | None, stream=None):
         """Derive z, s, r from the calibration and fold them into W and b."""
         if not self._calibrated:
