@@ -27,6 +27,8 @@ and the LayerNorm fused with the symmetrization and quantization (Section 3.2):
   layernorm_quantize   - exact row statistics, codes of LN(h) - z scaled by r
 and the token-wise clipping calibration of bias-free models (Appendix D):
   calibrate_clipped    - per-channel order statistics at quantile alpha
+and the epilogue that writes the next linear's codes (fc1 -> ReLU -> fc2):
+  epilogue_quantize    - round((fma(acc, sw, b') [ReLU] - z') * r')
 """
 from __future__ import annotations
 
@@ -82,10 +84,12 @@ def _load():
             lib.oracle_fold_layernorm.argtypes = [P, P, P, P, I64, P, P]
             lib.oracle_layernorm_quantize.argtypes = [P, I64, I64, I64, P, P, ctypes.c_float, I, P, P, P, P]
             lib.oracle_calibrate_clipped.argtypes = [P, I64, I64, I64, ctypes.c_double, P, P]
+            lib.oracle_epilogue_quantize.argtypes = [P, I64, I64, P, P, I, P, P, I, P]
             for f in ("oracle_calibrate", "oracle_params", "oracle_fold", "oracle_quantize",
                       "oracle_matmul", "oracle_epilogue", "oracle_quantize_tokens", "oracle_epilogue_tokens",
                       "oracle_fold_codes_asym", "oracle_rowsum", "oracle_epilogue_asym",
-                      "oracle_fold_layernorm", "oracle_layernorm_quantize", "oracle_calibrate_clipped"):
+                      "oracle_fold_layernorm", "oracle_layernorm_quantize", "oracle_calibrate_clipped",
+                      "oracle_epilogue_quantize"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -291,3 +295,14 @@ def calibrate_clipped(x: np.ndarray, alpha: float):
     lo, hi = np.empty(K, np.float32), np.empty(K, np.float32)
     _load().oracle_calibrate_clipped(_ptr(x), T, K, K, float(alpha), _ptr(lo), _ptr(hi))
     return lo, hi
+
+
+def epilogue_quantize(acc: np.ndarray, sw: np.ndarray, bfold: np.ndarray, z_next: np.ndarray, r_next: np.ndarray,
+                      bits_next: int, relu: bool = False) -> np.ndarray:
+    """int8 codes q'[M, N] = round((fma((float)acc, sw, b') [ReLU] - z') * r') of the next layer."""
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
+    M, N = acc.shape
+    q = np.empty((M, N), np.int8)
+    _load().oracle_epilogue_quantize(_ptr(acc), M, N, _ptr(_f32(sw)), _ptr(_f32(bfold)), 1 if relu else 0,
+                                     _ptr(_f32(z_next)), _ptr(_f32(r_next)), bits_next, _ptr(q))
+    return q

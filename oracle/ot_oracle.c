@@ -64,6 +64,13 @@
  *                the value of ascending rank rho and the lower end the value
  *                of ascending rank T' + 1 - rho (alpha = 1: max and min).
  *                fp16 values are ordered by value with -0 before +0.
+ *   R12 chaining when a linear's output feeds the next per-channel
+ *                quantized linear (fc1 -> ReLU -> fc2, Section 3.2's fusion
+ *                carried to the fc1 epilogue), the epilogue can write the
+ *                next layer's codes directly: the fp32 value v of R8 (after
+ *                ReLU) is quantized as round((v - z') * r') with the next
+ *                layer's z', r' (R1-R3, R6); the fp16 rounding of y is
+ *                skipped.
  *
  * Floating point: compile with -ffp-contract=off and no fast-math, so every
  * fp32 expression below rounds once per operation as written.
@@ -549,4 +556,26 @@ void oracle_calibrate_clipped(const uint16_t *x, int64_t T, int64_t K, int64_t l
         lo[k] = ot_half_to_float(bl);
     }
     free(keys);
+}
+
+/* ---------------------------------------------------------------------------
+ * Step A6'' (R12): the epilogue of a linear whose output is the next linear's
+ * input, writing that layer's codes instead of y:
+ *   v = fma((float)acc[m,n], sw_n, b'_n),  ReLU if relu,
+ *   q'[m,n] = round_half_even((v - z'_n) * r'_n) in [-qmax', qmax']   (fp32)
+ * z', r' [N] are the next layer's symmetrization and reciprocal scale.
+ * ------------------------------------------------------------------------- */
+void oracle_epilogue_quantize(const int64_t *acc, int64_t M, int64_t N, const float *sw,
+                              const float *bfold, int relu, const float *zn, const float *rn,
+                              int bits_next, int8_t *q)
+{
+    const int qmax = qmax_of(bits_next);
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t n = 0; n < N; ++n) {
+            float a = (float)acc[m * N + n];
+            float v = fmaf(a, sw[n], bfold[n]);
+            if (relu && !(v > 0.0f)) v = 0.0f;
+            float t = v - zn[n];
+            q[m * N + n] = (int8_t)quantize_code(t * rn[n], qmax);
+        }
 }
