@@ -610,7 +610,8 @@ def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):
     """The chained linear path of an OPT-30B-shaped decoder block (hidden 7168,
     FFN 28672; QKV -> V slice -> out -> fc1 + ReLU -> fc2, each layer calibrated
     on what it receives) at 8 x 512 tokens, Int8 and Int6: latency, weight and
-    activation bytes against the same chain of cuBLAS fp16 GEMMs."""
+    activation bytes against the same chain of cuBLAS fp16 GEMMs; also with
+    fc1's epilogue writing fc2's codes (the chained epilogue)."""
     import torch
 
     from paper_2406_18832_gb300 import QuantizedBlockLinears, synth
@@ -639,7 +640,11 @@ def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):
         blk = QuantizedBlockLinears(h, ffn, bits, bits, device=dev)
         blk.calibrate(x_cal, weights)
         ms = timed(lambda: blk.forward(x))
+        # fc1's epilogue writes fc2's codes: f is neither written nor re-read
+        ms_f = timed(lambda: blk.forward(x, fused=True))
         out[f"int{bits}"] = {"ms": round(ms, 4), "tops": round(ops / (ms * 1e-3) / 1e12, 1),
+                             "ms_fc1_fc2_chained": round(ms_f, 4),
+                             "tops_fc1_fc2_chained": round(ops / (ms_f * 1e-3) / 1e12, 1),
                              "weight_bytes": blk.weight_bytes()}
         del blk
     w16 = [w for w, _ in weights]
@@ -656,7 +661,9 @@ def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):
     # activation bytes per block: fp16 inputs read (x, v, o, f) and outputs written
     # (qkv, o, f, y); the quantized path also writes and reads each layer's fp16 codes
     act16 = 2 * tokens * ((h + h + h + ffn) + (3 * h + h + ffn + h))
-    out["activation_bytes"] = {"fp16_path": act16, "quantized_path": act16 + 4 * tokens * (h + h + h + ffn)}
+    quant = act16 + 4 * tokens * (h + h + h + ffn)
+    out["activation_bytes"] = {"fp16_path": act16, "quantized_path": quant,
+                               "quantized_fc1_fc2_chained": quant - 4 * tokens * ffn}
     del weights, x_cal, x
     torch.cuda.empty_cache()
     return out

@@ -307,6 +307,26 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
                          size_t workspace_bytes, void *stream);
 
 /*
+ * ot_linear_quantize_next -- a linear whose output is the input of the next
+ * per-channel quantized linear (fc1 -> ReLU -> fc2), with that layer's
+ * activation quantization done in this epilogue (Section 3.2 fuses the
+ * quantization into the producing kernel):
+ *   v = fma((float)acc[m,n], sw_n, b'_n), then ReLU if relu,
+ *   q_next[m,n] = round_half_even((v - z_next[n]) * r_next[n]) in [-qmax', qmax']
+ * written as fp16 integers [M, ldq] -- the codes ot_linear takes as q_f16 for
+ * the next layer, whose K is this layer's N.  The fp16 rounding of y is
+ * skipped, so codes can differ by one from quantizing the fp16 y at a tie.
+ * Arguments as ot_linear; z_next, r_next fp32 [N] (the next layer's z, r);
+ * bits_next in [2, 8].  Symmetric weights only.
+ */
+ot_status ot_linear_quantize_next(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
+                                  const float *sw, const float *b_fold, int64_t N, int bits_a,
+                                  int bits_w, int relu, const float *z_next,
+                                  const float *r_next, int bits_next, void *q_next_f16,
+                                  int64_t ldq, void *workspace, size_t workspace_bytes,
+                                  void *stream);
+
+/*
  * ot_linear_noalloc -- ot_linear for callers that cannot allocate device
  * memory: for example a server or plugin that owns all GPU memory through
  * its own pool and forbids further cudaMalloc calls, or code that must not

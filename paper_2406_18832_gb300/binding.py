@@ -45,6 +45,8 @@ _SIGNATURES = {
     "ot_fold_layernorm": ([_P, _P, _P, _P, _I64, _P, _P, _P], _I),
     "ot_layernorm_quantize": ([_P, _I64, _I64, _I64, _P, _P, _F, _I, _P, _I, _P, _P], _I),
     "ot_calibrate_clipped": ([_P, _I64, _I64, _I64, ctypes.c_double, _P, _P, _P], _I),
+    "ot_linear_quantize_next": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _I, _P, _P, _I, _P, _I64, _P,
+                                 ctypes.c_size_t, _P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -237,6 +239,25 @@ def ot_layernorm_quantize(h, gamma_r, beta_r, eps: float, bits_a: int, q, q_form
                                         _dev(beta_r, "beta_r", torch.float32), float(eps), bits_a,
                                         _dev(q, "q", want), q_format, prs, _stream(stream)),
            "ot_layernorm_quantize")
+
+
+def ot_linear_quantize_next(q, qw, sw, b_fold, bits_a: int, bits_w: int, z_next, r_next, bits_next: int, q_next,
+                            relu: bool = False, workspace=None, stream=None):
+    """The linear whose epilogue writes the next layer's fp16 codes q_next [M, N] (fc1 -> ReLU -> fc2)."""
+    _dense(q, "q")
+    _dense(qw, "qw")
+    M, K = q.shape
+    N = qw.shape[0]
+    qm, qn, ldq = _rows(q_next, "q_next")
+    if qm != M or qn != N:
+        raise ValueError("q_next must be [M, N]")
+    wp, wb = _ws_args(workspace, q.device, stream)
+    _check(load().ot_linear_quantize_next(_dev(q, "q", torch.float16), M, K, _dev(qw, "qw", torch.int8),
+                                          _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32), N,
+                                          bits_a, bits_w, 1 if relu else 0, _dev(z_next, "z_next", torch.float32),
+                                          _dev(r_next, "r_next", torch.float32), bits_next,
+                                          _dev(q_next, "q_next", torch.float16), ldq, wp, wb, _stream(stream)),
+           "ot_linear_quantize_next")
 
 
 def ot_linear_workspace_size() -> int:

@@ -232,6 +232,23 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
+ot_status ot_linear_quantize_next(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw,
+                                  const float *b_fold, int64_t N, int bits_a, int bits_w, int relu,
+                                  const float *z_next, const float *r_next, int bits_next, void *q_next_f16,
+                                  int64_t ldq, void *workspace, size_t workspace_bytes, void *stream) {
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, q_next_f16);
+    if (v != OT_OK) return v;
+    if (!sw || !b_fold || !z_next || !r_next || !bits_ok(bits_next) || ldq < N) return OT_ERR_INVALID_ARG;
+    if (!aligned(z_next, 4) || !aligned(r_next, 4) || (q_next_f16 && !aligned(q_next_f16, 2)))
+        return OT_ERR_INVALID_ARG;
+    if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
+    if (ldq > kIntMax) return OT_ERR_UNSUPPORTED;
+    ot::LinearArgs a{q_f16, qw, sw, b_fold, q_next_f16, M, N, K, ldq, bits_a, bits_w, relu ? 1 : 0, false,
+                     workspace, workspace ? workspace_bytes : 0, nullptr, nullptr, nullptr, z_next, r_next,
+                     (int)qmax_of(bits_next)};
+    return from_cuda(ot::launch_linear(a, as_stream(stream)));
+}
+
 ot_status ot_linear_noalloc(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw,
                             const float *b_fold, int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy,
                             int relu, void *stream) {

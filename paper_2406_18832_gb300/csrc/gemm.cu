@@ -94,12 +94,13 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     hi = *reinterpret_cast<const uint32_t *>(&hb);
 }
 
-template <int BN, bool kS32, bool kAsym>
+template <int BN, bool kS32, bool kAsym, bool kQOut>
 __global__ void __launch_bounds__(kThreads, 1)
     linear_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                   const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
                   int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok,
-                  const int32_t *__restrict__ zc, const int32_t *__restrict__ rowsum) {
+                  const int32_t *__restrict__ zc, const int32_t *__restrict__ rowsum,
+                  const float *__restrict__ zq, const float *__restrict__ rq, int qmax_out) {
     extern __shared__ uint8_t smem_raw[];
     Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -271,6 +272,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
                     const int32_t zn = kAsym ? __ldg(zc + n) : 0;
+                    // chained epilogue: the next layer's z', r' for channel n
+                    const float zqn = kQOut ? __ldg(zq + n) : 0.f, rqn = kQOut ? __ldg(rq + n) : 0.f;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
                     for (int j = 0; j < CPW; ++j) {
@@ -286,7 +289,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                              : tot[j]);
                         float v = __fmaf_rn(a, sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
-                        if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                        if constexpr (kQOut) {
+                            // the next layer's code round((v - z') * r'), as an fp16 integer
+                            const int c = __float2int_rn(__fmul_rn(__fsub_rn(v, zqn), rqn));
+                            if (m < M) o[(int64_t)m * ldy + n] = __int2half_rn(max(-qmax_out, min(qmax_out, c)));
+                        } else {
+                            if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                        }
                     }
                 }
             }
@@ -419,13 +428,14 @@ __device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) 
     return v;
 }
 
-template <bool kS32, bool kAsym>
+template <bool kS32, bool kAsym, bool kQOut>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
                        int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws, uint64_t epoch,
                        const float *__restrict__ s_tok, const int32_t *__restrict__ zc,
-                       const int32_t *__restrict__ rowsum) {
+                       const int32_t *__restrict__ rowsum, const float *__restrict__ zq,
+                       const float *__restrict__ rq, int qmax_out) {
     extern __shared__ uint8_t smem_raw[];
     SmemPair &S = *reinterpret_cast<SmemPair *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -656,6 +666,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
                     const int32_t zn = kAsym ? __ldg(zc + n) : 0;
+                    // chained epilogue: the next layer's z', r' for channel n
+                    const float zqn = kQOut ? __ldg(zq + n) : 0.f, rqn = kQOut ? __ldg(rq + n) : 0.f;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
                     for (int j = 0; j < 128; ++j) {
@@ -671,7 +683,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                                              : tot[j]);
                         float v = __fmaf_rn(a, sc, bias);
                         if (relu) v = fmaxf(v, 0.f);
-                        if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                        if constexpr (kQOut) {
+                            // the next layer's code round((v - z') * r'), as an fp16 integer
+                            const int c = __float2int_rn(__fmul_rn(__fsub_rn(v, zqn), rqn));
+                            if (m < M) o[(int64_t)m * ldy + n] = __int2half_rn(max(-qmax_out, min(qmax_out, c)));
+                        } else {
+                            if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                        }
                     }
                 }
             }
@@ -730,7 +748,7 @@ bool make_tmap_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uin
     return r == CUDA_SUCCESS;
 }
 
-template <int BN, bool kS32, bool kAsym>
+template <int BN, bool kS32, bool kAsym, bool kQOut>
 cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
     if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
@@ -743,15 +761,15 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32, kAsym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32, kAsym, kQOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
-    linear_kernel<BN, kS32, kAsym><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
+    linear_kernel<BN, kS32, kAsym, kQOut><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
                                                          (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
-                                                         a.rowsum);
+                                                         a.rowsum, a.zq, a.rq, a.qmax_out);
     return cudaGetLastError();
 }
 
@@ -765,7 +783,7 @@ int pair_max_clusters() {
     if (dev_cached == dev) return value;
     const size_t smem = sizeof(SmemPair) + 1024;
     int n = 0;
-    if (cudaFuncSetAttribute(linear_pair_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+    if (cudaFuncSetAttribute(linear_pair_kernel<false, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
         cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 256);
@@ -778,7 +796,7 @@ int pair_max_clusters() {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<false, false>, &cfg) != cudaSuccess) n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<false, false, false>, &cfg) != cudaSuccess) n = 0;
     }
     cudaGetLastError();
     if (n <= 0) n = num_sms() / 2;
@@ -787,7 +805,7 @@ int pair_max_clusters() {
     return n;
 }
 
-template <bool kS32, bool kAsym>
+template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
     if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
@@ -799,7 +817,7 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32, kAsym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32, kAsym, kQOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
@@ -818,18 +836,19 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
     const uint64_t epoch = streamk ? next_epoch() : 0;
-    linear_pair_kernel<kS32, kAsym><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
+    linear_pair_kernel<kS32, kAsym, kQOut><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
                                                                 (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
-                                                                epoch, a.s_tok, a.zc, a.rowsum);
+                                                                epoch, a.s_tok, a.zc, a.rowsum, a.zq, a.rq,
+                                                                a.qmax_out);
     return cudaGetLastError();
 }
 
 // M <= 32 goes to the decode kernel (gemv.cu) before this dispatch.
-template <bool kS32, bool kAsym>
+template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
-    if (a.M <= 64) return run_linear<64, kS32, kAsym>(a, kcb, st);
-    if (a.M <= 128) return run_linear<128, kS32, kAsym>(a, kcb, st);
-    return run_linear_pair<kS32, kAsym>(a, kcb, st);
+    if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut>(a, kcb, st);
+    if (a.M <= 128) return run_linear<128, kS32, kAsym, kQOut>(a, kcb, st);
+    return run_linear_pair<kS32, kAsym, kQOut>(a, kcb, st);
 }
 
 }  // namespace
@@ -917,8 +936,9 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
         d.workspace_bytes = room ? a.workspace_bytes - off : 0;
         return launch_linear_gemv(d, kcb, st);
     }
-    if (a.out_s32) return dispatch_bn<true, false>(a, kcb, st);
-    return a.zc ? dispatch_bn<false, true>(a, kcb, st) : dispatch_bn<false, false>(a, kcb, st);
+    if (a.out_s32) return dispatch_bn<true, false, false>(a, kcb, st);
+    if (a.zq) return dispatch_bn<false, false, true>(a, kcb, st);
+    return a.zc ? dispatch_bn<false, true, false>(a, kcb, st) : dispatch_bn<false, false, false>(a, kcb, st);
 }
 
 }  // namespace ot

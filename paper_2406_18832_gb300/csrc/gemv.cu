@@ -69,6 +69,8 @@ constexpr int kGvSlotInts = kGvRows * 32;         // workspace ints per split ti
 struct GvParams {
     const float *sw, *bfold, *s_tok;
     const int32_t *zc, *rowsum;    // asymmetric weights: zero points [N], code row sums [M] (or null)
+    const float *zq, *rq;          // chained epilogue: the next layer's z', r' [N] (or null)
+    int qmax_out;
     void *out;
     int32_t *part;                 // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
     unsigned long long *flags;     // [grid] launch epoch once a CTA's slot is complete
@@ -132,7 +134,14 @@ __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32
             p.zc ? (int32_t)((uint32_t)s - (uint32_t)__ldg(p.zc + n) * (uint32_t)__ldg(p.rowsum + m)) : s);
         float v = __fmaf_rn(a, sc, __ldg(p.bfold + n));
         if (p.relu) v = fmaxf(v, 0.f);
-        reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = __float2half_rn(v);
+        __half o;
+        if (p.zq) {  // the next layer's code round((v - z') * r'), as an fp16 integer
+            const int c = __float2int_rn(__fmul_rn(__fsub_rn(v, __ldg(p.zq + n)), __ldg(p.rq + n)));
+            o = __int2half_rn(max(-p.qmax_out, min(p.qmax_out, c)));
+        } else {
+            o = __float2half_rn(v);
+        }
+        reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = o;
     }
 }
 
@@ -422,6 +431,9 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     p.s_tok = a.s_tok;
     p.zc = a.zc;
     p.rowsum = a.rowsum;
+    p.zq = a.zq;
+    p.rq = a.rq;
+    p.qmax_out = a.qmax_out;
     p.out = a.out;
     p.status = device_status_word();
     if (!p.status) return cudaErrorUnknown;

@@ -51,6 +51,8 @@ struct LinearArgs {
     const float *s_tok;       // per-token path: token scales [M] (y uses s_tok[m] * sw[n]); null otherwise
     const int32_t *zc;        // asymmetric weights: zero points [N] (stored codes' scale), or null
     const int32_t *rowsum;    // with zc: sum_k q[m,k] [M]
+    const float *zq, *rq;     // chained epilogue: the next layer's z', r' [N] (out then holds fp16 codes), or null
+    int qmax_out;             // with zq: the next layer's qmax
 };
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();

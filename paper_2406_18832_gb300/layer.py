@@ -120,6 +120,21 @@ class QuantizedLinear:
                         stream=stream)
         return out
 
+    def linear_quantize_next(self, q: torch.Tensor, nxt: "QuantizedLinear", out: torch.Tensor | None = None,
+                             stream=None):
+        """This layer's linear with the next layer's activation quantization in
+        its epilogue (Section 3.2): returns nxt's fp16 codes [M, N], the q that
+        nxt.linear takes, without this layer's fp16 output."""
+        if self.asym:
+            raise ValueError("the chained epilogue takes symmetric weights")
+        if nxt.K != self.N:
+            raise ValueError("the next layer's in_features must equal this layer's out_features")
+        if out is None:
+            out = torch.empty(q.shape[0], self.N, dtype=torch.float16, device=q.device)
+        B.ot_linear_quantize_next(q, self.qw, self.sw, self.b_fold, self.bits_a, self.bits_w, nxt.z, nxt.r,
+                                  nxt.bits_a, out, relu=self.relu, stream=stream)
+        return out
+
     def forward(self, x: torch.Tensor, q_buf: torch.Tensor | None = None, out: torch.Tensor | None = None,
                 stream=None):
         if self.asym:
@@ -180,10 +195,15 @@ class QuantizedBlockLinears:
                 acts = nxt[:, 2 * self.h:] if ql is self.qkv else nxt
         return self
 
-    def forward(self, x: torch.Tensor, stream=None):
-        """All intermediate outputs: qkv, o, f, y (fp16)."""
+    def forward(self, x: torch.Tensor, stream=None, fused: bool = False):
+        """All intermediate outputs: qkv, o, f, y (fp16).  fused=True chains
+        fc1 into fc2 through codes: fc1's epilogue (ReLU) writes fc2's
+        activation codes qf in place of f, so f never reaches HBM."""
         qkv = self.qkv(x, stream=stream)
         o = self.out(qkv[:, 2 * self.h:], stream=stream)
+        if fused:
+            qf = self.fc1.linear_quantize_next(self.fc1.quantize(o, stream=stream), self.fc2, stream=stream)
+            return dict(qkv=qkv, o=o, qf=qf, y=self.fc2.linear(qf, stream=stream))
         f = self.fc1(o, stream=stream)
         y = self.fc2(f, stream=stream)
         return dict(qkv=qkv, o=o, f=f, y=y)

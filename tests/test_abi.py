@@ -69,6 +69,7 @@ def _linear_args(handle):
     handle.ot_linear_asym.argtypes = [P, I64, I64, P, P, P, P, P, I64, I, I, P, I64, I, P, S, P]
     handle.ot_quantize_act_rowsum.argtypes = [P, I64, I64, I64, P, P, I, P, I, P, P]
     handle.ot_fold_weights_asym.argtypes = [P, P, I, I, P, P, I64, I64, I, P, P, P, P, P, P, P, P]
+    handle.ot_linear_quantize_next.argtypes = [P, I64, I64, P, P, P, I64, I, I, I, P, P, I, P, I64, P, S, P]
 
 
 # Fake, 256-byte-aligned addresses: every call below must be rejected on the
@@ -120,6 +121,12 @@ def test_validation_rejects_bad_arguments_before_launch(lib):
     assert handle.ot_quantize_act_rowsum(A, 4, 64, 64, A, A, 8, A2, 1, None, None) == INV
     assert handle.ot_quantize_act_rowsum(A, 4, 64, 64, A, A, 8, A2, 1, A + 2, None) == INV
     assert handle.ot_fold_weights_asym(A, A, 8, 1, A, None, 16, 64, 8, A, A, A, A2, A, None, A, None) == INV
+    # chained epilogue: null / unaligned z', r', next bits outside [2, 8], ldq < N
+    qn = handle.ot_linear_quantize_next
+    assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, None, A, 8, A, 16, None, 0, None) == INV
+    assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, A, A + 2, 8, A, 16, None, 0, None) == INV
+    assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, A, A, 9, A, 16, None, 0, None) == INV
+    assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, A, A, 8, A, 15, None, 0, None) == INV
 
 
 def test_binding_refuses_host_tensors():
