@@ -543,6 +543,26 @@ def bench_clipping(dev, peaks, calib_ms, calib_bytes, reps: int = 3):
             "minmax_ms": round(calib_ms[0], 3), "note": "two passes over the data (radix select on fp16 keys)"}
 
 
+def _graph_ms(calls, reps):
+    """ms per call of `calls` (reps calls) captured in a CUDA graph, replayed 3 times."""
+    import torch
+    calls()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        calls()
+    graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(3):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    del graph
+    return e0.elapsed_time(e1) / (3 * reps)
+
+
 def bench_decode(dev, peaks, reps: int = 50):
     """Decode-sized linears of the OPT-13B shapes (Int6; 1 and 16 tokens): the
     product is bound by streaming the int8 weights from HBM, so the roofline is
@@ -596,12 +616,30 @@ def bench_decode(dev, peaks, reps: int = 50):
             ms = e0.elapsed_time(e1) / (3 * reps)
             del graph
             gbs = layer.N * layer.K / (ms * 1e-3) / 1e9
+            # with the activation quantization in front: two calls, or the
+            # fused call (the linear a programmatic dependent of the quantize)
+            x = q.clone()
+            z0, r1 = torch.zeros(layer.K, device=dev), torch.ones(layer.K, device=dev)
+            qs = torch.empty_like(q)
+
+            def two_calls():
+                for i in range(reps):
+                    binding.ot_quantize_act(x, z0, r1, 6, qs, binding.OT_CODE_F16)
+                    binding.ot_linear(qs, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
+
+            def fused_calls():
+                for i in range(reps):
+                    binding.ot_linear_fused(x, z0, r1, 6, qws[i % copies], sw, bf, 6, qs, y, workspace=ws)
+
+            ms_two, ms_fused = _graph_ms(two_calls, reps), _graph_ms(fused_calls, reps)
             res.append({"layer": layer.name, "K": layer.K, "N": layer.N, "tokens": M, "us": round(ms * 1e3, 2),
                         "weight_gbs": round(gbs, 1), "frac_hbm": round(gbs / peaks["hbm"], 4),
-                        "eager_us": round(eager_ms * 1e3, 2)})
+                        "eager_us": round(eager_ms * 1e3, 2), "quantize_then_linear_us": round(ms_two * 1e3, 2),
+                        "fused_us": round(ms_fused * 1e3, 2)})
         del qws
     return {"workload": "opt-13b decode-sized linears, Int6", "kernel": "linear_gemv_kernel (mma.sync, TMA stream)",
-            "bound": "hbm", "timing": "CUDA graph replay of consecutive calls (eager_us: one Python call each)",
+            "bound": "hbm", "timing": "CUDA graph replay of consecutive calls (eager_us: one Python call each); "
+            "quantize_then_linear_us / fused_us: ot_quantize_act + ot_linear per call, or ot_linear_fused",
             "l2": "consecutive calls read different weight copies, > 3x L2 in all",
             "per_shape": res}
 

@@ -134,7 +134,10 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  *   y_f16   fp16 [M, N], row stride ldy >= N
  *   workspace, workspace_bytes  optional device scratch (16-byte aligned) of
  *           at least ot_linear_workspace_size() bytes, ZERO-FILLED before its
- *           first use; the kernel leaves it valid for the next call.  With it,
+ *           first use; the kernels keep it valid for every later call,
+ *           including calls replayed from a CUDA graph (a launch counter in
+ *           the workspace, not a value fixed at launch, tells one call's
+ *           partial sums from another's).  With it,
  *           prefill-sized calls (M > 128) and decode-sized calls (M <= 32) may
  *           share the (tile, K-slice) work evenly over the SMs and exchange
  *           exact int32 partial sums through it (stream-K); with NULL / too
@@ -305,6 +308,26 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
                          const float *b_fold, int64_t N, int bits_a, int bits_w,
                          void *y_f16, int64_t ldy, int relu, void *workspace,
                          size_t workspace_bytes, void *stream);
+
+/*
+ * ot_linear_fused -- ot_quantize_act followed by ot_linear in one call (the
+ * activation quantization of Eq. 6-7 fused in front of the product, as
+ * Section 3.2 fuses it with the operation producing X): q = codes of X
+ * (fp16 integers), y = fp16(fma(sum_k q qw, sw_n, b'_n)), ReLU if relu.
+ * The linear is launched as a programmatic dependent of the quantization, so
+ * its weight stream and set-up overlap the quantization and only its reads of
+ * the codes wait for it.
+ * x_f16 fp16 [M, ldx] (ldx >= K, ldx % 8 == 0, 16-byte aligned); z, r fp32 [K]
+ * (16-byte aligned); q_f16: caller scratch fp16 [M, K], dense, 16-byte
+ * aligned, receives the codes (valid after the stream synchronizes); the
+ * remaining arguments as ot_linear.  Same validation and errors as the two
+ * calls; M == 0 launches nothing.
+ */
+ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z,
+                          const float *r, int bits_a, const int8_t *qw, const float *sw,
+                          const float *b_fold, int64_t N, int bits_w, void *q_f16, void *y_f16,
+                          int64_t ldy, int relu, void *workspace, size_t workspace_bytes,
+                          void *stream);
 
 /*
  * ot_linear_quantize_next -- a linear whose output is the input of the next

@@ -47,6 +47,8 @@ _SIGNATURES = {
     "ot_calibrate_clipped": ([_P, _I64, _I64, _I64, ctypes.c_double, _P, _P, _P], _I),
     "ot_linear_quantize_next": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _I, _P, _P, _I, _P, _I64, _P,
                                  ctypes.c_size_t, _P], _I),
+    "ot_linear_fused": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _P, _P, _I64, _I, _P, _P, _I64, _I, _P,
+                         ctypes.c_size_t, _P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
 }
@@ -239,6 +241,26 @@ def ot_layernorm_quantize(h, gamma_r, beta_r, eps: float, bits_a: int, q, q_form
                                         _dev(beta_r, "beta_r", torch.float32), float(eps), bits_a,
                                         _dev(q, "q", want), q_format, prs, _stream(stream)),
            "ot_layernorm_quantize")
+
+
+def ot_linear_fused(x, z, r, bits_a: int, qw, sw, b_fold, bits_w: int, q, y, relu: bool = False, workspace=None,
+                    stream=None):
+    """Quantize x into q (fp16 codes [M, K]) and run the linear into y [M, N] in one call."""
+    M, K, ldx = _rows(x, "x")
+    _dense(q, "q")
+    _dense(qw, "qw")
+    N = qw.shape[0]
+    if tuple(q.shape) != (M, K):
+        raise ValueError("q must be [M, K]")
+    ym, yn, ldy = _rows(y, "y")
+    if ym != M or yn != N:
+        raise ValueError("y must be [M, N]")
+    wp, wb = _ws_args(workspace, x.device, stream)
+    _check(load().ot_linear_fused(_dev(x, "x", torch.float16), M, K, ldx, _dev(z, "z", torch.float32),
+                                  _dev(r, "r", torch.float32), bits_a, _dev(qw, "qw", torch.int8),
+                                  _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32), N, bits_w,
+                                  _dev(q, "q", torch.float16), _dev(y, "y", torch.float16), ldy, 1 if relu else 0,
+                                  wp, wb, _stream(stream)), "ot_linear_fused")
 
 
 def ot_linear_quantize_next(q, qw, sw, b_fold, bits_a: int, bits_w: int, z_next, r_next, bits_next: int, q_next,

@@ -232,6 +232,28 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
+ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
+                          int bits_a, const int8_t *qw, const float *sw, const float *b_fold, int64_t N, int bits_w,
+                          void *q_f16, void *y_f16, int64_t ldy, int relu, void *workspace, size_t workspace_bytes,
+                          void *stream) {
+    if (ldx < K || ldx % 8 != 0) return OT_ERR_INVALID_ARG;
+    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
+    if (v != OT_OK) return v;
+    if (!z || !r || !aligned(z, 16) || !aligned(r, 16)) return OT_ERR_INVALID_ARG;
+    if (M > 0 && (!x_f16 || !aligned(x_f16, 16))) return OT_ERR_INVALID_ARG;
+    if (!sw || !b_fold || ldy < N || (y_f16 && !aligned(y_f16, 2))) return OT_ERR_INVALID_ARG;
+    if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
+    if (ldy > kIntMax || (M + 63) / 64 > 65535) return OT_ERR_UNSUPPORTED;
+    if (M == 0) return OT_OK;
+    const cudaStream_t st = as_stream(stream);
+    cudaError_t e = ot::launch_quantize(x_f16, M, K, ldx, z, r, bits_a, q_f16, OT_CODE_F16, st);
+    if (e != cudaSuccess) return from_cuda(e);
+    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+                     workspace, workspace ? workspace_bytes : 0};
+    a.pdl = true;
+    return from_cuda(ot::launch_linear(a, st));
+}
+
 ot_status ot_linear_quantize_next(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw,
                                   const float *b_fold, int64_t N, int bits_a, int bits_w, int relu,
                                   const float *z_next, const float *r_next, int bits_next, void *q_next_f16,

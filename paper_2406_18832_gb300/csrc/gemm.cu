@@ -141,6 +141,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == kWarpTma) {
         if (lane == 0) {
+            // weights of the first tile into L2 while a programmatic predecessor
+            // may still be writing the codes; then wait for it
+            if (blockIdx.x < num_tiles)
+                for (int kb = 0; kb < nkb && kb < kStages; ++kb)
+                    tma_prefetch_l2_2d(&tm_w, kb * kBK, (blockIdx.x / m_tiles) * kBM);
+            grid_dep_wait();
             uint32_t it = 0;
             for (int t = blockIdx.x; t < num_tiles && !*abort; t += gridDim.x) {
                 const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
@@ -354,6 +360,7 @@ struct alignas(1024) SmemPair {
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
+    unsigned long long epoch;  // stream-K: this launch's flag value
 };
 
 // Work of one CTA pair: a list of pieces (pair tile u, k-blocks [kb0, kb1)).
@@ -419,8 +426,20 @@ struct PairSched {
 // Stream-K workspace: per pair and CTA rank, 256 token columns x 128 weight
 // rows of int32 partial sums (column-major, so a warp's stores are
 // contiguous), then one 64-bit flag per pair and rank holding the launch
-// epoch once its partials are complete.
+// epoch once its partials are complete, then the epoch counter and a count of
+// the CTAs done with the launch.  Each launch takes epoch = counter + 1; the
+// last CTA to finish stores it back (a launch starts only after the previous
+// one on the stream ended, so all CTAs of a launch read one value), so the
+// epochs grow from launch to launch on the device -- also when the launch is
+// replayed from a CUDA graph -- and a flag left by an earlier launch never
+// matches.  A zero-filled workspace starts the count.
 __host__ __device__ constexpr size_t pair_slot_ints() { return (size_t)256 * 128; }
+
+// {epoch of the last launch, CTAs done with this one}, after the flags
+__device__ __forceinline__ unsigned long long *pair_ctl(int32_t *ws, int nclusters) {
+    return reinterpret_cast<unsigned long long *>(ws + (size_t)nclusters * 2 * pair_slot_ints()) +
+           (size_t)nclusters * 2;
+}
 
 __device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) {
     uint64_t v;
@@ -432,7 +451,7 @@ template <bool kS32, bool kAsym, bool kQOut>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
-                       int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws, uint64_t epoch,
+                       int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws,
                        const float *__restrict__ s_tok, const int32_t *__restrict__ zc,
                        const int32_t *__restrict__ rowsum, const float *__restrict__ zq,
                        const float *__restrict__ rq, int qmax_out) {
@@ -465,6 +484,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         mbar_init(smem_u32(&S.pub), kNumEpiWarps);
         mbar_init(smem_u32(&S.drain), 1);
         S.abort = 0;
+        S.epoch = ws ? __ldcg(pair_ctl(ws, nclusters)) + 1 : 0;
         fence_barrier_init();
     }
     if (warp == kWarpTma && lane == 0) {
@@ -484,6 +504,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (warp < 4) {
         regs_dec<56>();
         if (warp == kWarpTma && lane == 0) {
+            // weights of the first piece into L2 while a programmatic
+            // predecessor may still be writing the codes; then wait for it
+            if (sch.count > 0) {
+                int u, pk0, pk1;
+                sch.piece(0, u, pk0, pk1);
+                for (int kb = pk0; kb < pk1 && kb < pk0 + kRing; ++kb)
+                    tma_prefetch_l2_2d(&tm_w, kb * kBK, ((u / m_tiles) * 2 + (int)rank) * kBM);
+            }
+            grid_dep_wait();
             uint32_t it = 0;
             for (int p = 0; p < sch.count && !*abort; ++p) {
                 int u, pk0, pk1;
@@ -628,7 +657,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 // a pair has at most one partial piece per launch: phase 0 of pub
                 if (warp == kWarpEpi0 && lane == 0 && mbar_wait(smem_u32(&S.pub), 0, abort, &g_status)) {
                     __threadfence();
-                    atomicExch(flags + (size_t)cluster * 2 + rank, (unsigned long long)epoch);
+                    atomicExch(flags + (size_t)cluster * 2 + rank, S.epoch);
                 }
                 continue;
             }
@@ -638,7 +667,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 for (int c = c_lo; c < cluster && ok; ++c) {
                     const unsigned long long *f = flags + (size_t)c * 2 + rank;
                     const uint64_t t0 = globaltimer_ns();
-                    while (ld_acquire_u64(f) != epoch) {
+                    while (ld_acquire_u64(f) != S.epoch) {
                         if (*abort) { ok = false; break; }
                         if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
                             atomicExch(&g_status, (int)OT_ERR_TIMEOUT);
@@ -703,22 +732,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tc_fence_after();
         tmem_dealloc_pair(tmem, kTmemCols);
     }
+    if (ws && threadIdx.x == 0) {
+        unsigned long long *ctl = pair_ctl(ws, nclusters);
+        if (atomicAdd(ctl + 1, 1ull) == (unsigned long long)gridDim.x - 1) {
+            // the last CTA of the launch: hand the epoch to the next launch
+            ctl[1] = 0;
+            ctl[0] = S.epoch;
+        }
+    }
 }
 
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-// Launch epochs of the stream-K flags: strictly increasing across launches,
-// so a flag left by an earlier launch never matches (workspaces start zeroed).
-uint64_t next_epoch() {
-    static std::atomic<uint64_t> counter{0};
-    return ++counter;
-}
-
 constexpr int64_t kStreamKMinSaving = 32;  // k-blocks per pair
 
 size_t pair_workspace_bytes(int clusters) {
-    return (size_t)clusters * 2 * pair_slot_ints() * sizeof(int32_t) + (size_t)clusters * 2 * sizeof(uint64_t);
+    return (size_t)clusters * 2 * pair_slot_ints() * sizeof(int32_t) + (size_t)clusters * 2 * sizeof(uint64_t) +
+           2 * sizeof(uint64_t);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -767,10 +798,9 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     if (attr_err != cudaSuccess) return attr_err;
     const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
-    linear_kernel<BN, kS32, kAsym, kQOut><<<grid, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N,
-                                                         (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
-                                                         a.rowsum, a.zq, a.rq, a.qmax_out);
-    return cudaGetLastError();
+    return launch_kernel(linear_kernel<BN, kS32, kAsym, kQOut>, dim3(grid), dim3(kThreads), smem, st, a.pdl, tm_q, tm_w,
+                         a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
+                         a.rowsum, a.zq, a.rq, a.qmax_out);
 }
 
 // Clusters of the pair kernel that fit on the device at once (one per two SMs).
@@ -835,12 +865,9 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
                          whole - shared >= kStreamKMinSaving && units * nkb < ((int64_t)1 << 30);
     const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
-    const uint64_t epoch = streamk ? next_epoch() : 0;
-    linear_pair_kernel<kS32, kAsym, kQOut><<<2 * clusters, kThreads, smem, st>>>(tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M,
-                                                                (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
-                                                                epoch, a.s_tok, a.zc, a.rowsum, a.zq, a.rq,
-                                                                a.qmax_out);
-    return cudaGetLastError();
+    return launch_kernel(linear_pair_kernel<kS32, kAsym, kQOut>, dim3(2 * clusters), dim3(kThreads), smem, st, a.pdl,
+                         tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
+                         a.s_tok, a.zc, a.rowsum, a.zq, a.rq, a.qmax_out);
 }
 
 // M <= 32 goes to the decode kernel (gemv.cu) before this dispatch.
@@ -853,7 +880,6 @@ cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
 
 }  // namespace
 
-uint64_t next_launch_epoch() { return next_epoch(); }
 
 bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz) {
@@ -901,8 +927,8 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratch
 // Device address of g_noalloc_scratch on the current device.  In host code
 // the array's name is only a stand-in, so the address comes from
 // cudaGetSymbolAddress, once per device, with that device current; the first
-// use on a device also zero-fills the array on `st` (the stream-K flags must
-// start below every launch epoch; later launches leave them below the next).
+// use on a device also zero-fills the array on `st` (the stream-K flags and
+// epoch counters start at zero; the kernels keep them consistent after that).
 cudaError_t noalloc_scratch(void **ptr, cudaStream_t st) {
     static std::mutex mu;
     static void *addr[64] = {nullptr};

@@ -38,9 +38,11 @@
 //     on it first (at the start of theirs), store their int32 partials in a
 //     workspace slot of their own and publish it with a launch-epoch flag
 //     (release).  The finisher adds the slots (acquire; normally published
-//     long before) and applies the epilogue.  The epochs grow from launch to
-//     launch, so a flag left by an earlier launch never matches and nothing
-//     has to be cleared.
+//     long before) and applies the epilogue.  The epoch is a counter in the
+//     workspace: every launch takes counter + 1 and its last CTA stores that
+//     back, so epochs grow from launch to launch (graph replays included), a
+//     flag left by an earlier launch never matches and nothing has to be
+//     cleared.
 // Without a workspace the ranges are whole tiles (no split, less even).
 #include <cuda_fp16.h>
 
@@ -64,6 +66,7 @@ constexpr int kGvWBytes = 2 * kGvWBox;            // weights of a stage (two box
 constexpr int kGvMaxStages = 8;
 constexpr int kGvSmemBudget = 224 * 1024;
 constexpr int kGvHeader = 256;                    // barriers, counters, flags
+constexpr int kGvPdlUnits = 2;                    // units whose weights load before a programmatic wait
 constexpr int kGvSlotInts = kGvRows * 32;         // workspace ints per split tile (32 tokens x 128 rows)
 
 struct GvParams {
@@ -74,7 +77,8 @@ struct GvParams {
     void *out;
     int32_t *part;                 // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
     unsigned long long *flags;     // [grid] launch epoch once a CTA's slot is complete
-    uint64_t epoch;
+    unsigned long long *ctl;       // {epoch of the last launch, CTAs done with this one}
+    int pdl;                       // launched as a programmatic dependent of the codes' producer
     int *status;        // device status word
     int M, N, K, ldy, kcb, relu;
     int nks;            // units per tile
@@ -157,6 +161,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     unsigned *done = reinterpret_cast<unsigned *>(full + kGvMaxStages);  // warps finished with a slot, ever
     unsigned *loads = done + kGvMaxStages;                                // units loaded into a slot, ever
     volatile int *abort = reinterpret_cast<volatile int *>(loads + kGvMaxStages);
+    unsigned long long *epoch_s = reinterpret_cast<unsigned long long *>(base + 192);  // this launch's epoch
     int32_t(*red)[kGvRows + 1] = reinterpret_cast<int32_t(*)[kGvRows + 1]>(base + kGvHeader);  // [TN*8]
     uint8_t *ring = base + ((kGvHeader + p.red_bytes + 1023) & ~1023);
 
@@ -169,15 +174,23 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     const uint32_t abytes = (uint32_t)M * kGvKS * 2;  // activation box
     uint64_t pol_w = 0, pol_a = 0;
 
-    // Load unit (tile, ks) into `slot`, completing on full[slot].
-    auto load_unit = [&](int slot, int64_t tile, int ks) {
+    // Load unit (tile, ks) into `slot`, completing on full[slot]: the weight
+    // boxes, then (load_codes) the codes box.
+    auto load_weights = [&](int slot, int64_t tile, int ks) {
         const uint32_t bar = smem_u32(&full[slot]);
         mbar_arrive_expect_tx(bar, kGvWBytes + abytes);
         const uint32_t st = smem_u32(ring + (size_t)slot * p.stage_bytes);
         tma_load_2d_hint(st, &tm_w, bar, ks * kGvKS, (int32_t)(tile * kGvRows), pol_w);
         tma_load_2d_hint(st + kGvWBox, &tm_w, bar, ks * kGvKS + 128, (int32_t)(tile * kGvRows), pol_w);
-        tma_load_2d_hint(st + kGvWBytes, &tm_a, bar, ks * kGvKS, 0, pol_a);
         loads[slot] += 1;
+    };
+    auto load_codes = [&](int slot, int ks) {
+        const uint32_t st = smem_u32(ring + (size_t)slot * p.stage_bytes);
+        tma_load_2d_hint(st + kGvWBytes, &tm_a, smem_u32(&full[slot]), ks * kGvKS, 0, pol_a);
+    };
+    auto load_unit = [&](int slot, int64_t tile, int ks) {
+        load_weights(slot, tile, ks);
+        load_codes(slot, ks);
     };
 
     if (lane == 0) {
@@ -194,10 +207,28 @@ __global__ void __launch_bounds__(kGvThreads, 1)
             loads[s] = 0;
         }
         *abort = 0;
+        *epoch_s = p.whole ? 0 : __ldcg(p.ctl) + 1;
         fence_barrier_init();
+        // launched as a programmatic dependent of the kernel writing the
+        // codes: the first units' weights go out before waiting for it, their
+        // codes after it.  Otherwise the loads go out unit by unit, so that the
+        // first unit completes first.
+        const int pre = p.pdl ? (S < kGvPdlUnits ? S : kGvPdlUnits) : 0;
         int64_t tile = tile0;
         int ks = ks0;
-        for (int s = 0; s < S && u_begin + s < u_end; ++s) {
+        for (int s = 0; s < pre && u_begin + s < u_end; ++s) {
+            load_weights(s, tile, ks);
+            if (++ks == nks) {
+                ks = 0;
+                ++tile;
+            }
+        }
+        grid_dep_wait();
+        for (int s = 0, k2 = ks0; s < pre && u_begin + s < u_end; ++s) {
+            load_codes(s, k2);
+            if (++k2 == nks) k2 = 0;
+        }
+        for (int s = pre; s < S && u_begin + s < u_end; ++s) {
             load_unit(s, tile, ks);
             if (++ks == nks) {
                 ks = 0;
@@ -349,7 +380,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
             __syncthreads();
             if (threadIdx.x == 0) {
                 __threadfence();
-                atomicExch(p.flags + blockIdx.x, (unsigned long long)p.epoch);
+                atomicExch(p.flags + blockIdx.x, *epoch_s);
             }
         } else {
             // the first part: add the later parts (CTAs blockIdx.x + 1 .. last) and finish the tile
@@ -358,7 +389,8 @@ __global__ void __launch_bounds__(kGvThreads, 1)
             if (threadIdx.x < nc) {
                 const unsigned long long *f = p.flags + blockIdx.x + 1 + threadIdx.x;
                 const uint64_t t0 = globaltimer_ns();
-                while (ld_acquire_flag(f) != p.epoch) {
+                const unsigned long long epoch = *epoch_s;
+                while (ld_acquire_flag(f) != epoch) {
                     if (*abort) break;
                     if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
                         atomicExch(p.status, (int)OT_ERR_TIMEOUT);
@@ -382,13 +414,20 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     }
     // teardown (only matters after a timeout): every copy issued must land
     // before the CTA's shared memory goes away
-    if (threadIdx.x == 0)
+    if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s)
             if (loads[s] > 0) wait_teardown_status(smem_u32(&full[s]), (loads[s] - 1) & 1, p.status);
+        if (!p.whole && atomicAdd(p.ctl + 1, 1ull) == (unsigned long long)gridDim.x - 1) {
+            // the last CTA of the launch: hand the epoch to the next launch
+            p.ctl[1] = 0;
+            p.ctl[0] = *epoch_s;
+        }
+    }
 }
 
 template <int TN, bool kS32>
-cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvParams &base, cudaStream_t st) {
+cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvParams &base, cudaStream_t st,
+                     bool pdl) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
@@ -405,15 +444,14 @@ cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvP
     if (p.stages > kGvMaxStages) p.stages = kGvMaxStages;
     if (p.stages < 2) return cudaErrorInvalidConfiguration;
     const size_t smem = 1024 + ring_off + (size_t)p.stages * p.stage_bytes;
-    linear_gemv_kernel<TN, kS32><<<p.grid, kGvThreads, smem, st>>>(tm_w, tm_a, p);
-    return cudaGetLastError();
+    return launch_kernel(linear_gemv_kernel<TN, kS32>, dim3(p.grid), dim3(kGvThreads), smem, st, pdl, tm_w, tm_a, p);
 }
 
 }  // namespace
 
 size_t gemv_workspace_bytes() {
     const size_t g = (size_t)num_sms();
-    return g * kGvSlotInts * sizeof(int32_t) + g * sizeof(unsigned long long);
+    return g * kGvSlotInts * sizeof(int32_t) + g * sizeof(unsigned long long) + 2 * sizeof(unsigned long long);
 }
 
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
@@ -434,6 +472,7 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     p.zq = a.zq;
     p.rq = a.rq;
     p.qmax_out = a.qmax_out;
+    p.pdl = a.pdl ? 1 : 0;
     p.out = a.out;
     p.status = device_status_word();
     if (!p.status) return cudaErrorUnknown;
@@ -464,14 +503,15 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
         p.grid = (int)(p.units < sms ? p.units : sms);
         p.part = reinterpret_cast<int32_t *>(a.workspace);
         p.flags = reinterpret_cast<unsigned long long *>(p.part + (size_t)sms * kGvSlotInts);
-        p.epoch = next_launch_epoch();
+        p.ctl = p.flags + sms;
     } else {
         p.whole = 1;
         p.grid = (int)(p.ntiles < sms ? p.ntiles : sms);
     }
-    if (a.M <= 8) return a.out_s32 ? run_gemv<1, true>(tm_w, tm_a, p, st) : run_gemv<1, false>(tm_w, tm_a, p, st);
-    if (a.M <= 16) return a.out_s32 ? run_gemv<2, true>(tm_w, tm_a, p, st) : run_gemv<2, false>(tm_w, tm_a, p, st);
-    return a.out_s32 ? run_gemv<4, true>(tm_w, tm_a, p, st) : run_gemv<4, false>(tm_w, tm_a, p, st);
+    const bool d = a.pdl;
+    if (a.M <= 8) return a.out_s32 ? run_gemv<1, true>(tm_w, tm_a, p, st, d) : run_gemv<1, false>(tm_w, tm_a, p, st, d);
+    if (a.M <= 16) return a.out_s32 ? run_gemv<2, true>(tm_w, tm_a, p, st, d) : run_gemv<2, false>(tm_w, tm_a, p, st, d);
+    return a.out_s32 ? run_gemv<4, true>(tm_w, tm_a, p, st, d) : run_gemv<4, false>(tm_w, tm_a, p, st, d);
 }
 
 }  // namespace ot

@@ -53,6 +53,8 @@ struct LinearArgs {
     const int32_t *rowsum;    // with zc: sum_k q[m,k] [M]
     const float *zq, *rq;     // chained epilogue: the next layer's z', r' [N] (out then holds fp16 codes), or null
     int qmax_out;             // with zq: the next layer's qmax
+    bool pdl;                 // launched as a programmatic dependent of the kernel that wrote q (weights are
+                              // read before that kernel ends, codes only after)
 };
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();
@@ -65,8 +67,6 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st);
 // bytes of the decode region (split-tile partial sums and counters)
 size_t gemv_workspace_bytes();
-// strictly increasing per call (stream-K flags of both linear kernels)
-uint64_t next_launch_epoch();
 // device address of the status word that bounded waits write on timeout
 int *device_status_word();
 // 2-D tiled tensor map of a row-major [rows, inner] array (false if the

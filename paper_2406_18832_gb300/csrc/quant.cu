@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict_
                                                        int64_t ldx, const float *__restrict__ z,
                                                        const float *__restrict__ r, int qmax, void *q,
                                                        int32_t *rowsum) {
+    grid_dep_launch();  // a linear launched as a programmatic dependent may start its weight loads now
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int64_t c0 = (int64_t)blockIdx.x * 256 + tx * 8;
     const bool active = c0 < K;  // K % 8 == 0: a lane's 8 channels are whole or absent

@@ -61,3 +61,36 @@ def test_workspace_size_is_stable():
     from paper_2406_18832_gb300 import binding as B
     n = B.ot_linear_workspace_size()
     assert n > 0 and n == B.ot_linear_workspace_size()
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 5120, 20480), (16, 2048, 4096), (2048, 4096, 16384), (256, 512, 4096)])
+def test_streamk_under_cuda_graph_replay(M, N, K):
+    """A captured call replayed many times: each replay must take a new launch
+    epoch on the device (one fixed at capture would let a finisher read the
+    previous replay's partial sums).  Inputs change between replays; every
+    replay is checked against whole-tile scheduling of the same inputs."""
+    from paper_2406_18832_gb300 import binding as B
+    dev = "cuda"
+    qw = _codes((N, K), 127, K + 1).to(torch.int8).to(dev)
+    q = torch.empty(M, K, dtype=torch.float16, device=dev)
+    acc = torch.empty(M, N, dtype=torch.int32, device=dev)
+    want = torch.empty(M, N, dtype=torch.int32, device=dev)
+    ws = torch.zeros(B.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+    s = torch.cuda.Stream()
+    q.copy_(_codes((M, K), 127, 1).half().to(dev))
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        B.ot_linear_s32(q, qw, 8, 8, acc, workspace=ws, stream=s)
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        B.ot_linear_s32(q, qw, 8, 8, acc, workspace=ws, stream=s)
+    for seed in range(2, 8):
+        q.copy_(_codes((M, K), 127, seed).half().to(dev))
+        acc.fill_(-7)
+        g.replay()
+        B.ot_linear_s32(q, qw, 8, 8, want, workspace=False)
+        torch.cuda.synchronize()
+        assert B.ot_get_device_status() == B.OT_OK
+        assert torch.equal(acc, want), seed
