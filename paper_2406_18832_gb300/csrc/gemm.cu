@@ -139,50 +139,57 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
 
+    // the TMA and MMA roles run their loops with the whole warp and issue from one elected lane
     if (warp == kWarpTma) {
-        if (lane == 0) {
-            // weights of the first tile into L2 while a programmatic predecessor
-            // may still be writing the codes; then wait for it
-            if (blockIdx.x < num_tiles)
-                for (int kb = 0; kb < nkb && kb < kStages; ++kb)
-                    tma_prefetch_l2_2d(&tm_w, kb * kBK, (blockIdx.x / m_tiles) * kBM);
-            grid_dep_wait();
-            uint32_t it = 0;
-            for (int t = blockIdx.x; t < num_tiles && !*abort; t += gridDim.x) {
-                const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
-                    const int s = it % kStages;
-                    const uint32_t ph = (it / kStages) & 1;
-                    if (!mbar_wait(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status)) break;
+        // weights of the first tile into L2 while a programmatic predecessor
+        // may still be writing the codes; then wait for it
+        if (blockIdx.x < num_tiles && elect_one())
+            for (int kb = 0; kb < nkb && kb < kStages; ++kb)
+                tma_prefetch_l2_2d(&tm_w, kb * kBK, (blockIdx.x / m_tiles) * kBM);
+        __syncwarp();
+        grid_dep_wait();
+        uint32_t it = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+            const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
+            for (int kb = 0; kb < nkb; ++kb, ++it) {
+                const int s = it % kStages;
+                const uint32_t ph = (it / kStages) & 1;
+                if (!(ok = mbar_wait_warp(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status))) break;
+                if (elect_one()) {
                     mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
                     tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
                     tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
                 }
+                __syncwarp();
             }
-            // teardown: every load issued must have landed before the CTA exits
+        }
+        // teardown: every load issued must have landed before the CTA exits
+        if (lane == 0) {
             const uint32_t issued = it;
             for (uint32_t j = issued > (uint32_t)kStages ? issued - kStages : 0; j < issued; ++j)
                 wait_teardown(smem_u32(&S.full[j % kStages]), (j / kStages) & 1);
         }
+        __syncwarp();
     } else if (warp == kWarpMma) {
-        if (lane == 0) {
-            const uint32_t idesc = idesc_f16_f32(kBM, BN);
-            uint32_t it = 0, g = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
-                for (int kb0 = 0; kb0 < nkb && ok; kb0 += kcb, ++g) {
-                    const int buf = g & 1;
-                    if (!(ok = mbar_wait(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
+        const uint32_t idesc = idesc_f16_f32(kBM, BN);
+        uint32_t it = 0, g = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+            for (int kb0 = 0; kb0 < nkb && ok; kb0 += kcb, ++g) {
+                const int buf = g & 1;
+                if (!(ok = mbar_wait_warp(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
+                tc_fence_after();
+                const uint32_t d = tmem + kTmemAccCol + buf * BN;
+                const int kb1 = min(nkb, kb0 + kcb);
+                for (int kb = kb0; kb < kb1; ++kb, ++it) {
+                    const int s = it % kStages;
+                    const uint32_t ph = (it / kStages) & 1;
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
                     tc_fence_after();
-                    const uint32_t d = tmem + kTmemAccCol + buf * BN;
-                    const int kb1 = min(nkb, kb0 + kcb);
-                    for (int kb = kb0; kb < kb1; ++kb, ++it) {
-                        const int s = it % kStages;
-                        const uint32_t ph = (it / kStages) & 1;
-                        if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
-                        if (!(ok = mbar_wait(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
-                        tc_fence_after();
-                        const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
+                    const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
+                    if (elect_one()) {
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk)
                             mma_f16_ts(d, tmem + s * 32 + kk * 8, bdesc + (uint64_t)((kk * 32) >> 4), idesc,
@@ -190,13 +197,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mma_commit(smem_u32(&S.empty[s]));
                         mma_commit(smem_u32(&S.aempty[s]));
                     }
-                    if (ok) mma_commit(smem_u32(&S.accfull[buf]));
+                    __syncwarp();
                 }
+                if (ok && elect_one()) mma_commit(smem_u32(&S.accfull[buf]));
+                __syncwarp();
             }
-            // teardown: all issued MMAs complete before TMEM is freed
+        }
+        // teardown: all issued MMAs complete before TMEM is freed
+        if (elect_one()) {
             mma_commit(smem_u32(&S.drain));
             wait_teardown(smem_u32(&S.drain), 0);
         }
+        __syncwarp();
     } else if (warp >= kWarpConv0 && warp < kWarpConv0 + 4) {
         const int q = warp & 3;
         const int row = q * 32 + lane;           // weight row of the tile = TMEM lane
@@ -319,49 +331,77 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ---------------------------------------------------------------------------
 // Wide-tile CTA-pair variant for prefill-sized token counts (M > 128).
 //
-// Measured on GB300: a 128 x N x 16 kind::f16 MMA costs about as much for
-// N = 64 or 128 as for N = 256, so only N = 256 instructions reach the tensor
-// peak; and TMA ingest per SM is latency-bound (about 1.6 us per load under
-// load), so the fewer bytes an SM must receive per MMA the better.
+// Measured on GB300: a cta_group::2 kind::f16 MMA of 256 x N x 16 runs at
+// the full tensor rate (4096 MACs per clock per SM, dependent accumulation,
+// one commit per 4 MMAs) for every N from 128 to 256, with A in shared
+// memory or in TMEM.  TMA copies from L2 cost about 270 ns per copy per SM
+// when all SMs stream, whatever their size from 8 to 48 KB (8 KB copies:
+// 4.6 TB/s over the GPU; 48 KB copies: 22 TB/s), so the copies must be large:
+// one copy per operand brings four 64-wide k-blocks (a 3-D view of the
+// row-major array whose outer dimension steps along K).
 // So the two CTAs of a cluster run one cta_group::2 MMA of 256 weight rows x
-// 256 tokens: each CTA loads its own 128 int8 weight rows (8 KB per 64-wide
-// k-block) and half of the token tile (128 rows of fp16 codes, 16 KB); B is
-// split along N between the pair and each CTA's TMEM receives its 128 rows x
-// 256 tokens of the accumulator.
-// The converters widen each CTA's int8 weight rows into an fp16 A tile in
-// shared memory (128-byte swizzle), so all 512 TMEM columns can hold two
-// 256-column chunk accumulators: while the MMA fills one, the epilogue
-// converts the other (fp32 -> int32 conversions run at a quarter rate and
-// would otherwise stall the tensor core at every chunk boundary).
+// 192 tokens: per group of four k-blocks each CTA loads its own 128 int8
+// weight rows (32 KB, one copy) and half of the token tile (96 rows of fp16
+// codes, 48 KB, one copy); B is split along N between the pair and each
+// CTA's TMEM receives its 128 rows x 192 tokens of the accumulator.
+// The converters widen each CTA's int8 weight rows to fp16 and store them in
+// TMEM as the MMA's A operand (tcgen05.st), so shared memory carries only
+// the TMA ingest, the converters' read of the int8 rows and the tensor
+// core's read of B.  TMEM (512 columns) holds two 192-column chunk
+// accumulators -- while the MMA fills one, the epilogue converts the other
+// (fp32 -> int32 conversions run at a quarter rate and would otherwise stall
+// the tensor core at every chunk boundary) -- and four 32-column A stages.
+// 192-token tiles cover 2048 tokens with 3 % padding.
 //   Rank 0 of the pair issues the MMAs.  The converters and epilogue warps
 //   of both CTAs signal rank 0's barriers; rank 0's commits arrive on the
-//   barriers of both CTAs (multicast).  One commit per k-block (done[s])
-//   frees both the TMA slot and, kAStages k-blocks later, the A tile: each
-//   extra tcgen05.commit per k-block costs about 10% of tensor throughput.
+//   barriers of both CTAs (multicast): one per k-block frees its A stage,
+//   one per group frees the group's B stage.  A converter waits for its own
+//   CTA's B stage as well as its weights, so rank 0's wait on the converters
+//   of both CTAs covers both halves of B.
 //   Warpgroups: 0 = TMA producer / MMA issuer / TMEM allocator (56 regs),
-//   1 = converters (88 regs), 2-3 = epilogue (184 regs: 128 int32 totals).
+//   1 = converters (88 regs), 2-3 = epilogue (184 regs: 96 int32 totals).
+//   Needs K % 128 == 0 (the 3-D views must not reach past a row's end);
+//   other K use linear_kernel.
 // ---------------------------------------------------------------------------
-constexpr int kPairBN = 256;   // tokens per pair tile (MMA N)
-constexpr int kRing = 6;       // TMA stages: token half-tile + weight rows
-constexpr int kAStages = 3;    // fp16 A tiles written by the converters
-static_assert(kRing % kAStages == 0, "A tile of k-block i is freed by the commit of k-block i - kAStages");
+constexpr int kPairBN = 192;                      // tokens per pair tile (MMA N)
+constexpr int kPairHalf = kPairBN / 2;            // token rows per CTA (B is split along N)
+constexpr int kPairACol = 2 * kPairBN;            // TMEM: accumulators in [0, 2 kPairBN), then A stages
+constexpr int kAStages = (512 - kPairACol) / 32;  // 32-column fp16 A stages (128 rows x 64 k)
+constexpr int kGroupKB = 4;                       // k-blocks per TMA copy
+constexpr int kWStages = 2;                       // weight stages: 2 x 128 rows x 128 int8, 128-byte swizzle (32 KB)
+constexpr int kBStages = 3;                       // token stages: 4 x 96 rows x 64 fp16, 128-byte swizzle (48 KB)
+constexpr uint32_t kWStageBytes = 2 * kBM * 128;
+constexpr uint32_t kBTileBytes = kPairHalf * 128;
+constexpr uint32_t kBStageBytes = kGroupKB * kBTileBytes;
+static_assert(kAStages >= 2, "A stage of k-block i is freed by the commit of k-block i - kAStages");
+static_assert(kPairBN % 32 == 0 && kPairHalf % 32 == 0, "the epilogue drains 32 columns at a time");
+static_assert(kBTileBytes % 1024 == 0, "each k-block of B is a whole number of 1024-byte swizzle atoms");
 
 struct alignas(1024) SmemPair {
-    uint8_t b[kRing][kBM * 128];      // this CTA's 128 token rows of fp16 codes, 128-byte swizzle (16 KB)
-    uint8_t a[kAStages][kBM * 128];   // this CTA's 128 weight rows widened to fp16, 128-byte swizzle (16 KB)
-    uint8_t w[kRing][kBM * kBK];      // this CTA's 128 weight rows of int8 codes, 64-byte swizzle (8 KB)
-    uint64_t full[kRing];             // own TMA landed
-    uint64_t done[kRing];             // pair MMA of the k-block done (rank 0 commit, both CTAs)
-    uint64_t wread[kRing];            // own 4 converter warps read w[]
-    uint64_t afull[kAStages];         // rank 0 only: both CTAs' converters wrote their A tiles (8 warps)
-    uint64_t accfull[2];              // pair MMA finished the chunk (rank 0 commit)
-    uint64_t accempty[2];             // rank 0 only: both CTAs' epilogues drained the chunk (16 warps)
-    uint64_t pub;                     // stream-K: the 8 epilogue warps stored their partial sums
+    uint8_t b[kBStages][kBStageBytes];  // this CTA's 96 token rows of fp16 codes, [k-block][row][64 fp16]
+    uint8_t w[kWStages][kWStageBytes];  // this CTA's 128 weight rows of int8 codes, [k-block pair][row][128 int8]
+    uint64_t wfull[kWStages];           // own weight copy landed
+    uint64_t wempty[kWStages];          // own 4 converter warps read the group's weights
+    uint64_t bfull[kBStages];           // own token copy landed
+    uint64_t bdone[kBStages];           // pair MMA of the group done (rank 0 commit, both CTAs)
+    uint64_t afull[kAStages];           // rank 0 only: both CTAs' converters wrote their A stages (8 warps)
+    uint64_t adone[kAStages];           // pair MMA of the k-block done (rank 0 commit, both CTAs)
+    uint64_t accfull[2];                // pair MMA finished the chunk (rank 0 commit)
+    uint64_t accempty[2];               // rank 0 only: both CTAs' epilogues drained the chunk (16 warps)
+    uint64_t pub;                       // stream-K: the 8 epilogue warps stored their partial sums
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
     unsigned long long epoch;  // stream-K: this launch's flag value
 };
+
+// Groups: a piece's k-blocks [kb0, kb1) are cut at multiples of kGroupKB;
+// each group takes one token copy starting at its first k-block and one
+// weight copy starting at the even k-block at or below it.
+__device__ __forceinline__ bool group_start(int kb, int kb0) { return kb == kb0 || (kb & (kGroupKB - 1)) == 0; }
+__device__ __forceinline__ bool group_end(int kb, int kb1) {
+    return kb == kb1 - 1 || (kb & (kGroupKB - 1)) == kGroupKB - 1;
+}
 
 // Work of one CTA pair: a list of pieces (pair tile u, k-blocks [kb0, kb1)).
 // Without a workspace the pieces are whole tiles dealt round-robin.  With a
@@ -465,18 +505,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int num_units = m_tiles * n_pairs;
     const int nkb = (K + kBK - 1) / kBK;
     volatile int *abort = &S.abort;
-    constexpr uint32_t kTxBytes = kBM * 128 + kBM * kBK;
     constexpr uint16_t kBoth = 0x3;
     PairSched sch;
     sch.init(num_units, nkb, nclusters, cluster, ws != nullptr);
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kRing; ++s) {
-            mbar_init(smem_u32(&S.full[s]), 1);
-            mbar_init(smem_u32(&S.done[s]), 1);
-            mbar_init(smem_u32(&S.wread[s]), 4);
+        for (int s = 0; s < kWStages; ++s) {
+            mbar_init(smem_u32(&S.wfull[s]), 1);
+            mbar_init(smem_u32(&S.wempty[s]), 4);
         }
-        for (int s = 0; s < kAStages; ++s) mbar_init(smem_u32(&S.afull[s]), 8);
+        for (int s = 0; s < kBStages; ++s) {
+            mbar_init(smem_u32(&S.bfull[s]), 1);
+            mbar_init(smem_u32(&S.bdone[s]), 1);
+        }
+        for (int s = 0; s < kAStages; ++s) {
+            mbar_init(smem_u32(&S.afull[s]), 8);
+            mbar_init(smem_u32(&S.adone[s]), 1);
+        }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&S.accfull[b]), 1);
             mbar_init(smem_u32(&S.accempty[b]), 2 * kNumEpiWarps);
@@ -503,106 +548,153 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
     if (warp < 4) {
         regs_dec<56>();
-        if (warp == kWarpTma && lane == 0) {
-            // weights of the first piece into L2 while a programmatic
-            // predecessor may still be writing the codes; then wait for it
-            if (sch.count > 0) {
+        if (warp == kWarpTma) {
+            // the first weights into L2 while a programmatic predecessor may
+            // still be writing the codes; then wait for it
+            if (sch.count > 0 && elect_one()) {
                 int u, pk0, pk1;
                 sch.piece(0, u, pk0, pk1);
-                for (int kb = pk0; kb < pk1 && kb < pk0 + kRing; ++kb)
-                    tma_prefetch_l2_2d(&tm_w, kb * kBK, ((u / m_tiles) * 2 + (int)rank) * kBM);
+                tma_prefetch_l2_3d(&tm_w, 0, ((u / m_tiles) * 2 + (int)rank) * kBM, pk0 >> 1);
             }
+            __syncwarp();
             grid_dep_wait();
-            uint32_t it = 0;
-            for (int p = 0; p < sch.count && !*abort; ++p) {
+            uint32_t gi = 0;
+            bool ok = true;
+            for (int p = 0; p < sch.count && ok; ++p) {
                 int u, pk0, pk1;
                 sch.piece(p, u, pk0, pk1);
-                const int m0 = (u % m_tiles) * kPairBN + (int)rank * kBM;
+                const int m0 = (u % m_tiles) * kPairBN + (int)rank * kPairHalf;
                 const int n0 = ((u / m_tiles) * 2 + (int)rank) * kBM;
-                for (int kb = pk0; kb < pk1; ++kb, ++it) {
-                    const int s = it % kRing;
-                    const uint32_t ph = (it / kRing) & 1;
-                    // slot s was last used by k-block it - kRing: the pair MMA and the converters are done with it
-                    if (!mbar_wait(smem_u32(&S.done[s]), ph ^ 1, abort, &g_status)) break;
-                    if (!mbar_wait(smem_u32(&S.wread[s]), ph ^ 1, abort, &g_status)) break;
-                    mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
-                    tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
-                    tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
+                for (int g0 = pk0; g0 < pk1; g0 = (g0 | (kGroupKB - 1)) + 1, ++gi) {
+                    const int ws = gi % kWStages, bs = gi % kBStages;
+                    // stages last used by group gi - stages: the converters / the pair MMA are done with them
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.wempty[ws]), ((gi / kWStages) & 1) ^ 1, abort, &g_status)))
+                        break;
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.bdone[bs]), ((gi / kBStages) & 1) ^ 1, abort, &g_status)))
+                        break;
+                    if (elect_one()) {
+                        mbar_arrive_expect_tx(smem_u32(&S.wfull[ws]), kWStageBytes);
+                        tma_load_3d(smem_u32(S.w[ws]), &tm_w, smem_u32(&S.wfull[ws]), 0, n0, g0 >> 1);
+                        mbar_arrive_expect_tx(smem_u32(&S.bfull[bs]), kBStageBytes);
+                        tma_load_3d(smem_u32(S.b[bs]), &tm_q, smem_u32(&S.bfull[bs]), 0, m0, g0);
+                    }
+                    __syncwarp();
                 }
             }
-            const uint32_t issued = it;
-            for (uint32_t j = issued > (uint32_t)kRing ? issued - kRing : 0; j < issued; ++j)
-                wait_teardown(smem_u32(&S.full[j % kRing]), (j / kRing) & 1);
-        } else if (warp == kWarpMma && lane == 0 && rank == 0) {
+            // teardown: every copy issued must have landed before the CTA exits
+            if (lane == 0) {
+                for (uint32_t j = gi > (uint32_t)kWStages ? gi - kWStages : 0; j < gi; ++j)
+                    wait_teardown(smem_u32(&S.wfull[j % kWStages]), (j / kWStages) & 1);
+                for (uint32_t j = gi > (uint32_t)kBStages ? gi - kBStages : 0; j < gi; ++j)
+                    wait_teardown(smem_u32(&S.bfull[j % kBStages]), (j / kBStages) & 1);
+            }
+            __syncwarp();
+        } else if (warp == kWarpMma && rank == 0) {
+            // the whole warp runs the loop and waits; one elected lane issues the MMAs and commits
             const uint32_t idesc = idesc_f16_f32(2 * kBM, kPairBN);
-            uint32_t it = 0, g = 0;
+            const uint32_t a_tm = tmem + kPairACol;
+            uint32_t it = 0, g = 0, gi = 0, b_base = 0;
+            int g0 = 0, bs = 0;
             bool ok = true;
             for (int p = 0; p < sch.count && ok; ++p) {
                 int u, pk0, pk1;
                 sch.piece(p, u, pk0, pk1);
                 for (int kb0 = pk0; kb0 < pk1 && ok; kb0 += kcb, ++g) {
                     const int buf = g & 1;
-                    if (!(ok = mbar_wait(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status)))
+                        break;
                     tc_fence_after();
                     const uint32_t d = tmem + buf * kPairBN;
                     const int kb1 = min(pk1, kb0 + kcb);
                     for (int kb = kb0; kb < kb1; ++kb, ++it) {
-                        const int s = it % kRing, sa = it % kAStages;
-                        if (!(ok = mbar_wait(smem_u32(&S.full[s]), (it / kRing) & 1, abort, &g_status))) break;
-                        if (!(ok = mbar_wait(smem_u32(&S.afull[sa]), (it / kAStages) & 1, abort, &g_status))) break;
+                        if (group_start(kb, pk0)) {
+                            bs = gi % kBStages;
+                            g0 = kb;
+                            b_base = smem_u32(S.b[bs]);
+                            ++gi;
+                        }
+                        const int sa = it % kAStages;
+                        // both CTAs' converters wrote A stage sa, after their B stage landed
+                        if (!(ok = mbar_wait_warp(smem_u32(&S.afull[sa]), (it / kAStages) & 1, abort, &g_status)))
+                            break;
                         tc_fence_after();
-                        const uint64_t adesc = smem_desc_sw128(smem_u32(S.a[sa]));
-                        const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
+                        const uint64_t bdesc = smem_desc_sw128(b_base + (uint32_t)(kb - g0) * kBTileBytes);
+                        if (elect_one()) {
 #pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk)
-                            mma_f16_ss_pair(d, adesc + (uint64_t)((kk * 32) >> 4), bdesc + (uint64_t)((kk * 32) >> 4),
-                                            idesc, (kb != kb0 || kk != 0) ? 1u : 0u);
-                        mma_commit_pair_mc(smem_u32(&S.done[s]), kBoth);
+                            for (int kk = 0; kk < kBK / 16; ++kk)
+                                mma_f16_ts_pair(d, a_tm + sa * 32 + kk * 8, bdesc + (uint64_t)((kk * 32) >> 4), idesc,
+                                                (kb != kb0 || kk != 0) ? 1u : 0u);
+                            mma_commit_pair_mc(smem_u32(&S.adone[sa]), kBoth);
+                            if (group_end(kb, pk1)) mma_commit_pair_mc(smem_u32(&S.bdone[bs]), kBoth);
+                        }
+                        __syncwarp();
                     }
-                    if (ok) mma_commit_pair_mc(smem_u32(&S.accfull[buf]), kBoth);
+                    if (ok && elect_one()) mma_commit_pair_mc(smem_u32(&S.accfull[buf]), kBoth);
+                    __syncwarp();
                 }
             }
-            mma_commit_pair_mc(smem_u32(&S.drain), 0x1);
-            wait_teardown(smem_u32(&S.drain), 0);
+            if (elect_one()) {
+                mma_commit_pair_mc(smem_u32(&S.drain), 0x1);
+                wait_teardown(smem_u32(&S.drain), 0);
+            }
+            __syncwarp();
         }
     } else if (warp < 8) {
         regs_dec<88>();
-        const int row = (warp & 3) * 32 + lane;
-        const uint32_t sw64 = (row >> 1) & 3;
+        const int row = (warp & 3) * 32 + lane;  // weight row = TMEM lane
         const uint32_t afull0 = mapa_shared(smem_u32(&S.afull[0]), 0);
-        uint32_t it = 0;
+        const uint32_t a_tm = tmem + ((uint32_t)((warp & 3) * 32) << 16) + kPairACol;
+        uint32_t it = 0, gi = 0;
+        int ws = 0, w0 = 0;
         bool ok = true;
         for (int p = 0; p < sch.count && ok; ++p) {
             int u, pk0, pk1;
             sch.piece(p, u, pk0, pk1);
             for (int kb = pk0; kb < pk1; ++kb, ++it) {
-                const int s = it % kRing, sa = it % kAStages;
-                if (!(ok = mbar_wait(smem_u32(&S.full[s]), (it / kRing) & 1, abort, &g_status))) break;
+                if (group_start(kb, pk0)) {
+                    ws = gi % kWStages;
+                    w0 = kb & ~1;  // the weight copy starts at this even k-block
+                    if (!(ok = mbar_wait(smem_u32(&S.wfull[ws]), (gi / kWStages) & 1, abort, &g_status))) break;
+                    // the pair MMA reads this CTA's half of B: it must have landed before afull
+                    if (!(ok = mbar_wait(smem_u32(&S.bfull[gi % kBStages]), (gi / kBStages) & 1, abort, &g_status)))
+                        break;
+                    ++gi;
+                }
+                const int sa = it % kAStages;
+                // this row's 64 bytes of k-block kb: line (kb - w0) / 2 of 128 bytes, 16-byte chunks
+                // (kb - w0) % 2 * 4 + c, placed by the 128-byte swizzle at chunk ^ (row % 8)
+                const int j = kb - w0;
+                const uint8_t *line = S.w[ws] + (j >> 1) * (kBM * 128) + row * 128;
                 uint4 raw[4];
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
-                    raw[c] = *reinterpret_cast<const uint4 *>(S.w[s] + row * 64 + ((c ^ sw64) << 4));
+                    raw[c] = *reinterpret_cast<const uint4 *>(line + ((((j & 1) * 4 + c) ^ (row & 7)) << 4));
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&S.wread[s]));
-                uint4 h[8];
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    i8x4_to_f16x4(raw[c].x, h[2 * c].x, h[2 * c].y);
-                    i8x4_to_f16x4(raw[c].y, h[2 * c].z, h[2 * c].w);
-                    i8x4_to_f16x4(raw[c].z, h[2 * c + 1].x, h[2 * c + 1].y);
-                    i8x4_to_f16x4(raw[c].w, h[2 * c + 1].z, h[2 * c + 1].w);
-                }
-                // A tile sa was last read by the MMA of k-block it - kAStages
+                // the group's last weights are in registers: the stage may be refilled
+                if (lane == 0 && group_end(kb, pk1)) mbar_arrive(smem_u32(&S.wempty[ws]));
+                // A stage sa was last read by the MMA of k-block it - kAStages
                 if (it >= (uint32_t)kAStages) {
                     const uint32_t prev = it - kAStages;
-                    if (!(ok = mbar_wait(smem_u32(&S.done[prev % kRing]), (prev / kRing) & 1, abort, &g_status)))
+                    if (!(ok = mbar_wait(smem_u32(&S.adone[sa]), (prev / kAStages) & 1, abort, &g_status)))
                         break;
+                    tc_fence_after();
                 }
-                // row of 64 fp16 = 8 chunks of 16 bytes; 128-byte swizzle puts chunk c at c ^ (row % 8)
+                // the row's 64 fp16 values, two per 32-bit TMEM column, k ascending, in two halves
 #pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    *reinterpret_cast<uint4 *>(S.a[sa] + row * 128 + ((c ^ (row & 7)) << 4)) = h[c];
-                fence_proxy_async_smem();
+                for (int half = 0; half < 2; ++half) {
+                    uint32_t h[16];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const uint4 r4 = raw[2 * half + c];
+                        i8x4_to_f16x4(r4.x, h[8 * c + 0], h[8 * c + 1]);
+                        i8x4_to_f16x4(r4.y, h[8 * c + 2], h[8 * c + 3]);
+                        i8x4_to_f16x4(r4.z, h[8 * c + 4], h[8 * c + 5]);
+                        i8x4_to_f16x4(r4.w, h[8 * c + 6], h[8 * c + 7]);
+                    }
+                    tmem_st16(a_tm + sa * 32 + half * 16, h);
+                }
+                tmem_wait_st();
+                tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_remote(afull0 + (uint32_t)(sa * sizeof(uint64_t)));
             }
@@ -611,7 +703,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         regs_inc<184>();
         const int e = warp - kWarpEpi0;
         const int q = warp & 3;
-        const int col0 = (e >> 2) * 128;
+        const int col0 = (e >> 2) * kPairHalf;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         const uint32_t accempty0 = mapa_shared(smem_u32(&S.accempty[0]), 0);
         uint32_t g = 0;
@@ -625,16 +717,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             sch.piece(p, u, pk0, pk1);
             const int m0 = (u % m_tiles) * kPairBN;
             const int n0 = ((u / m_tiles) * 2 + (int)rank) * kBM;
-            int32_t tot[128];
+            int32_t tot[kPairHalf];
 #pragma unroll
-            for (int j = 0; j < 128; ++j) tot[j] = 0;
+            for (int j = 0; j < kPairHalf; ++j) tot[j] = 0;
             for (int kb0 = pk0; kb0 < pk1; kb0 += kcb, ++g) {
                 const int buf = g & 1;
                 if (!(ok = mbar_wait(smem_u32(&S.accfull[buf]), (g >> 1) & 1, abort, &g_status))) break;
                 tc_fence_after();
                 const uint32_t base = tmem + lane_base + buf * kPairBN + col0;
 #pragma unroll
-                for (int p = 0; p < 4; ++p) {
+                for (int p = 0; p < kPairHalf / 32; ++p) {
                     uint32_t v[32];
                     tmem_ld32(base + p * 32, v);
                     tmem_wait_ld();
@@ -650,7 +742,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 // partial piece: publish the int32 sums for the pair that ends this tile
                 int32_t *slot = slots + ((size_t)cluster * 2 + rank) * pair_slot_ints();
 #pragma unroll
-                for (int j = 0; j < 128; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
+                for (int j = 0; j < kPairHalf; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.pub));
@@ -679,7 +771,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     if (!ok) break;
                     const int32_t *slot = slots + ((size_t)c * 2 + rank) * pair_slot_ints();
 #pragma unroll
-                    for (int j = 0; j < 128; ++j) tot[j] += __ldcg(slot + (size_t)(col0 + j) * 128 + row);
+                    for (int j = 0; j < kPairHalf; ++j) tot[j] += __ldcg(slot + (size_t)(col0 + j) * 128 + row);
                 }
                 if (!ok) break;
             }
@@ -688,7 +780,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 if constexpr (kS32) {
                     int32_t *o = reinterpret_cast<int32_t *>(out);
 #pragma unroll
-                    for (int j = 0; j < 128; ++j) {
+                    for (int j = 0; j < kPairHalf; ++j) {
                         const int m = m0 + col0 + j;
                         if (m < M) o[(int64_t)m * N + n] = tot[j];
                     }
@@ -699,7 +791,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     const float zqn = kQOut ? __ldg(zq + n) : 0.f, rqn = kQOut ? __ldg(rq + n) : 0.f;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
-                    for (int j = 0; j < 128; ++j) {
+                    for (int j = 0; j < kPairHalf; ++j) {
                         const int m = m0 + col0 + j;
                         const int mc = m < M ? m : M - 1;
                         // per-token path (Eq. 3): one fp32 product s_m * sw_n
@@ -779,6 +871,24 @@ bool make_tmap_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uin
     return r == CUDA_SUCCESS;
 }
 
+// 3-D view {inner, rows, outer} of a row-major array with `row_bytes` per
+// row: element (i, r, o) sits at base + r row_bytes + o outer_bytes + i * size.
+// With outer_bytes equal to the inner span the view covers each row once, as
+// consecutive slices along it.
+bool make_tmap_3d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
+                  uint64_t outer, uint64_t row_bytes, uint64_t outer_bytes, uint32_t box_inner, uint32_t box_rows,
+                  uint32_t box_outer, CUtensorMapSwizzle swz) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {inner, rows, outer};
+    cuuint64_t strides[2] = {row_bytes, outer_bytes};
+    cuuint32_t box[3] = {box_inner, box_rows, box_outer};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(tm, dt, 3, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 template <int BN, bool kS32, bool kAsym, bool kQOut>
 cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
@@ -837,11 +947,15 @@ int pair_max_clusters() {
 
 template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
+    // codes as {64 fp16, M rows, K / 64 k-blocks}: a box of 96 rows x 4 k-blocks;
+    // weights as {128 int8, N rows, K / 128 k-block pairs}: a box of 128 rows x 2 pairs.
+    // Each inner span is a whole slice of the row (K % 128 == 0), so no copy
+    // reaches past a row; rows past M or N and k-blocks past K are zero-filled.
     CUtensorMap tm_q, tm_w;
-    if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
-                      (uint64_t)a.K * 2, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
-                      kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
+    if (!make_tmap_3d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, kBK, (uint64_t)a.M, (uint64_t)a.K / kBK,
+                      (uint64_t)a.K * 2, kBK * 2, kBK, kPairHalf, kGroupKB, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_3d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, 128, (uint64_t)a.N, (uint64_t)a.K / 128,
+                      (uint64_t)a.K, 128, 128, kBM, kGroupKB / 2, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(SmemPair) + 1024;
     static std::once_flag once;
@@ -874,7 +988,7 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
 template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
     if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut>(a, kcb, st);
-    if (a.M <= 128) return run_linear<128, kS32, kAsym, kQOut>(a, kcb, st);
+    if (a.M <= 128 || a.K % 128 != 0) return run_linear<128, kS32, kAsym, kQOut>(a, kcb, st);
     return run_linear_pair<kS32, kAsym, kQOut>(a, kcb, st);
 }
 
