@@ -358,8 +358,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 //   one per group frees the group's B stage.  A converter waits for its own
 //   CTA's B stage as well as its weights, so rank 0's wait on the converters
 //   of both CTAs covers both halves of B.
-//   Warpgroups: 0 = TMA producer / MMA issuer / TMEM allocator (56 regs),
-//   1 = converters (88 regs), 2-3 = epilogue (184 regs: 96 int32 totals).
+//   Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator (warpgroup 0,
+//   48 regs); 4-7 and 16-19 converters, taking the even and the odd k-blocks
+//   of the CTA's sequence in turn (72 regs: one warp per 32 TMEM lanes could
+//   not keep up); 8-15 epilogue (144 regs: 96 int32 totals).
 //   Needs K % 128 == 0 (the 3-D views must not reach past a row's end);
 //   other K use linear_kernel.
 // ---------------------------------------------------------------------------
@@ -368,6 +370,10 @@ constexpr int kPairHalf = kPairBN / 2;            // token rows per CTA (B is sp
 constexpr int kPairACol = 2 * kPairBN;            // TMEM: accumulators in [0, 2 kPairBN), then A stages
 constexpr int kAStages = (512 - kPairACol) / 32;  // 32-column fp16 A stages (128 rows x 64 k)
 constexpr int kGroupKB = 4;                       // k-blocks per TMA copy
+// 20 warps: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, 4-7 and 16-19
+// converters (even / odd k-blocks of the CTA's sequence), 8-15 epilogue
+constexpr int kPairThreads = 640;
+constexpr int kWarpConv1 = 16;
 constexpr int kWStages = 2;                       // weight stages: 2 x 128 rows x 128 int8, 128-byte swizzle (32 KB)
 constexpr int kBStages = 3;                       // token stages: 4 x 96 rows x 64 fp16, 128-byte swizzle (48 KB)
 constexpr uint32_t kWStageBytes = 2 * kBM * 128;
@@ -488,7 +494,7 @@ __device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) 
 }
 
 template <bool kS32, bool kAsym, bool kQOut>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
                        int N, int K, int ldy, int kcb, int relu, int32_t *__restrict__ ws,
@@ -512,7 +518,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kWStages; ++s) {
             mbar_init(smem_u32(&S.wfull[s]), 1);
-            mbar_init(smem_u32(&S.wempty[s]), 4);
+            mbar_init(smem_u32(&S.wempty[s]), 8);
         }
         for (int s = 0; s < kBStages; ++s) {
             mbar_init(smem_u32(&S.bfull[s]), 1);
@@ -546,8 +552,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
 
+    // registers at launch: 640 threads x 96; after the split 48 / 72 / 144 / 144 / 72 per warpgroup
     if (warp < 4) {
-        regs_dec<56>();
+        regs_dec<48>();
         if (warp == kWarpTma) {
             // the first weights into L2 while a programmatic predecessor may
             // still be writing the codes; then wait for it
@@ -639,39 +646,55 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
             __syncwarp();
         }
-    } else if (warp < 8) {
-        regs_dec<88>();
+    } else if (warp < kWarpEpi0 || warp >= kWarpConv1) {
+        regs_dec<72>();
+        // converters: warps 4-7 widen the even k-blocks of the CTA's sequence,
+        // warps 16-19 the odd ones; both release each weight stage
+        const uint32_t set = warp >= kWarpConv1 ? 1u : 0u;
         const int row = (warp & 3) * 32 + lane;  // weight row = TMEM lane
         const uint32_t afull0 = mapa_shared(smem_u32(&S.afull[0]), 0);
         const uint32_t a_tm = tmem + ((uint32_t)((warp & 3) * 32) << 16) + kPairACol;
         uint32_t it = 0, gi = 0;
-        int ws = 0, w0 = 0;
-        bool ok = true;
+        int wst = 0, w0 = 0;
+        bool gwait = false, ok = true;
         for (int p = 0; p < sch.count && ok; ++p) {
             int u, pk0, pk1;
             sch.piece(p, u, pk0, pk1);
             for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 if (group_start(kb, pk0)) {
-                    ws = gi % kWStages;
+                    wst = gi % kWStages;
                     w0 = kb & ~1;  // the weight copy starts at this even k-block
-                    if (!(ok = mbar_wait(smem_u32(&S.wfull[ws]), (gi / kWStages) & 1, abort, &g_status))) break;
-                    // the pair MMA reads this CTA's half of B: it must have landed before afull
-                    if (!(ok = mbar_wait(smem_u32(&S.bfull[gi % kBStages]), (gi / kBStages) & 1, abort, &g_status)))
-                        break;
                     ++gi;
+                    gwait = false;
+                }
+                const bool last = group_end(kb, pk1);
+                if ((it & 1u) != set) {
+                    if (last) {
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(smem_u32(&S.wempty[wst]));
+                    }
+                    continue;
+                }
+                if (!gwait) {
+                    const uint32_t gp = gi - 1;
+                    if (!(ok = mbar_wait(smem_u32(&S.wfull[wst]), (gp / kWStages) & 1, abort, &g_status))) break;
+                    // the pair MMA reads this CTA's half of B: it must have landed before afull
+                    if (!(ok = mbar_wait(smem_u32(&S.bfull[gp % kBStages]), (gp / kBStages) & 1, abort, &g_status)))
+                        break;
+                    gwait = true;
                 }
                 const int sa = it % kAStages;
                 // this row's 64 bytes of k-block kb: line (kb - w0) / 2 of 128 bytes, 16-byte chunks
                 // (kb - w0) % 2 * 4 + c, placed by the 128-byte swizzle at chunk ^ (row % 8)
                 const int j = kb - w0;
-                const uint8_t *line = S.w[ws] + (j >> 1) * (kBM * 128) + row * 128;
+                const uint8_t *line = S.w[wst] + (j >> 1) * (kBM * 128) + row * 128;
                 uint4 raw[4];
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
                     raw[c] = *reinterpret_cast<const uint4 *>(line + ((((j & 1) * 4 + c) ^ (row & 7)) << 4));
                 __syncwarp();
                 // the group's last weights are in registers: the stage may be refilled
-                if (lane == 0 && group_end(kb, pk1)) mbar_arrive(smem_u32(&S.wempty[ws]));
+                if (lane == 0 && last) mbar_arrive(smem_u32(&S.wempty[wst]));
                 // A stage sa was last read by the MMA of k-block it - kAStages
                 if (it >= (uint32_t)kAStages) {
                     const uint32_t prev = it - kAStages;
@@ -700,7 +723,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
         }
     } else {
-        regs_inc<184>();
+        regs_inc<144>();
         const int e = warp - kWarpEpi0;
         const int q = warp & 3;
         const int col0 = (e >> 2) * kPairHalf;
@@ -726,12 +749,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const uint32_t base = tmem + lane_base + buf * kPairBN + col0;
 #pragma unroll
-                for (int p = 0; p < kPairHalf / 32; ++p) {
-                    uint32_t v[32];
-                    tmem_ld32(base + p * 32, v);
+                for (int p = 0; p < kPairHalf / 16; ++p) {
+                    uint32_t v[16];
+                    tmem_ld16(base + p * 16, v);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) tot[p * 32 + j] += __float2int_rn(__uint_as_float(v[j]));
+                    for (int j = 0; j < 16; ++j) tot[p * 16 + j] += __float2int_rn(__uint_as_float(v[j]));
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -927,7 +950,7 @@ int pair_max_clusters() {
         cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 256);
-        cfg.blockDim = dim3(kThreads);
+        cfg.blockDim = dim3(kPairThreads);
         cfg.dynamicSmemBytes = smem;
         cudaLaunchAttribute attr;
         attr.id = cudaLaunchAttributeClusterDimension;
@@ -979,7 +1002,7 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
                          whole - shared >= kStreamKMinSaving && units * nkb < ((int64_t)1 << 30);
     const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
-    return launch_kernel(linear_pair_kernel<kS32, kAsym, kQOut>, dim3(2 * clusters), dim3(kThreads), smem, st, a.pdl,
+    return launch_kernel(linear_pair_kernel<kS32, kAsym, kQOut>, dim3(2 * clusters), dim3(kPairThreads), smem, st, a.pdl,
                          tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
                          a.s_tok, a.zc, a.rowsum, a.zq, a.rq, a.qmax_out);
 }
