@@ -366,6 +366,7 @@ def run_ours(args):
     decode = bench_decode(dev, peaks)
     asym = bench_asym(dev, layers, xs, ops_step, ms_per_step)
     lnq = bench_layernorm(dev, peaks)
+    qsweep = bench_quantize_sweep(dev, peaks)
     clip = bench_clipping(dev, peaks, calib_ms, calib_bytes)
 
     cpu = None
@@ -393,7 +394,8 @@ def run_ours(args):
         "clocks": clocks,
         "quantize": {"gbs": round(quant_gbs, 1), "hbm_peak_gbs": peaks["hbm"],
                      "frac": round(quant_gbs / peaks["hbm"], 4),
-                     "bytes_per_step": qbytes_total, "note": "fp16 X in + fp16 codes out + z, r"},
+                     "bytes_per_step": qbytes_total, "note": "fp16 X in + fp16 codes out + z, r",
+                     "sweep": qsweep},
         "calibrate": {"gbs": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9, 1),
                       "frac": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9 / peaks["hbm"], 4),
                       "tokens": cfg.T_cal, "ms_per_layer": [round(v, 3) for v in calib_ms]},
@@ -472,6 +474,51 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
             "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
             "over_symmetric_step": round(ms / ms_sym, 4),
             "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
+
+
+def bench_quantize_sweep(dev, peaks, reps: int = 20):
+    """The quantize kernel alone on OPT-6.7B-wide activations (K = 4096) from
+    2048 to 65,536 tokens (34 MB to 1.07 GB of traffic), L2 flushed before each
+    launch: small launches are bound by launch and first-load latency like a
+    plain copy, large ones by HBM bandwidth."""
+    import torch
+
+    from paper_2406_18832_gb300 import binding
+    K = 4096
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    g = torch.Generator(device=dev).manual_seed(77)
+    z = torch.randn(K, generator=g, device=dev)
+    r = torch.rand(K, generator=g, device=dev) * 10 + 1
+    out = []
+    for M in (2048, 8192, 65536):
+        x = (torch.randn(M, K, generator=g, device=dev) * 4).half()
+        q = torch.empty(M, K, dtype=torch.float16, device=dev)
+        y = torch.empty_like(x)
+
+        def med(fn):
+            for _ in range(3):
+                fn()
+            ts = []
+            for _ in range(reps):
+                flush.fill_(1)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                fn()
+                e1.record()
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            return statistics.median(ts)
+        ms = med(lambda: binding.ot_quantize_act(x, z, r, 8, q, binding.OT_CODE_F16))
+        mc = med(lambda: y.copy_(x))
+        byt = 4 * M * K + 8 * K
+        out.append({"tokens": M, "bytes": byt, "us": round(ms * 1e3, 2), "gbs": round(byt / (ms * 1e-3) / 1e9, 1),
+                    "frac_hbm": round(byt / (ms * 1e-3) / 1e9 / peaks["hbm"], 4),
+                    "torch_copy_gbs": round(4 * M * K / (mc * 1e-3) / 1e9, 1)})
+        del x, q, y
+    del flush
+    torch.cuda.empty_cache()
+    return {"workload": "quantize_kernel, K = 4096, fp16 X in + fp16 codes out", "l2": "flushed before each launch",
+            "per_size": out}
 
 
 def bench_layernorm(dev, peaks, reps: int = 200):
