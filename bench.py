@@ -367,6 +367,7 @@ def run_ours(args):
     asym = bench_asym(dev, layers, xs, ops_step, ms_per_step)
     lnq = bench_layernorm(dev, peaks)
     qsweep = bench_quantize_sweep(dev, peaks)
+    large = bench_large_gemm(dev, peaks)
     clip = bench_clipping(dev, peaks, calib_ms, calib_bytes)
 
     cpu = None
@@ -408,6 +409,7 @@ def run_ours(args):
                       "note": "GB300 has no tcgen05 int8 MMA; cuBLASLt int8 (torch._int_mm) of the QKV shape, "
                               "measured in this run"},
         "per_layer": per_layer,
+        "large_gemm": large,
         "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
                    "ratio": round(weights_fp16 / weights_int8, 3)},
         "block": block,
@@ -474,6 +476,53 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
             "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
             "over_symmetric_step": round(ms / ms_sym, 4),
             "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
+
+
+def bench_large_gemm(dev, peaks, reps: int = 10):
+    """OPT-66B fc1 / fc2 (9216 <-> 36864) at 4096 tokens, W8A8: the linear
+    alone (codes resident) against a cuBLAS fp16 GEMM of the same shape.
+    Codes and weights are drawn directly (uniform in [-127, 127]); every
+    launch streams ~0.5 GB, above the L2."""
+    import torch
+
+    from paper_2406_18832_gb300 import binding
+    M = 4096
+    ws = torch.zeros(binding.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+    g = torch.Generator(device=dev).manual_seed(66)
+    out = []
+    for name, K, N in (("fc1", 9216, 36864), ("fc2", 36864, 9216)):
+        q = torch.randint(-127, 128, (M, K), generator=g, device=dev, dtype=torch.int32).half()
+        qw = torch.randint(-127, 128, (N, K), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+        sw = torch.rand(N, generator=g, device=dev) * 1e-5
+        bf = torch.zeros(N, device=dev)
+        y = torch.empty(M, N, dtype=torch.float16, device=dev)
+        x16 = torch.randn(M, K, generator=g, device=dev).half()
+        w16 = (torch.randn(N, K, generator=g, device=dev) * 0.02).half()
+
+        def med(fn):
+            for _ in range(2):
+                fn()
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(reps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                fn()
+                e1.record()
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            return statistics.median(ts)
+        ms = med(lambda: binding.ot_linear(q, qw, sw, bf, 8, 8, y, workspace=ws))
+        del y
+        ms16 = med(lambda: torch.matmul(x16, w16.t()))
+        ops = 2 * M * K * N
+        out.append({"layer": name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 1),
+                    "tops": round(ops / (ms * 1e-3) / 1e12, 1), "frac_peak": round(ops / (ms * 1e-3) / 1e12 / peaks["bf16"], 4),
+                    "cublas_fp16_us": round(ms16 * 1e3, 1), "cublas_fp16_tflops": round(ops / (ms16 * 1e-3) / 1e12, 1)})
+        del q, qw, x16, w16
+    del ws
+    torch.cuda.empty_cache()
+    return {"workload": "opt-66b fc1 / fc2 at 4096 tokens, W8A8", "kernel": "linear_pair_kernel", "per_layer": out}
 
 
 def bench_quantize_sweep(dev, peaks, reps: int = 20):
