@@ -9,7 +9,12 @@
 // kcb k-blocks with kcb * 64 * qmax_a * qmax_w <= 2^24; each chunk's fp32
 // accumulator is converted to int32 (exact) and summed in registers.
 //
-// Design (one persistent CTA per SM, 16 warps):
+// Two kernels: linear_kernel (below; 32 < M <= 128, and any M when K % 128
+// != 0) and linear_pair_kernel (M > 128: CTA pairs, 192-token tiles; its own
+// comment further down).  The TMA and MMA roles of both run their loops with
+// the whole warp and issue from one elected lane.
+//
+// linear_kernel (one persistent CTA per SM, 16 warps):
 //   warp 0        TMA producer: per 64-wide k-block, the activation-code tile
 //                 (BN tokens x 64, fp16, 128-byte swizzle) and the weight tile
 //                 (128 rows x 64, int8, 64-byte swizzle) into a 6-stage ring.
@@ -393,7 +398,7 @@ struct alignas(1024) SmemPair {
     uint64_t afull[kAStages];           // rank 0 only: both CTAs' converters wrote their A stages (8 warps)
     uint64_t adone[kAStages];           // pair MMA of the k-block done (rank 0 commit, both CTAs)
     uint64_t accfull[2];                // pair MMA finished the chunk (rank 0 commit)
-    uint64_t accempty[2];               // rank 0 only: both CTAs' epilogues drained the chunk (16 warps)
+    uint64_t accempty[2];               // rank 0 only: both CTAs' epilogues drained the chunk (2 x 8 warps)
     uint64_t pub;                       // stream-K: the 8 epilogue warps stored their partial sums
     uint64_t drain;
     uint32_t tmem_base;
