@@ -128,9 +128,8 @@ __device__ __forceinline__ void ln_add8(LnSums &s, const uint4 &d) {
     s.sl += clo;
 }
 
-// mean and rstd of the row from the warp's exact sums (lane 0; IEEE fp32 in
-// the order documented above), broadcast to the warp.
-__device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
+// The warp's sums, added over its lanes (exact).
+__device__ __forceinline__ void ln_warp_reduce(LnSums &s) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         s.sh += __shfl_xor_sync(0xffffffffu, s.sh, o);
@@ -140,6 +139,11 @@ __device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float 
         s.c += __shfl_xor_sync(0xffffffffu, s.c, o);
         s.bad |= __shfl_xor_sync(0xffffffffu, s.bad, o);
     }
+}
+
+// mean and rstd of the row from its exact sums (lane 0; IEEE fp32 in the
+// order documented above), broadcast to the warp.
+__device__ __forceinline__ void ln_finish(const LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
     mean = 0.f;
     rstd = 0.f;
     if ((threadIdx.x & 31) == 0 && !s.bad) {
@@ -157,6 +161,89 @@ __device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float 
     }
     mean = __shfl_sync(0xffffffffu, mean, 0);
     rstd = __shfl_sync(0xffffffffu, rstd, 0);
+}
+
+__device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
+    ln_warp_reduce(s);
+    ln_finish(s, K, eps, mean, rstd);
+}
+
+// kWpr warps per row (kLnWarps / kWpr rows per CTA, grid-stride): lane l of
+// the row's warp w holds the 16-byte chunks l + 32 (i kWpr + w), i < kCh, in
+// registers (K <= 256 kWpr kCh).  Each warp adds its share of the exact sums;
+// the shares meet in shared memory (one named barrier per row group) and
+// every warp of the row finishes the same statistics from them, so the
+// result is that of one warp over the whole row.  Four 256-thread CTAs per
+// SM (64 registers) for rows of up to 4096 halves: measured on GB300 for
+// 2048 x 4096, 18.7 us against 20.9 us with one warp per row (the exact sums
+// cost ~40 instructions per element, so the kernel is issue-bound, not
+// HBM-bound).
+template <bool kF16Out, int kCh, int kWpr>
+__global__ void __launch_bounds__(kLnThreads, kCh <= 4 ? 4 : 2) layernorm_quantize_rows_kernel(
+    const __half *__restrict__ h, int64_t M, int64_t K, int64_t ldh, const float *__restrict__ gamma_r,
+    const float *__restrict__ beta_r, float eps, int qmax, void *q, int32_t *rowsum) {
+    constexpr int kRows = kLnWarps / kWpr;
+    __shared__ LnSums part[kLnWarps];
+    __shared__ int rsum[kLnWarps];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int rr = warp / kWpr, w = warp % kWpr;  // row of the CTA, warp of the row
+    const int bar = 1 + rr;                        // named barrier of the row's warps
+    for (int64_t m = (int64_t)blockIdx.x * kRows + rr; m < M; m += (int64_t)gridDim.x * kRows) {
+        const __half *row = h + m * ldh;
+        LnSums s{0, 0, 0, 0, 0, 0};
+        uint4 d[kCh];
+#pragma unroll
+        for (int i = 0; i < kCh; ++i) {
+            const int64_t k = (int64_t)(lane + 32 * (i * kWpr + w)) * 8;
+            d[i] = k < K ? __ldcs(reinterpret_cast<const uint4 *>(row + k)) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int i = 0; i < kCh; ++i)
+            if ((int64_t)(lane + 32 * (i * kWpr + w)) * 8 < K) ln_add8(s, d[i]);
+        ln_warp_reduce(s);
+        if (kWpr > 1) {
+            if (lane == 0) part[warp] = s;
+            asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(32 * kWpr) : "memory");
+            LnSums t{0, 0, 0, 0, 0, 0};
+#pragma unroll
+            for (int v = 0; v < kWpr; ++v) {
+                const LnSums &o = part[rr * kWpr + v];
+                t.sh += o.sh;
+                t.sl += o.sl;
+                t.a += o.a;
+                t.b += o.b;
+                t.c += o.c;
+                t.bad |= o.bad;
+            }
+            s = t;
+        }
+        float mean, rstd;
+        ln_finish(s, K, eps, mean, rstd);
+        int rs = 0;
+#pragma unroll
+        for (int i = 0; i < kCh; ++i) {
+            const int64_t k = (int64_t)(lane + 32 * (i * kWpr + w)) * 8;
+            if (k < K) rs += ln_codes8<kF16Out>(d[i], k, mean, rstd, gamma_r, beta_r, qmax, q, m * K + k, s.bad);
+        }
+        if (rowsum) {
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) rs += __shfl_xor_sync(0xffffffffu, rs, o);
+            if (kWpr > 1) {
+                if (lane == 0) rsum[warp] = rs;
+                asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(32 * kWpr) : "memory");
+                if (w == 0 && lane == 0) {
+                    int t = 0;
+#pragma unroll
+                    for (int v = 0; v < kWpr; ++v) t += rsum[rr * kWpr + v];
+                    rowsum[m] = t;
+                }
+            } else if (lane == 0) {
+                rowsum[m] = rs;
+            }
+        }
+        // the shares of this row may be overwritten by the next row only after every warp read them
+        if (kWpr > 1) asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(32 * kWpr) : "memory");
+    }
 }
 
 // One warp per row (kLnWarps rows per CTA, grid-stride).  kCh > 0: the lane
@@ -232,19 +319,22 @@ template <bool kF16Out>
 cudaError_t run_layernorm_quantize(const __half *h, int64_t M, int64_t K, int64_t ldh, const float *gamma_r,
                                    const float *beta_r, float eps, int qmax, void *q, int32_t *rowsum,
                                    cudaStream_t st) {
-    const int64_t ctas = (M + kLnWarps - 1) / kLnWarps;
-    const unsigned grid = (unsigned)(ctas < (1 << 30) ? ctas : (1 << 30));
-    const int64_t ch = (K + 255) / 256;  // 16-byte chunks per lane
-#define OT_LN_LAUNCH(C)                                                                                         \
-    layernorm_quantize_kernel<kF16Out, C><<<grid, kLnThreads, 0, st>>>(h, M, K, ldh, gamma_r, beta_r, eps, qmax, \
-                                                                       q, rowsum)
-    if (ch <= 4) OT_LN_LAUNCH(4);
-    else if (ch <= 8) OT_LN_LAUNCH(8);
-    else if (ch <= 16) OT_LN_LAUNCH(16);
-    else if (ch <= 24) OT_LN_LAUNCH(24);
-    else if (ch <= 32) OT_LN_LAUNCH(32);
-    else OT_LN_LAUNCH(0);
-#undef OT_LN_LAUNCH
+    const int64_t ch = (K + 255) / 256;  // 16-byte chunks per lane of one warp
+    auto grid_for = [&](int rows_per_cta) {
+        const int64_t ctas = (M + rows_per_cta - 1) / rows_per_cta;
+        return (unsigned)(ctas < (1 << 30) ? ctas : (1 << 30));
+    };
+#define OT_LN_ROWS(C, W)                                                                                      \
+    layernorm_quantize_rows_kernel<kF16Out, C, W><<<grid_for(kLnWarps / W), kLnThreads, 0, st>>>(              \
+        h, M, K, ldh, gamma_r, beta_r, eps, qmax, q, rowsum)
+    if (ch <= 4) OT_LN_ROWS(4, 1);
+    else if (ch <= 8) OT_LN_ROWS(4, 2);
+    else if (ch <= 16) OT_LN_ROWS(4, 4);
+    else if (ch <= 32) OT_LN_ROWS(8, 4);
+    else
+        layernorm_quantize_kernel<kF16Out, 0><<<grid_for(kLnWarps), kLnThreads, 0, st>>>(h, M, K, ldh, gamma_r, beta_r,
+                                                                                        eps, qmax, q, rowsum);
+#undef OT_LN_ROWS
     return cudaGetLastError();
 }
 
