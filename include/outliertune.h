@@ -138,7 +138,7 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  *           including calls replayed from a CUDA graph (a launch counter in
  *           the workspace, not a value fixed at launch, tells one call's
  *           partial sums from another's).  With it,
- *           prefill-sized calls (M > 128) and decode-sized calls (M <= 32) may
+ *           calls with M > 16 (tcgen05 kernels) and decode-sized calls (M <= 16) may
  *           share the (tile, K-slice) work evenly over the SMs and exchange
  *           exact int32 partial sums through it (stream-K); with NULL / too
  *           small, whole tiles are dealt out.  Calls that overlap on the GPU

@@ -9,7 +9,7 @@
 // kcb k-blocks with kcb * 64 * qmax_a * qmax_w <= 2^24; each chunk's fp32
 // accumulator is converted to int32 (exact) and summed in registers.
 //
-// Two kernels: linear_kernel (below; 32 < M <= 128, and any M when K % 128
+// Two kernels: linear_kernel (below; 16 < M <= 128, and any M when K % 128
 // != 0) and linear_pair_kernel (M > 128: CTA pairs, 192-token tiles; its own
 // comment further down).  The TMA and MMA roles of both run their loops with
 // the whole warp and issue from one elected lane.
@@ -69,8 +69,10 @@ struct alignas(1024) Smem {
     uint64_t accfull[2];            // chunk accumulator complete (MMA commit)
     uint64_t accempty[2];           // chunk accumulator drained (8 epilogue warps)
     uint64_t drain;                 // teardown: all issued MMAs complete
+    uint64_t pub;                   // stream-K: the 8 epilogue warps stored their partial sums
     uint32_t tmem_base;
     int abort;
+    unsigned long long epoch;       // stream-K: this launch's flag value
 };
 
 // Bounded wait that ignores the abort flag (used only while tearing down).
@@ -99,13 +101,99 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     hi = *reinterpret_cast<const uint32_t *>(&hb);
 }
 
+// Work of one worker (a CTA pair of linear_pair_kernel, a CTA of
+// linear_kernel): a list of pieces (tile u, k-blocks [kb0, kb1)).
+// Without a workspace the pieces are whole tiles dealt round-robin.  With a
+// workspace (stream-K) all but the last full round of tiles are still dealt
+// whole (neighbouring pairs then share weight and token tiles in L2), and
+// the remaining tiles' flattened (tile, k-block) space is cut into equal
+// contiguous ranges, one per pair, so no pair idles in a last partial round.
+// A pair walks its stream-K tiles in reverse, so the piece that does not end
+// a tile (its partial int32 sums go to the workspace) comes first and the
+// piece that ends a tile (it adds the partials of the earlier pairs) last.
+struct PairSched {
+    int nkb, streamk, count;
+    int first, stride, dp;      // whole tiles: u = first + p * stride for p < dp
+    int sk0;                    // first stream-K tile
+    int begin, end, u_last;     // this pair's stream-K range (flattened, relative to sk0)
+    int per, rem;
+
+    __device__ void init(int num_units, int nkb_, int nclusters, int cluster, bool use_streamk) {
+        nkb = nkb_;
+        streamk = use_streamk ? 1 : 0;
+        first = cluster;
+        stride = nclusters;
+        if (!streamk) {
+            dp = cluster < num_units ? (num_units - cluster + nclusters - 1) / nclusters : 0;
+            count = dp;
+            return;
+        }
+        const int rounds = num_units / nclusters;
+        dp = rounds >= 2 ? rounds - 1 : 0;
+        sk0 = dp * nclusters;
+        const int total = (num_units - sk0) * nkb;
+        const int active = total < nclusters ? total : nclusters;
+        per = active > 0 ? total / active : 0;
+        rem = active > 0 ? total % active : 0;
+        count = dp;
+        if (cluster >= active) return;
+        begin = cluster * per + (cluster < rem ? cluster : rem);
+        end = begin + per + (cluster < rem ? 1 : 0);
+        u_last = (end - 1) / nkb;
+        count += u_last - begin / nkb + 1;
+    }
+    __device__ void piece(int p, int &u, int &kb0, int &kb1) const {
+        if (p < dp) {
+            u = first + p * stride;
+            kb0 = 0;
+            kb1 = nkb;
+            return;
+        }
+        const int v = u_last - (p - dp);  // stream-K tile, relative to sk0
+        u = sk0 + v;
+        kb0 = max(begin, v * nkb) - v * nkb;
+        kb1 = min(end, (v + 1) * nkb) - v * nkb;
+    }
+    // the first pair whose stream-K range holds part of tile u
+    __device__ int first_owner(int u) const {
+        const int x = (u - sk0) * nkb;
+        const int big = rem * (per + 1);
+        return x < big ? x / (per + 1) : rem + (x - big) / per;
+    }
+};
+
+// Stream-K workspace: per pair and CTA rank, 256 token columns x 128 weight
+// rows of int32 partial sums (column-major, so a warp's stores are
+// contiguous), then one 64-bit flag per pair and rank holding the launch
+// epoch once its partials are complete, then the epoch counter and a count of
+// the CTAs done with the launch.  Each launch takes epoch = counter + 1; the
+// last CTA to finish stores it back (a launch starts only after the previous
+// one on the stream ended, so all CTAs of a launch read one value), so the
+// epochs grow from launch to launch on the device -- also when the launch is
+// replayed from a CUDA graph -- and a flag left by an earlier launch never
+// matches.  A zero-filled workspace starts the count.
+__host__ __device__ constexpr size_t pair_slot_ints() { return (size_t)256 * 128; }
+
+// {epoch of the last launch, CTAs done with this one}, after the flags
+__device__ __forceinline__ unsigned long long *pair_ctl(int32_t *ws, int nclusters) {
+    return reinterpret_cast<unsigned long long *>(ws + (size_t)nclusters * 2 * pair_slot_ints()) +
+           (size_t)nclusters * 2;
+}
+
+__device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) {
+    uint64_t v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
 template <int BN, bool kS32, bool kAsym, bool kQOut>
 __global__ void __launch_bounds__(kThreads, 1)
     linear_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                   const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
                   int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok,
                   const int32_t *__restrict__ zc, const int32_t *__restrict__ rowsum,
-                  const float *__restrict__ zq, const float *__restrict__ rq, int qmax_out) {
+                  const float *__restrict__ zq, const float *__restrict__ rq, int qmax_out,
+                  int32_t *__restrict__ ws, int ws_pairs) {
     extern __shared__ uint8_t smem_raw[];
     Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -115,6 +203,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nkb = (K + kBK - 1) / kBK;
     volatile int *abort = &S.abort;
     constexpr uint32_t kTxBytes = BN * 128 + kBM * kBK;
+    // With a workspace (the prefill kernel's layout, ws_pairs pairs of slots)
+    // the CTAs split tiles along K like the pairs of linear_pair_kernel.
+    PairSched sch;
+    sch.init(num_tiles, nkb, gridDim.x, blockIdx.x, ws != nullptr);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -128,7 +220,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(smem_u32(&S.accempty[b]), kNumEpiWarps);
         }
         mbar_init(smem_u32(&S.drain), 1);
+        mbar_init(smem_u32(&S.pub), kNumEpiWarps);
         S.abort = 0;
+        S.epoch = ws ? __ldcg(pair_ctl(ws, ws_pairs)) + 1 : 0;
         fence_barrier_init();
     }
     if (warp == kWarpTma && lane == 0) {
@@ -148,16 +242,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kWarpTma) {
         // weights of the first tile into L2 while a programmatic predecessor
         // may still be writing the codes; then wait for it
-        if (blockIdx.x < num_tiles && elect_one())
-            for (int kb = 0; kb < nkb && kb < kStages; ++kb)
-                tma_prefetch_l2_2d(&tm_w, kb * kBK, (blockIdx.x / m_tiles) * kBM);
+        if (sch.count > 0 && elect_one()) {
+            int u, pk0, pk1;
+            sch.piece(0, u, pk0, pk1);
+            for (int kb = pk0; kb < pk1 && kb < pk0 + kStages; ++kb)
+                tma_prefetch_l2_2d(&tm_w, kb * kBK, (u / m_tiles) * kBM);
+        }
         __syncwarp();
         grid_dep_wait();
         uint32_t it = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
-            const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
-            for (int kb = 0; kb < nkb; ++kb, ++it) {
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
+            const int m0 = (u % m_tiles) * BN, n0 = (u / m_tiles) * kBM;
+            for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 const int s = it % kStages;
                 const uint32_t ph = (it / kStages) & 1;
                 if (!(ok = mbar_wait_warp(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status))) break;
@@ -180,13 +279,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t idesc = idesc_f16_f32(kBM, BN);
         uint32_t it = 0, g = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
-            for (int kb0 = 0; kb0 < nkb && ok; kb0 += kcb, ++g) {
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
+            for (int kb0 = pk0; kb0 < pk1 && ok; kb0 += kcb, ++g) {
                 const int buf = g & 1;
                 if (!(ok = mbar_wait_warp(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
                 tc_fence_after();
                 const uint32_t d = tmem + kTmemAccCol + buf * BN;
-                const int kb1 = min(nkb, kb0 + kcb);
+                const int kb1 = min(pk1, kb0 + kcb);
                 for (int kb = kb0; kb < kb1; ++kb, ++it) {
                     const int s = it % kStages;
                     const uint32_t ph = (it / kStages) & 1;
@@ -221,8 +322,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t it = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
-            for (int kb = 0; kb < nkb; ++kb, ++it) {
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
+            for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 const int s = it % kStages;
                 const uint32_t ph = (it / kStages) & 1;
                 if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
@@ -258,12 +361,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t g = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
-            const int m0 = (t % m_tiles) * BN, n0 = (t / m_tiles) * kBM;
+        const int row = q * 32 + lane;  // weight row of the tile
+        unsigned long long *flags =
+            ws ? reinterpret_cast<unsigned long long *>(ws + (size_t)ws_pairs * 2 * pair_slot_ints()) : nullptr;
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
+            const int m0 = (u % m_tiles) * BN, n0 = (u / m_tiles) * kBM;
             int32_t tot[CPW];
 #pragma unroll
             for (int j = 0; j < CPW; ++j) tot[j] = 0;
-            for (int kb0 = 0; kb0 < nkb; kb0 += kcb, ++g) {
+            for (int kb0 = pk0; kb0 < pk1; kb0 += kcb, ++g) {
                 const int buf = g & 1;
                 if (!(ok = mbar_wait(smem_u32(&S.accfull[buf]), (g >> 1) & 1, abort, &g_status))) break;
                 tc_fence_after();
@@ -283,6 +391,43 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(smem_u32(&S.accempty[buf]));
             }
             if (!ok) break;
+            if (pk1 < nkb) {
+                // partial piece: publish the int32 sums for the CTA that ends this tile
+                int32_t *slot = ws + (size_t)blockIdx.x * pair_slot_ints();
+#pragma unroll
+                for (int j = 0; j < CPW; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&S.pub));
+                // a CTA has at most one partial piece per launch: phase 0 of pub
+                if (warp == kWarpEpi0 && lane == 0 && mbar_wait(smem_u32(&S.pub), 0, abort, &g_status)) {
+                    __threadfence();
+                    atomicExch(flags + blockIdx.x, S.epoch);
+                }
+                continue;
+            }
+            if (pk0 > 0) {
+                // this CTA ends the tile: add the partial sums of the CTAs that began it
+                const int c_lo = sch.first_owner(u);
+                for (int c = c_lo; c < (int)blockIdx.x && ok; ++c) {
+                    const unsigned long long *f = flags + c;
+                    const uint64_t t0 = globaltimer_ns();
+                    while (ld_acquire_u64(f) != S.epoch) {
+                        if (*abort) { ok = false; break; }
+                        if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                            atomicExch(&g_status, (int)OT_ERR_TIMEOUT);
+                            *abort = 1;
+                            ok = false;
+                            break;
+                        }
+                    }
+                    if (!ok) break;
+                    const int32_t *slot = ws + (size_t)c * pair_slot_ints();
+#pragma unroll
+                    for (int j = 0; j < CPW; ++j) tot[j] += __ldcg(slot + (size_t)(col0 + j) * 128 + row);
+                }
+                if (!ok) break;
+            }
             const int n = n0 + q * 32 + lane;
             if (n < N) {
                 if constexpr (kS32) {
@@ -330,6 +475,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kWarpAlloc) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
+    }
+    if (ws && threadIdx.x == 0) {
+        unsigned long long *ctl = pair_ctl(ws, ws_pairs);
+        if (atomicAdd(ctl + 1, 1ull) == (unsigned long long)gridDim.x - 1) {
+            // the last CTA of the launch: hand the epoch to the next launch
+            ctl[1] = 0;
+            ctl[0] = S.epoch;
+        }
     }
 }
 
@@ -412,90 +565,6 @@ struct alignas(1024) SmemPair {
 __device__ __forceinline__ bool group_start(int kb, int kb0) { return kb == kb0 || (kb & (kGroupKB - 1)) == 0; }
 __device__ __forceinline__ bool group_end(int kb, int kb1) {
     return kb == kb1 - 1 || (kb & (kGroupKB - 1)) == kGroupKB - 1;
-}
-
-// Work of one CTA pair: a list of pieces (pair tile u, k-blocks [kb0, kb1)).
-// Without a workspace the pieces are whole tiles dealt round-robin.  With a
-// workspace (stream-K) all but the last full round of tiles are still dealt
-// whole (neighbouring pairs then share weight and token tiles in L2), and
-// the remaining tiles' flattened (tile, k-block) space is cut into equal
-// contiguous ranges, one per pair, so no pair idles in a last partial round.
-// A pair walks its stream-K tiles in reverse, so the piece that does not end
-// a tile (its partial int32 sums go to the workspace) comes first and the
-// piece that ends a tile (it adds the partials of the earlier pairs) last.
-struct PairSched {
-    int nkb, streamk, count;
-    int first, stride, dp;      // whole tiles: u = first + p * stride for p < dp
-    int sk0;                    // first stream-K tile
-    int begin, end, u_last;     // this pair's stream-K range (flattened, relative to sk0)
-    int per, rem;
-
-    __device__ void init(int num_units, int nkb_, int nclusters, int cluster, bool use_streamk) {
-        nkb = nkb_;
-        streamk = use_streamk ? 1 : 0;
-        first = cluster;
-        stride = nclusters;
-        if (!streamk) {
-            dp = cluster < num_units ? (num_units - cluster + nclusters - 1) / nclusters : 0;
-            count = dp;
-            return;
-        }
-        const int rounds = num_units / nclusters;
-        dp = rounds >= 2 ? rounds - 1 : 0;
-        sk0 = dp * nclusters;
-        const int total = (num_units - sk0) * nkb;
-        const int active = total < nclusters ? total : nclusters;
-        per = active > 0 ? total / active : 0;
-        rem = active > 0 ? total % active : 0;
-        count = dp;
-        if (cluster >= active) return;
-        begin = cluster * per + (cluster < rem ? cluster : rem);
-        end = begin + per + (cluster < rem ? 1 : 0);
-        u_last = (end - 1) / nkb;
-        count += u_last - begin / nkb + 1;
-    }
-    __device__ void piece(int p, int &u, int &kb0, int &kb1) const {
-        if (p < dp) {
-            u = first + p * stride;
-            kb0 = 0;
-            kb1 = nkb;
-            return;
-        }
-        const int v = u_last - (p - dp);  // stream-K tile, relative to sk0
-        u = sk0 + v;
-        kb0 = max(begin, v * nkb) - v * nkb;
-        kb1 = min(end, (v + 1) * nkb) - v * nkb;
-    }
-    // the first pair whose stream-K range holds part of tile u
-    __device__ int first_owner(int u) const {
-        const int x = (u - sk0) * nkb;
-        const int big = rem * (per + 1);
-        return x < big ? x / (per + 1) : rem + (x - big) / per;
-    }
-};
-
-// Stream-K workspace: per pair and CTA rank, 256 token columns x 128 weight
-// rows of int32 partial sums (column-major, so a warp's stores are
-// contiguous), then one 64-bit flag per pair and rank holding the launch
-// epoch once its partials are complete, then the epoch counter and a count of
-// the CTAs done with the launch.  Each launch takes epoch = counter + 1; the
-// last CTA to finish stores it back (a launch starts only after the previous
-// one on the stream ended, so all CTAs of a launch read one value), so the
-// epochs grow from launch to launch on the device -- also when the launch is
-// replayed from a CUDA graph -- and a flag left by an earlier launch never
-// matches.  A zero-filled workspace starts the count.
-__host__ __device__ constexpr size_t pair_slot_ints() { return (size_t)256 * 128; }
-
-// {epoch of the last launch, CTAs done with this one}, after the flags
-__device__ __forceinline__ unsigned long long *pair_ctl(int32_t *ws, int nclusters) {
-    return reinterpret_cast<unsigned long long *>(ws + (size_t)nclusters * 2 * pair_slot_ints()) +
-           (size_t)nclusters * 2;
-}
-
-__device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) {
-    uint64_t v;
-    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-    return v;
 }
 
 template <bool kS32, bool kAsym, bool kQOut>
@@ -917,6 +986,8 @@ bool make_tmap_3d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uin
     return r == CUDA_SUCCESS;
 }
 
+int pair_max_clusters();
+
 template <int BN, bool kS32, bool kAsym, bool kQOut>
 cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     CUtensorMap tm_q, tm_w;
@@ -935,10 +1006,22 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
-    const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
+    const int64_t nkb = (a.K + kBK - 1) / kBK;
+    // Stream-K over CTAs, in the prefill kernel's workspace layout (a slot and
+    // a flag per CTA; one CTA per SM, at most 2 x pair_max_clusters of them),
+    // when it shortens the busiest CTA's work by at least kStreamKMinSaving
+    // k-blocks (e.g. OPT-13B fc2 at 128 tokens: 40 tiles of 320 k-blocks).
+    const int pairs = pair_max_clusters();
+    const int workers = num_sms() < 2 * pairs ? num_sms() : 2 * pairs;
+    const int64_t whole = (tiles + workers - 1) / workers * nkb;
+    const int64_t shared = (tiles * nkb + workers - 1) / workers;
+    const bool streamk = a.workspace != nullptr && a.workspace_bytes >= pair_workspace_bytes(pairs) &&
+                         whole - shared >= kStreamKMinSaving && tiles * nkb < ((int64_t)1 << 30);
+    const int grid = streamk ? workers : (int)(tiles < num_sms() ? tiles : num_sms());
+    int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
     return launch_kernel(linear_kernel<BN, kS32, kAsym, kQOut>, dim3(grid), dim3(kThreads), smem, st, a.pdl, tm_q, tm_w,
                          a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
-                         a.rowsum, a.zq, a.rq, a.qmax_out);
+                         a.rowsum, a.zq, a.rq, a.qmax_out, ws, pairs);
 }
 
 // Clusters of the pair kernel that fit on the device at once (one per two SMs).
@@ -1012,7 +1095,7 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
                          a.s_tok, a.zc, a.rowsum, a.zq, a.rq, a.qmax_out);
 }
 
-// M <= 32 goes to the decode kernel (gemv.cu) before this dispatch.
+// M <= 16 goes to the decode kernel (gemv.cu) before this dispatch.
 template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
     if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut>(a, kcb, st);
@@ -1028,8 +1111,10 @@ bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, ui
     return make_tmap_2d(tm, dt, base, inner, rows, row_bytes, box_inner, box_rows, swz);
 }
 
-// Token counts up to this go to the mma.sync weight-streaming kernel (gemv.cu).
-constexpr int64_t kGemvMaxTokens = 32;
+// Token counts up to this go to the mma.sync weight-streaming kernel (gemv.cu)
+// (measured crossover on GB300: OPT-13B QKV at 17-32 tokens 27.0-27.6 us in
+// linear_kernel against 27.8-32.0 us in gemv.cu; fc2 33.4-33.6 against 35.0-41.6).
+constexpr int64_t kGemvMaxTokens = 16;
 
 // Largest number of 64-wide k-blocks whose fp32 partial sums stay exact:
 // kcb * 64 * qmax_a * qmax_w <= 2^24.

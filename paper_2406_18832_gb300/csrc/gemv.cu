@@ -1,11 +1,12 @@
 // gemv.cu -- the quantized linear of Eq. 6 / Eq. 7 for decode-sized token
-// counts (M <= 32), where the product is bound by reading the int8 weights
+// counts (M <= 16), where the product is bound by reading the int8 weights
 // from HBM (each weight byte is used by only M tokens).
 //
-// A 128-row tcgen05 MMA costs about 118 cycles whatever its token count, which
-// caps weight consumption at ~17 bytes per clock per SM (~5 TB/s on GB300),
-// below the HBM rate.  Warp-level mma.sync m16n8k16 (f16 in, f32 accumulate)
-// has throughput to spare at M <= 32, so the kernel is a weight stream:
+// At a few tokens a tcgen05 tile wastes most of its N width and its fixed
+// per-MMA cost caps the weight stream; warp-level mma.sync m16n8k16 (f16 in,
+// f32 accumulate) has throughput to spare, so the kernel is a weight stream
+// (measured on GB300, OPT-13B QKV and fc2 shapes: faster than the tcgen05
+// kernel up to 16 tokens, slower from 17):
 //   - work units are (tile of 128 weight rows, 256-wide K slice); one
 //     persistent CTA per SM takes a contiguous range of units, an equal share
 //     of all of them (stream-K), so every SM streams the same number of bytes;
@@ -511,7 +512,7 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     const bool d = a.pdl;
     if (a.M <= 8) return a.out_s32 ? run_gemv<1, true>(tm_w, tm_a, p, st, d) : run_gemv<1, false>(tm_w, tm_a, p, st, d);
     if (a.M <= 16) return a.out_s32 ? run_gemv<2, true>(tm_w, tm_a, p, st, d) : run_gemv<2, false>(tm_w, tm_a, p, st, d);
-    return a.out_s32 ? run_gemv<4, true>(tm_w, tm_a, p, st, d) : run_gemv<4, false>(tm_w, tm_a, p, st, d);
+    return cudaErrorInvalidValue;  // more than 16 tokens go to the tcgen05 kernels
 }
 
 }  // namespace ot

@@ -1,6 +1,6 @@
 """Asymmetric per-output-channel weights (the paper's "Int8"): the fold, the
 code row sums and the corrected linear against the oracle, bit for bit, on
-every kernel of the path (decode M <= 32, 32 < M <= 128, prefill M > 128),
+every kernel of the path (decode M <= 16, 16 < M <= 128, prefill M > 128),
 with and without the stream-K workspace."""
 import numpy as np
 import pytest

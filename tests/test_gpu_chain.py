@@ -2,7 +2,7 @@
 the kernel that produces the activation): fc1's epilogue, ReLU included,
 writes fc2's activation codes round((v - z') * r') instead of its fp16
 output.  Against the oracle bit for bit on every kernel of the path (decode
-M <= 32, 32 < M <= 128, prefill M > 128), with and without the stream-K
+M <= 16, 16 < M <= 128, prefill M > 128), with and without the stream-K
 workspace, on cases built to land on exact rounding ties, and at the full
 size of an OPT-30B block's fc1 on sampled rows."""
 import numpy as np

@@ -1,11 +1,13 @@
-"""Decode-sized linears (M <= 32 tokens): the weight-streaming kernel against
+"""Decode-sized linears (up to 32 tokens; the weight-streaming kernel takes
+M <= 16, the single-CTA tcgen05 kernel 17-32): both against
 the oracle, bit for bit, with the workspace (tiles split between CTAs along K,
 int32 partials exchanged through it) and without (whole tiles per CTA).
 
 Shapes cover ragged N (not a multiple of the 128-row tile), ragged K (not a
 multiple of the 256-wide unit, nor of the 64-wide window), K long enough that
 every warp flushes its fp32 chunk sums into int32 several times, tiles split
-over up to 128 CTAs, and both token-group widths (M <= 16, M <= 32)."""
+over up to 128 CTAs, both token-group widths of the weight stream (M <= 8,
+M <= 16) and the tcgen05 kernel just above them (17-32 tokens)."""
 import numpy as np
 import pytest
 import torch

@@ -1,8 +1,8 @@
 """ot_linear_fused: the activation quantization (Eq. 6-7) and the linear in one
 call, the linear launched as a programmatic dependent of the quantization
 (its weight loads overlap it; its code loads wait for it).  Against the
-oracle bit for bit on every kernel of the path (decode M <= 32,
-32 < M <= 128, prefill M > 128), with and without the stream-K workspace,
+oracle bit for bit on every kernel of the path (decode M <= 16,
+16 < M <= 128, prefill M > 128), with and without the stream-K workspace,
 with a strided X, under CUDA-graph capture, and in back-to-back calls that
 reuse one code buffer or follow a kernel that rewrote the weights."""
 import numpy as np

@@ -94,3 +94,25 @@ def test_streamk_under_cuda_graph_replay(M, N, K):
         torch.cuda.synchronize()
         assert B.ot_get_device_status() == B.OT_OK
         assert torch.equal(acc, want), seed
+
+
+@pytest.mark.parametrize("M,N,K", [(129, 1, 128), (193, 257, 384), (256, 512, 640), (385, 1024, 4224),
+                                   (512, 1024, 2176), (700, 2048, 896)])
+def test_pair_kernel_groups_and_ragged_edges(M, N, K):
+    """The prefill kernel (M > 128, K % 128 == 0) loads four k-blocks per copy:
+    K of 2, 6, 10, 66, 34 and 14 k-blocks (last group short), stream-K pieces
+    that start at odd k-blocks, one-row and one-column tails, N = 1.  Against
+    the oracle's int64 product, with and without the workspace."""
+    from paper_2406_18832_gb300 import binding as B
+    dev = "cuda"
+    q = _codes((M, K), 127, 3 * M + K)
+    qw = _codes((N, K), 127, 5 * N + K).to(torch.int8)
+    want = oracle.matmul(q.numpy().astype(np.int8), qw.numpy())
+    qd, qwd = q.half().to(dev), qw.to(dev)
+    ws = torch.zeros(B.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+    for workspace in (False, ws, ws):
+        acc = torch.full((M, N), -3, dtype=torch.int32, device=dev)
+        B.ot_linear_s32(qd, qwd, 8, 8, acc, workspace=workspace)
+        torch.cuda.synchronize()
+        assert B.ot_get_device_status() == B.OT_OK
+        assert np.array_equal(acc.cpu().numpy().astype(np.int64), want)
