@@ -368,6 +368,7 @@ def run_ours(args):
     lnq = bench_layernorm(dev, peaks)
     qsweep = bench_quantize_sweep(dev, peaks)
     large = bench_large_gemm(dev, peaks)
+    sweep = bench_token_sweep(dev, peaks)
     clip = bench_clipping(dev, peaks, calib_ms, calib_bytes)
 
     cpu = None
@@ -410,6 +411,7 @@ def run_ours(args):
                               "measured in this run"},
         "per_layer": per_layer,
         "large_gemm": large,
+        "token_sweep": sweep,
         "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
                    "ratio": round(weights_fp16 / weights_int8, 3)},
         "block": block,
@@ -476,6 +478,51 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
             "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
             "over_symmetric_step": round(ms / ms_sym, 4),
             "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
+
+
+def bench_token_sweep(dev, peaks, reps: int = 20):
+    """OPT-13B QKV and fc2 (Int6) at 1, 16, 128, 1024 and 4096 tokens: the
+    linear alone (codes resident, consecutive calls on rotating weight copies
+    so that weights come from HBM), CUDA-graph replay.  The roofline time of a
+    point is the larger of its weight bytes over the HBM peak and its
+    operations over the dense tensor peak; frac = roofline time / time."""
+    import torch
+
+    from paper_2406_18832_gb300 import binding, synth
+    c = synth.CONFIGS[3]
+    ws = torch.zeros(binding.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+    out = []
+    for li in (0, 3):
+        layer = c.layers[li]
+        N, K = layer.N, layer.K
+        g = torch.Generator(device=dev).manual_seed(4000 + li)
+        copies = max(2, -(-3 * 129 * 2 ** 20 // (N * K)))
+        qws = [torch.randint(-31, 32, (N, K), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+               for _ in range(copies)]
+        sw = torch.rand(N, generator=g, device=dev) * 1e-3
+        bf = torch.zeros(N, device=dev)
+        for M in (1, 16, 128, 1024, 4096):
+            q = torch.randint(-31, 32, (M, K), generator=g, device=dev, dtype=torch.int32).half()
+            y = torch.empty(M, N, dtype=torch.float16, device=dev)
+            n = reps if M <= 128 else 4
+
+            def calls():
+                for i in range(n):
+                    binding.ot_linear(q, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
+            ms = _graph_ms(calls, n)
+            ops = 2 * M * N * K
+            t_roof = max(N * K / (peaks["hbm"] * 1e9), ops / (peaks["bf16"] * 1e12))
+            out.append({"layer": layer.name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 2),
+                        "tops": round(ops / (ms * 1e-3) / 1e12, 1),
+                        "weight_gbs": round(N * K / (ms * 1e-3) / 1e9, 1),
+                        "bound": "hbm" if N * K / (peaks["hbm"] * 1e9) > ops / (peaks["bf16"] * 1e12) else "tensor",
+                        "frac_roofline": round(t_roof / (ms * 1e-3), 4)})
+            del q, y
+        del qws
+    del ws
+    torch.cuda.empty_cache()
+    return {"workload": "opt-13b QKV and fc2, Int6, 1-4096 tokens", "timing": "CUDA graph replay, rotating weights",
+            "per_point": out}
 
 
 def bench_large_gemm(dev, peaks, reps: int = 10):
