@@ -5,15 +5,16 @@
 //   q = round(((h - mean) * rstd) * gamma_r + beta_r),
 //   gamma_r = gamma * r,  beta_r = (beta - z) * r   (folded once, offline).
 // The row statistics are exact so the codes do not depend on a reduction
-// order: h * 2^24 is an integer H for every fp16 h (|H| < 2^40), sum H is an
-// exact int64 and sum H^2 is kept as three exact 64-bit partial sums of
-// 20-bit halves (H = a 2^20 + b:  H^2 = a^2 2^40 + 2ab 2^20 + b^2), combined in
-// 128 bits once per row.  Mean and 1/sqrt(var + eps) then follow by a fixed
-// sequence of IEEE fp32 operations (one lane per row) and the codes by one
-// fp32 fma per element.
-// HBM-bound: one warp per row, no block barriers; rows up to 8192 wide are
-// held in registers (one HBM read with the whole row in flight), longer ones
-// are streamed and read again from L2 for the codes.
+// order: h * 2^24 is an integer H for every fp16 h (|H| < 2^40), split as
+// H = A 2^20 + B with |A| <= 2^20, |B| <= 2^19 (h rounded to a multiple of
+// 2^-4, and the rest); sum H is kept as the exact sums of A and of B, and
+// sum H^2 = 2^40 sum A^2 + 2^21 sum AB + sum B^2 as three exact 64-bit sums,
+// combined in 128 bits once per row.  Mean and 1/sqrt(var + eps) then follow
+// by a fixed sequence of IEEE fp32 operations (one lane per row) and the
+// codes by one fp32 fma per element.
+// Rows up to 8192 wide are held in registers by one to eight warps (one HBM
+// read with the whole row in flight), longer ones are streamed by one warp
+// and read again from L2 for the codes.
 #include <cuda_fp16.h>
 
 #include "ot_common.cuh"
@@ -39,35 +40,59 @@ __global__ void __launch_bounds__(256) fold_layernorm_kernel(const __half *__res
 }
 
 struct LnSums {
-    long long sh, sl;             // sum of the signed 20-bit halves of H: S1 = sh 2^20 + sl
-    unsigned long long a, b, c;   // sum hi^2, sum hi*lo, sum lo^2 of the 20-bit halves of |H|
+    long long s1;                 // S1 = sum H = 2^20 sum A + sum B
+    unsigned long long a, b, c;   // sum A^2, sum AB (two's complement), sum B^2
     int bad;                      // non-finite values seen
 };
 
-// One fp16 value (bits u) into the sums, in 32-bit integer arithmetic: for
-// exponent field e and fraction f, |H| = h 2^24 = mant << sh with mant =
-// f | 1024 (f for e = 0) and sh = max(e - 1, 0) <= 29; its 20-bit halves are
-// hi = |H| >> 20 and lo = |H| & (2^20 - 1).  The caller's chunk of 8 values
-// keeps the signed half sums in int32 (|sum| < 2^23).
-__device__ __forceinline__ void ln_add_bits(uint32_t u, int &chi, int &clo, LnSums &s) {
-    const uint32_t e = (u >> 10) & 31u, f = u & 1023u;
-    s.bad |= (e == 31u);
-    const uint32_t nz = e != 0u;
-    const uint32_t mant = f | (nz << 10);
-    const uint32_t sh = e - nz;
-    const uint32_t t = mant << (sh < 20u ? sh : 0u);                 // < 2^31 when sh < 20
-    const uint32_t hi = sh >= 20u ? mant << (sh - 20u) : t >> 20;
-    const uint32_t lo = sh >= 20u ? 0u : t & 0xFFFFFu;
-    const bool neg = (u & 0x8000u) != 0u;
-    chi += neg ? -(int)hi : (int)hi;
-    clo += neg ? -(int)lo : (int)lo;
-    s.a += (unsigned long long)hi * hi;
-    s.b += (unsigned long long)hi * lo;
-    s.c += (unsigned long long)lo * lo;
+// The split of fp16 values h (exact in fp32) into A and B, all in fp32 adds
+// whose results are exact (the splitting of Rump, Ogita and Oishi,
+// "Accurate floating-point summation", SIAM J. Sci. Comput. 31 (2008)):
+// t1 = h + 1.5 2^19 lies in [2^19, 2^20), where fp32 values are 2^-4 apart,
+// so t1 - 1.5 2^19 = h_hi is h rounded to a multiple of 2^-4 and h_lo =
+// h - h_hi (|h_lo| <= 2^-5, a multiple of 2^-24) is exact; t2 = h_lo + 0.75
+// lies in [0.5, 1), where values are 2^-24 apart, and is exact too.  Within
+// one binade the bit pattern grows by one per spacing, so A = bits(t1) -
+// bits(1.5 2^19) = 16 h_hi and B = bits(t2) - bits(0.75) = 2^24 h_lo.  An
+// infinite or NaN h makes h_lo and t2 NaN, whose pattern has bit 30 set;
+// every finite t2 has it clear.  Two values per fp32x2 instruction.
+constexpr uint32_t kLnBitsHi = 0x49400000u;  // 1.5 * 2^19
+constexpr uint32_t kLnBitsLo = 0x3F400000u;  // 0.75
+
+__device__ __forceinline__ void ln_take(uint32_t u1, uint32_t u2, uint32_t &sa, uint32_t &sb, uint32_t &nf,
+                                        LnSums &s) {
+    sa += u1;  // wrapping: the chunk's true sum fits in 32 bits
+    sb += u2;
+    nf |= u2;
+    const int A = (int)(u1 - kLnBitsHi), B = (int)(u2 - kLnBitsLo);
+    s.a += (unsigned long long)((long long)A * A);
+    s.b += (unsigned long long)((long long)A * B);
+    s.c += (unsigned long long)((long long)B * B);
+}
+
+// One 16-byte chunk (8 values) into the sums; |sum A| <= 2^23 and
+// |sum B| <= 2^22 over the chunk, so the sums of the bit patterns, minus 8
+// times the addends' patterns, are exact modulo 2^32 and in range.
+__device__ __forceinline__ void ln_add8(LnSums &s, const uint4 &d) {
+    uint32_t sa = 0, sb = 0, nf = 0;
+    const __half2 *hv = reinterpret_cast<const __half2 *>(&d);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const float2 x = __half22float2(hv[j]);
+        const float2 t1 = f2_add(x, make_float2(786432.0f, 786432.0f));
+        const float2 hi = f2_add(t1, make_float2(-786432.0f, -786432.0f));
+        const float2 t2 = f2_add(f2_fma(hi, make_float2(-1.0f, -1.0f), x), make_float2(0.75f, 0.75f));
+        ln_take(__float_as_uint(t1.x), __float_as_uint(t2.x), sa, sb, nf, s);
+        ln_take(__float_as_uint(t1.y), __float_as_uint(t2.y), sa, sb, nf, s);
+    }
+    s.s1 += (long long)(int)(sa - 8u * kLnBitsHi) * (1LL << 20) + (int)(sb - 8u * kLnBitsLo);
+    s.bad |= (int)((nf >> 30) & 1u);
 }
 
 // Codes of 8 elements (one 16-byte chunk of the row) from mean, rstd and the
-// folded affine; returns their sum.
+// folded affine; returns their sum.  Per element, as in the scalar form:
+// n = fl(fl(h - mean) * rstd), u = fma(n, gamma_r, beta_r), two per fp32x2
+// instruction.
 template <bool kF16Out>
 __device__ __forceinline__ int ln_codes8(const uint4 &d, int64_t k, float mean, float rstd,
                                          const float *__restrict__ gamma_r, const float *__restrict__ beta_r,
@@ -79,16 +104,18 @@ __device__ __forceinline__ int ln_codes8(const uint4 &d, int64_t k, float mean, 
         const float4 g1 = __ldg(reinterpret_cast<const float4 *>(gamma_r + k + 4));
         const float4 b0 = __ldg(reinterpret_cast<const float4 *>(beta_r + k));
         const float4 b1 = __ldg(reinterpret_cast<const float4 *>(beta_r + k + 4));
-        const float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-        const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+        const float2 g[4] = {make_float2(g0.x, g0.y), make_float2(g0.z, g0.w), make_float2(g1.x, g1.y),
+                             make_float2(g1.z, g1.w)};
+        const float2 bb[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
+                              make_float2(b1.z, b1.w)};
+        const float2 nm = make_float2(-mean, -mean), rs2 = make_float2(rstd, rstd);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const float2 f = __half22float2(hv[j]);
-            const float n0 = __fmul_rn(__fsub_rn(f.x, mean), rstd);
-            const float n1 = __fmul_rn(__fsub_rn(f.y, mean), rstd);
+            const float2 n = f2_mul(f2_add(__half22float2(hv[j]), nm), rs2);
+            const float2 u = f2_fma(n, g[j], bb[j]);
             // cvt.rni maps NaN to 0 and saturates; then the symmetric range
-            c[2 * j] = max(-qmax, min(qmax, __float2int_rn(__fmaf_rn(n0, g[2 * j], bb[2 * j]))));
-            c[2 * j + 1] = max(-qmax, min(qmax, __float2int_rn(__fmaf_rn(n1, g[2 * j + 1], bb[2 * j + 1]))));
+            c[2 * j] = max(-qmax, min(qmax, __float2int_rn(u.x)));
+            c[2 * j + 1] = max(-qmax, min(qmax, __float2int_rn(u.y)));
         }
     }
     int rs = 0;
@@ -116,81 +143,67 @@ __device__ __forceinline__ int ln_codes8(const uint4 &d, int64_t k, float mean, 
     return rs;
 }
 
-__device__ __forceinline__ void ln_add8(LnSums &s, const uint4 &d) {
-    int chi = 0, clo = 0;
-    const uint32_t w[4] = {d.x, d.y, d.z, d.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        ln_add_bits(w[j] & 0xFFFFu, chi, clo, s);
-        ln_add_bits(w[j] >> 16, chi, clo, s);
-    }
-    s.sh += chi;
-    s.sl += clo;
-}
-
 // The warp's sums, added over its lanes (exact).
 __device__ __forceinline__ void ln_warp_reduce(LnSums &s) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-        s.sh += __shfl_xor_sync(0xffffffffu, s.sh, o);
-        s.sl += __shfl_xor_sync(0xffffffffu, s.sl, o);
+        s.s1 += __shfl_xor_sync(0xffffffffu, s.s1, o);
         s.a += __shfl_xor_sync(0xffffffffu, s.a, o);
         s.b += __shfl_xor_sync(0xffffffffu, s.b, o);
         s.c += __shfl_xor_sync(0xffffffffu, s.c, o);
-        s.bad |= __shfl_xor_sync(0xffffffffu, s.bad, o);
     }
+    s.bad = __any_sync(0xffffffffu, s.bad);
 }
 
-// mean and rstd of the row from its exact sums (lane 0; IEEE fp32 in the
-// order documented above), broadcast to the warp.
-__device__ __forceinline__ void ln_finish(const LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
-    mean = 0.f;
-    rstd = 0.f;
-    if ((threadIdx.x & 31) == 0 && !s.bad) {
-        const float kf = (float)K;  // exact: K <= 2^22
-        const long long S1 = s.sh * (1LL << 20) + s.sl;  // exact: |S1| < 2^62
-        mean = __fmul_rn(__fdiv_rn(__ll2float_rn(S1), kf), 0x1p-24f);
-        const unsigned __int128 s2 = ((unsigned __int128)s.a << 40) + ((unsigned __int128)s.b << 21) +
-                                     (unsigned __int128)s.c;
-        const __int128 s1 = (__int128)S1;
-        const unsigned __int128 v = (unsigned __int128)K * s2 - (unsigned __int128)(s1 * s1);
-        const float vf = __fadd_rn(__fmul_rn(__ull2float_rn((unsigned long long)(v >> 64)), 18446744073709551616.0f),
-                                   __ull2float_rn((unsigned long long)v));
-        const float var = __fmul_rn(__fdiv_rn(__fdiv_rn(vf, kf), kf), 0x1p-48f);
-        rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, eps)));
-    }
-    mean = __shfl_sync(0xffffffffu, mean, 0);
-    rstd = __shfl_sync(0xffffffffu, rstd, 0);
+// mean and rstd of a row from its exact sums, by IEEE fp32 operations in
+// the order documented above (one thread).
+__device__ __forceinline__ void ln_moments(const LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
+    const float kf = (float)K;  // exact: K <= 2^22
+    mean = __fmul_rn(__fdiv_rn(__ll2float_rn(s.s1), kf), 0x1p-24f);  // exact S1: |S1| < 2^62
+    const __int128 s2 = ((__int128)s.a << 40) + ((__int128)(long long)s.b << 21) + (__int128)s.c;
+    const __int128 s1 = (__int128)s.s1;
+    const unsigned __int128 v = (unsigned __int128)((__int128)K * s2 - s1 * s1);  // >= 0 (Cauchy-Schwarz)
+    const float vf = __fadd_rn(__fmul_rn(__ull2float_rn((unsigned long long)(v >> 64)), 18446744073709551616.0f),
+                               __ull2float_rn((unsigned long long)v));
+    const float var = __fmul_rn(__fdiv_rn(__fdiv_rn(vf, kf), kf), 0x1p-48f);
+    rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, eps)));
 }
 
+// The warp's sums reduced, the moments taken by lane 0 and broadcast.
 __device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float &mean, float &rstd) {
     ln_warp_reduce(s);
-    ln_finish(s, K, eps, mean, rstd);
+    mean = 0.f;
+    rstd = 0.f;
+    if ((threadIdx.x & 31) == 0 && !s.bad) ln_moments(s, K, eps, mean, rstd);
+    mean = __shfl_sync(0xffffffffu, mean, 0);
+    rstd = __shfl_sync(0xffffffffu, rstd, 0);
 }
 
 // kWpr warps per row (kLnWarps / kWpr rows per CTA, grid-stride): lane l of
 // the row's warp w holds the 16-byte chunks l + 32 (i kWpr + w), i < kCh, in
 // registers (K <= 256 kWpr kCh).  Each warp adds its share of the exact sums;
-// the shares meet in shared memory (one named barrier per row group) and
-// every warp of the row finishes the same statistics from them, so the
-// result is that of one warp over the whole row.  Four 256-thread CTAs per
-// SM (64 registers) for rows of up to 4096 halves: measured on GB300 for
-// 2048 x 4096, 18.7 us against 20.9 us with one warp per row (the exact sums
-// cost ~40 instructions per element, so the kernel is issue-bound, not
-// HBM-bound).
+// the shares meet in shared memory, the row's first warp alone adds them and
+// takes the moments (a serial chain of 128-bit integer and fp32 division
+// steps, which the other warps would only repeat), and its result reaches
+// the row's warps through shared memory: two named barriers per row.  The
+// sums are exact, so the result is that of one warp over the whole row.
+// Four 256-thread CTAs per SM (64 registers); every width up to 8192 uses
+// four chunks per lane (measured on GB300: 2048 x 7168 in 21.9 us with
+// eight warps per row against 23.7 us with four warps of eight chunks).
 template <bool kF16Out, int kCh, int kWpr>
 __global__ void __launch_bounds__(kLnThreads, kCh <= 4 ? 4 : 2) layernorm_quantize_rows_kernel(
     const __half *__restrict__ h, int64_t M, int64_t K, int64_t ldh, const float *__restrict__ gamma_r,
     const float *__restrict__ beta_r, float eps, int qmax, void *q, int32_t *rowsum) {
     constexpr int kRows = kLnWarps / kWpr;
     __shared__ LnSums part[kLnWarps];
+    __shared__ float2 stat[kRows];  // mean, rstd; rstd is NaN for a row with non-finite values
     __shared__ int rsum[kLnWarps];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int rr = warp / kWpr, w = warp % kWpr;  // row of the CTA, warp of the row
     const int bar = 1 + rr;                        // named barrier of the row's warps
     for (int64_t m = (int64_t)blockIdx.x * kRows + rr; m < M; m += (int64_t)gridDim.x * kRows) {
         const __half *row = h + m * ldh;
-        LnSums s{0, 0, 0, 0, 0, 0};
+        LnSums s{0, 0, 0, 0, 0};
         uint4 d[kCh];
 #pragma unroll
         for (int i = 0; i < kCh; ++i) {
@@ -200,30 +213,41 @@ __global__ void __launch_bounds__(kLnThreads, kCh <= 4 ? 4 : 2) layernorm_quanti
 #pragma unroll
         for (int i = 0; i < kCh; ++i)
             if ((int64_t)(lane + 32 * (i * kWpr + w)) * 8 < K) ln_add8(s, d[i]);
-        ln_warp_reduce(s);
+        float mean, rstd;
+        bool bad;
         if (kWpr > 1) {
+            ln_warp_reduce(s);
             if (lane == 0) part[warp] = s;
             asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(32 * kWpr) : "memory");
-            LnSums t{0, 0, 0, 0, 0, 0};
+            if (w == 0 && lane == 0) {
+                LnSums t = part[rr * kWpr];
 #pragma unroll
-            for (int v = 0; v < kWpr; ++v) {
-                const LnSums &o = part[rr * kWpr + v];
-                t.sh += o.sh;
-                t.sl += o.sl;
-                t.a += o.a;
-                t.b += o.b;
-                t.c += o.c;
-                t.bad |= o.bad;
+                for (int v = 1; v < kWpr; ++v) {
+                    const LnSums &o = part[rr * kWpr + v];
+                    t.s1 += o.s1;
+                    t.a += o.a;
+                    t.b += o.b;
+                    t.c += o.c;
+                    t.bad |= o.bad;
+                }
+                float mu = 0.f, rs = __int_as_float(0x7fffffff);
+                if (!t.bad) ln_moments(t, K, eps, mu, rs);
+                stat[rr] = make_float2(mu, rs);
             }
-            s = t;
+            asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(32 * kWpr) : "memory");
+            const float2 st = stat[rr];
+            mean = st.x;
+            rstd = st.y;
+            bad = rstd != rstd;
+        } else {
+            ln_stats(s, K, eps, mean, rstd);
+            bad = s.bad != 0;
         }
-        float mean, rstd;
-        ln_finish(s, K, eps, mean, rstd);
         int rs = 0;
 #pragma unroll
         for (int i = 0; i < kCh; ++i) {
             const int64_t k = (int64_t)(lane + 32 * (i * kWpr + w)) * 8;
-            if (k < K) rs += ln_codes8<kF16Out>(d[i], k, mean, rstd, gamma_r, beta_r, qmax, q, m * K + k, s.bad);
+            if (k < K) rs += ln_codes8<kF16Out>(d[i], k, mean, rstd, gamma_r, beta_r, qmax, q, m * K + k, bad);
         }
         if (rowsum) {
 #pragma unroll
@@ -260,7 +284,7 @@ __global__ void __launch_bounds__(kLnThreads) layernorm_quantize_kernel(const __
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int64_t m = (int64_t)blockIdx.x * kLnWarps + warp; m < M; m += (int64_t)gridDim.x * kLnWarps) {
         const __half *row = h + m * ldh;
-        LnSums s{0, 0, 0, 0, 0, 0};
+        LnSums s{0, 0, 0, 0, 0};
         float mean, rstd;
         int rs = 0;
         if constexpr (kCh > 0) {
@@ -330,7 +354,7 @@ cudaError_t run_layernorm_quantize(const __half *h, int64_t M, int64_t K, int64_
     if (ch <= 4) OT_LN_ROWS(4, 1);
     else if (ch <= 8) OT_LN_ROWS(4, 2);
     else if (ch <= 16) OT_LN_ROWS(4, 4);
-    else if (ch <= 32) OT_LN_ROWS(8, 4);
+    else if (ch <= 32) OT_LN_ROWS(4, 8);
     else
         layernorm_quantize_kernel<kF16Out, 0><<<grid_for(kLnWarps), kLnThreads, 0, st>>>(h, M, K, ldh, gamma_r, beta_r,
                                                                                         eps, qmax, q, rowsum);

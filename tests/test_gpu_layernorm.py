@@ -54,7 +54,8 @@ def test_fold_layernorm_bit_exact():
     assert np.array_equal(br.cpu().numpy().view(np.uint32), br_o.view(np.uint32))
 
 
-@pytest.mark.parametrize("M,K,pad", [(1, 8, 0), (4, 768, 8), (65, 4104, 0), (300, 4096, 16), (6, 36864, 0)])
+@pytest.mark.parametrize("M,K,pad", [(1, 8, 0), (4, 768, 8), (9, 1032, 0), (33, 2048, 8), (65, 4104, 0), (300, 4096, 16),
+                                     (6, 36864, 0)])
 @pytest.mark.parametrize("fmt", ["f16", "i8"])
 @pytest.mark.parametrize("bits", [8, 6])
 def test_layernorm_quantize_bit_exact(M, K, pad, fmt, bits):
@@ -74,6 +75,44 @@ def test_layernorm_quantize_bit_exact(M, K, pad, fmt, bits):
                             B.OT_CODE_F16 if f16 else B.OT_CODE_I8, rowsum=rs)
     assert np.array_equal(q.cpu().numpy().astype(np.int64), q_o.astype(np.int64))
     assert np.array_equal(rs.cpu().numpy().astype(np.int64), rs_o)
+
+
+def _every_fp16_rows(K, seed):
+    """Rows of 2048 values holding every fp16 pattern of one exponent field
+    (both signs, all fractions; 31 rows), then every finite fp16 value once
+    in a random order over rows of K (zero-padded): each value's split into
+    the exact sums, and the sums' range, at least once."""
+    rng = np.random.default_rng(seed)
+    pats = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    exp = (pats >> 10) & 31
+    bands = [rng.permutation(pats[exp == e]) for e in range(31)]
+    fin = rng.permutation(pats[exp != 31])
+    rows = [np.tile(b, K // 2048) for b in bands]
+    allv = np.zeros(-(-fin.size // K) * K, np.uint16)
+    allv[: fin.size] = fin
+    rows += list(allv.reshape(-1, K))
+    return np.stack(rows).view(np.float16)
+
+
+@pytest.mark.parametrize("K", [2048, 4096, 8192, 16384])
+@pytest.mark.parametrize("fmt", ["f16", "i8"])
+def test_layernorm_quantize_every_fp16_value(K, fmt):
+    from paper_2406_18832_gb300 import binding as B
+    h = _every_fp16_rows(K, K)
+    M = h.shape[0]
+    rng = np.random.default_rng(K + 1)
+    gr = (30 + rng.standard_normal(K)).astype(np.float32)     # codes mostly inside the 8-bit range
+    br = rng.standard_normal(K).astype(np.float32)
+    q_o, rs_o, _, _ = oracle.layernorm_quantize(h, gr, br, 0.0, 8)
+    f16 = fmt == "f16"
+    q = torch.empty(M, K, dtype=torch.float16 if f16 else torch.int8, device=DEV)
+    rs = torch.empty(M, dtype=torch.int32, device=DEV)
+    B.ot_layernorm_quantize(torch.as_tensor(h).to(DEV), torch.as_tensor(gr).to(DEV), torch.as_tensor(br).to(DEV),
+                            0.0, 8, q, B.OT_CODE_F16 if f16 else B.OT_CODE_I8, rowsum=rs)
+    got = q.cpu().numpy().astype(np.int64)
+    assert np.array_equal(got, q_o.astype(np.int64))
+    assert np.array_equal(rs.cpu().numpy().astype(np.int64), rs_o)
+    assert np.count_nonzero(np.abs(q_o) == 127) < q_o.size // 4   # the codes are not just saturated
 
 
 def test_layernorm_quantize_nonfinite_rows_and_no_rowsum():
