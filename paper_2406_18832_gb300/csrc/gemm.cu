@@ -17,9 +17,7 @@
 // linear_kernel (one persistent CTA per SM, 16 warps):
 //   warp 0        TMA producer: per 64-wide k-block, the activation-code tile
 //                 (BN tokens x 64, fp16, 128-byte swizzle) and the weight tile
-//                 (128 rows x 64, int8, 64-byte swizzle) into an 8-stage ring;
-//                 two k-blocks of a piece that start at an even stage arrive
-//                 in one copy per operand (3-D views, K % 64 == 0).
+//                 (128 rows x 64, int8, 64-byte swizzle) into a 6-stage ring.
 //   warp 1        MMA issuer (one thread): D[128 x BN] += A[128 x 16] * B,
 //                 A read from tensor memory, B from shared memory.
 //   warp 2        allocates / frees the 512 TMEM columns.
@@ -52,7 +50,7 @@ namespace {
 
 constexpr int kBM = 128;        // weight rows per tile (TMEM lanes, MMA M)
 constexpr int kBK = 64;         // K elements per k-block (128 bytes of fp16)
-constexpr int kStages = 8;      // shared-memory ring and TMEM A buffers (even: slot pairs)
+constexpr int kStages = 6;      // shared-memory ring and TMEM A buffers
 constexpr int kThreads = 512;   // 16 warps
 constexpr int kWarpTma = 0, kWarpMma = 1, kWarpAlloc = 2, kWarpConv0 = 4, kWarpEpi0 = 8;
 constexpr int kNumEpiWarps = 8;
@@ -195,8 +193,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok,
                   const int32_t *__restrict__ zc, const int32_t *__restrict__ rowsum,
                   const float *__restrict__ zq, const float *__restrict__ rq, int qmax_out,
-                  int32_t *__restrict__ ws, int ws_pairs, const __grid_constant__ CUtensorMap tm_q3,
-                  const __grid_constant__ CUtensorMap tm_w3, int pair_copies) {
+                  int32_t *__restrict__ ws, int ws_pairs) {
     extern __shared__ uint8_t smem_raw[];
     Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
@@ -231,16 +228,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kWarpTma && lane == 0) {
         tma_prefetch_desc(&tm_q);
         tma_prefetch_desc(&tm_w);
-        if (pair_copies) {
-            tma_prefetch_desc(&tm_q3);
-            tma_prefetch_desc(&tm_w3);
-        }
     }
-    // A k-block is a "second" when it shares its predecessor's copy: it sits
-    // at an odd stage and its predecessor (at the even stage before it) is in
-    // the same piece.  The producer copies the two as one; the consumers wait
-    // for the first one's barrier only (the pair's data lands together).
-    auto second = [pair_copies](uint32_t it_, int kb_, int pk0_) { return pair_copies && (it_ & 1u) && kb_ > pk0_; };
     if (warp == kWarpAlloc) {
         tmem_alloc(smem_u32(&S.tmem_base), kTmemCols);
         tmem_relinquish();
@@ -268,28 +256,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             int u, pk0, pk1;
             sch.piece(p, u, pk0, pk1);
             const int m0 = (u % m_tiles) * BN, n0 = (u / m_tiles) * kBM;
-            for (int kb = pk0; kb < pk1;) {
+            for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 const int s = it % kStages;
                 const uint32_t ph = (it / kStages) & 1;
-                // stages s, s + 1 (same ring pass: kStages is even) for k-blocks kb, kb + 1
-                const bool two = pair_copies && (s & 1) == 0 && kb + 1 < pk1;
                 if (!(ok = mbar_wait_warp(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status))) break;
-                if (two && !(ok = mbar_wait_warp(smem_u32(&S.empty[s + 1]), ph ^ 1, abort, &g_status))) break;
                 if (elect_one()) {
-                    if (two) {
-                        mbar_arrive_expect_tx(smem_u32(&S.full[s]), 2 * kTxBytes);
-                        tma_load_3d(smem_u32(S.b[s]), &tm_q3, smem_u32(&S.full[s]), 0, m0, kb);
-                        tma_load_3d(smem_u32(S.w[s]), &tm_w3, smem_u32(&S.full[s]), 0, n0, kb);
-                        mbar_arrive(smem_u32(&S.full[s + 1]));  // keeps stage s + 1's phases in step
-                    } else {
-                        mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
-                        tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
-                        tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
-                    }
+                    mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
+                    tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
+                    tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
                 }
                 __syncwarp();
-                kb += two ? 2 : 1;
-                it += two ? 2 : 1;
             }
         }
         // teardown: every load issued must have landed before the CTA exits
@@ -315,8 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int kb = kb0; kb < kb1; ++kb, ++it) {
                     const int s = it % kStages;
                     const uint32_t ph = (it / kStages) & 1;
-                    if (!second(it, kb, pk0) && !(ok = mbar_wait_warp(smem_u32(&S.full[s]), ph, abort, &g_status)))
-                        break;
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
                     if (!(ok = mbar_wait_warp(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
                     tc_fence_after();
                     const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
@@ -353,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 const int s = it % kStages;
                 const uint32_t ph = (it / kStages) & 1;
-                if (!second(it, kb, pk0) && !(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
+                if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
                 uint4 raw[4];
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
@@ -1021,17 +996,6 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
         !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
                       kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
         return cudaErrorInvalidValue;
-    // The same operands as {64, rows, K / 64 k-blocks} views, a box of two
-    // k-blocks: the stage layout of two consecutive stages.  Only when the
-    // k-blocks tile K exactly (a view's k-block never reaches past a row).
-    CUtensorMap tm_q3 = tm_q, tm_w3 = tm_w;
-    const int pair_copies = a.K % kBK == 0 ? 1 : 0;
-    if (pair_copies &&
-        (!make_tmap_3d(&tm_q3, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, kBK, (uint64_t)a.M, (uint64_t)a.K / kBK,
-                       (uint64_t)a.K * 2, kBK * 2, kBK, BN, 2, CU_TENSOR_MAP_SWIZZLE_128B) ||
-         !make_tmap_3d(&tm_w3, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, kBK, (uint64_t)a.N, (uint64_t)a.K / kBK,
-                       (uint64_t)a.K, kBK, kBK, kBM, 2, CU_TENSOR_MAP_SWIZZLE_64B)))
-        return cudaErrorInvalidValue;
     // at least 120 KB so two CTAs never share an SM (each takes all 512 TMEM columns)
     const size_t smem = sizeof(Smem<BN>) + 1024 > 120 * 1024 ? sizeof(Smem<BN>) + 1024 : 120 * 1024;
     static std::once_flag once;
@@ -1057,7 +1021,7 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
     return launch_kernel(linear_kernel<BN, kS32, kAsym, kQOut>, dim3(grid), dim3(kThreads), smem, st, a.pdl, tm_q, tm_w,
                          a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
-                         a.rowsum, a.zq, a.rq, a.qmax_out, ws, pairs, tm_q3, tm_w3, pair_copies);
+                         a.rowsum, a.zq, a.rq, a.qmax_out, ws, pairs);
 }
 
 // Clusters of the pair kernel that fit on the device at once (one per two SMs).
