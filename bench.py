@@ -277,7 +277,7 @@ def run_ours(args):
     clocks = clk.summary()
     long_run = total_ms > 4000.0
     peak = peaks["bf16_sus"] if long_run else peaks["bf16"]
-    roofline = {"kernel": "linear_kernel (tcgen05 kind::f16, exact int8 codes)", "bound": "tensor",
+    roofline = {"kernel": "linear_pair_kernel (tcgen05 cta_group::2 kind::f16, exact int8 codes)", "bound": "tensor",
                 "achieved": round(gemm_tops, 1), "peak": peak, "unit": "TFLOP/s",
                 "frac": round(gemm_tops / peak, 4), "traffic": _traffic_record(),
                 "peak_source": f"{peaks['source']} bf16 dense {'sustained' if long_run else 'burst'} "
