@@ -66,6 +66,36 @@ def test_ln_fused_codes_dyadic_exact(a, c, eps):
     assert rs[0] == int(q[0].astype(np.int64).sum())
 
 
+def test_ln_statistics_every_fp16_value_exact_rational():
+    """Every fp16 bit pattern: one row per exponent field (all 2048 patterns of
+    that exponent, both signs), then every finite value once over rows of
+    4096.  The exact mean and biased variance of each row, in rationals from
+    the fp16 values themselves, bound the oracle's fp32 mean (2 roundings) and
+    1/sqrt(var + eps) (at most 7), from subnormals to 65504."""
+    rng = np.random.default_rng(5)
+    pats = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    exp = (pats >> 10) & 31
+    rows = [rng.permutation(pats[exp == e]) for e in range(31)]
+    fin = rng.permutation(pats[exp != 31])
+    allv = np.zeros(-(-fin.size // 4096) * 4096, np.uint16)
+    allv[: fin.size] = fin
+    h_bands = np.stack(rows).view(np.float16)
+    h_all = allv.reshape(-1, 4096).view(np.float16)
+    eps = np.float32(1e-5)
+    for h in (h_bands, h_all):
+        K = h.shape[1]
+        gr, br = oracle.fold_layernorm(np.ones(K, np.float16), np.zeros(K, np.float16), np.zeros(K, np.float32),
+                                       np.ones(K, np.float32))
+        _, _, mean, rstd = oracle.layernorm_quantize(h, gr, br, float(eps), 8)
+        for i in range(h.shape[0]):
+            vals = [Fraction(float(v)) for v in h[i].astype(np.float64)]
+            mu = sum(vals) / K
+            var = sum((v - mu) ** 2 for v in vals) / K
+            assert abs(Fraction(float(mean[i])) - mu) <= abs(mu) * Fraction(2, 2 ** 24) * Fraction(10001, 10000)
+            want = 1 / np.sqrt(float(var + Fraction(float(eps))))
+            assert abs(float(rstd[i]) - want) <= want * 7 * 2 ** -24
+
+
 def test_ln_fused_matches_unfused_away_from_ties():
     """The fused codes equal round((LN(h) - z) * r) computed in fp64 wherever
     the fp64 value is not within 1e-3 of a rounding boundary."""
