@@ -12,7 +12,7 @@
 // combined in 128 bits once per row.  Mean and 1/sqrt(var + eps) then follow
 // by a fixed sequence of IEEE fp32 operations (one lane per row) and the
 // codes by one fp32 fma per element.
-// Rows up to 8192 wide are held in registers by one to eight warps (one HBM
+// Rows up to 16384 wide are held in registers by one to eight warps (one HBM
 // read with the whole row in flight), longer ones are streamed by one warp
 // and read again from L2 for the codes.
 #include <cuda_fp16.h>
@@ -187,9 +187,12 @@ __device__ __forceinline__ void ln_stats(LnSums &s, int64_t K, float eps, float 
 // steps, which the other warps would only repeat), and its result reaches
 // the row's warps through shared memory: two named barriers per row.  The
 // sums are exact, so the result is that of one warp over the whole row.
-// Four 256-thread CTAs per SM (64 registers); every width up to 8192 uses
-// four chunks per lane (measured on GB300: 2048 x 7168 in 21.9 us with
-// eight warps per row against 23.7 us with four warps of eight chunks).
+// Four 256-thread CTAs per SM (64 registers) for every width up to 8192,
+// with four chunks per lane (measured on GB300: 2048 x 7168 in 21.9 us with
+// eight warps per row against 23.7 us with four warps of eight chunks); two
+// CTAs per SM with six or eight chunks per lane of eight warps up to 16384
+// (against the streaming kernel below: 4096 x 9216 62 vs 69 us, 2048 x 12288
+// 38 vs 41 us, 2048 x 16384 48 vs 58 us; 2048 x 9216 32 vs 31 us).
 template <bool kF16Out, int kCh, int kWpr>
 __global__ void __launch_bounds__(kLnThreads, kCh <= 4 ? 4 : 2) layernorm_quantize_rows_kernel(
     const __half *__restrict__ h, int64_t M, int64_t K, int64_t ldh, const float *__restrict__ gamma_r,
@@ -355,6 +358,8 @@ cudaError_t run_layernorm_quantize(const __half *h, int64_t M, int64_t K, int64_
     else if (ch <= 8) OT_LN_ROWS(4, 2);
     else if (ch <= 16) OT_LN_ROWS(4, 4);
     else if (ch <= 32) OT_LN_ROWS(4, 8);
+    else if (ch <= 48) OT_LN_ROWS(6, 8);
+    else if (ch <= 64) OT_LN_ROWS(8, 8);
     else
         layernorm_quantize_kernel<kF16Out, 0><<<grid_for(kLnWarps), kLnThreads, 0, st>>>(h, M, K, ldh, gamma_r, beta_r,
                                                                                         eps, qmax, q, rowsum);

@@ -55,7 +55,7 @@ def test_fold_layernorm_bit_exact():
 
 
 @pytest.mark.parametrize("M,K,pad", [(1, 8, 0), (4, 768, 8), (9, 1032, 0), (33, 2048, 8), (65, 4104, 0), (300, 4096, 16),
-                                     (6, 36864, 0)])
+                                     (7, 9224, 8), (12, 12288, 0), (5, 12296, 0), (6, 36864, 0)])
 @pytest.mark.parametrize("fmt", ["f16", "i8"])
 @pytest.mark.parametrize("bits", [8, 6])
 def test_layernorm_quantize_bit_exact(M, K, pad, fmt, bits):
@@ -94,7 +94,7 @@ def _every_fp16_rows(K, seed):
     return np.stack(rows).view(np.float16)
 
 
-@pytest.mark.parametrize("K", [2048, 4096, 8192, 16384])
+@pytest.mark.parametrize("K", [2048, 4096, 8192, 12288, 16384, 18432])
 @pytest.mark.parametrize("fmt", ["f16", "i8"])
 def test_layernorm_quantize_every_fp16_value(K, fmt):
     from paper_2406_18832_gb300 import binding as B
