@@ -136,6 +136,63 @@ def test_validation_rejects_bad_arguments_before_launch(lib):
     assert fz(A, 4, 64, 64, A, A, 8, A2, A, A, 16, 8, None, A, 16, 0, None, 0, None) == INV
 
 
+def test_validation_of_the_layernorm_calibration_and_per_token_entry_points(lib):
+    """Host-side checks of the remaining entry points, each rejected before any
+    CUDA call: LayerNorm fusion, token-wise clipping, per-token quantization."""
+    handle, _ = lib
+    INV, UNS = 1, 2
+    P, I64, I, S = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_size_t
+    F, D = ctypes.c_float, ctypes.c_double
+    handle.ot_layernorm_quantize.argtypes = [P, I64, I64, I64, P, P, F, I, P, I, P, P]
+    handle.ot_fold_layernorm.argtypes = [P, P, P, P, I64, P, P, P]
+    handle.ot_calibrate_clipped.argtypes = [P, I64, I64, I64, D, P, P, P]
+    handle.ot_quantize_tokens.argtypes = [P, I64, I64, I64, I, P, I, P, P]
+    handle.ot_quantize_weights.argtypes = [P, I64, I64, I, P, P, P]
+    handle.ot_linear_per_token.argtypes = [P, I64, I64, P, P, P, P, I64, I, I, P, I64, I, P, S, P]
+    handle.ot_derive_params.argtypes = [P, P, I64, I, I, P, P, P, P]
+    nan = float("nan")
+    ln = handle.ot_layernorm_quantize
+    assert ln(A, 4, 12, 12, A, A, 1e-5, 8, A2, 1, None, None) == INV            # K % 8
+    assert ln(A, 4, 64, 56, A, A, 1e-5, 8, A2, 1, None, None) == INV            # ldh < K
+    assert ln(A, 4, 64, 64, A, A, 1e-5, 8, A2, 7, None, None) == INV            # code format
+    assert ln(A, 4, 64, 64, A, A, nan, 8, A2, 1, None, None) == INV             # eps NaN
+    assert ln(A, 4, 64, 64, A, A, -1.0, 8, A2, 1, None, None) == INV            # eps < 0
+    assert ln(A, 4, 64, 64, None, A, 1e-5, 8, A2, 1, None, None) == INV         # gamma_r
+    assert ln(A + 8, 4, 64, 64, A, A, 1e-5, 8, A2, 1, None, None) == INV        # h alignment
+    assert ln(A, 4, 64, 64, A, A, 1e-5, 8, A2, 1, A + 2, None) == INV           # rowsum alignment
+    assert ln(A, 4, 64, 64, A, A, 1e-5, 1, A2, 1, None, None) == INV            # bits
+    big = (1 << 22) + 8
+    assert ln(A, 4, big, big, A, A, 1e-5, 8, A2, 1, None, None) == UNS          # exact 64-bit sums bound
+    fl = handle.ot_fold_layernorm
+    assert fl(A, A, A, A, 0, A, A, None) == INV
+    assert fl(None, A, A, A, 64, A, A, None) == INV
+    assert fl(A, A, A, A, 64, A + 2, A, None) == INV
+    assert fl(A, A, A, A, 1 << 31, A, A, None) == UNS
+    cc = handle.ot_calibrate_clipped
+    assert cc(A, 16, 64, 64, 0.0, A, A, None) == INV
+    assert cc(A, 16, 64, 64, 1.5, A, A, None) == INV
+    assert cc(A, 16, 64, 64, nan, A, A, None) == INV
+    assert cc(A, 16, 64, 64, 0.99, None, A, None) == INV
+    assert cc(A, 16, 64, 32, 0.99, A, A, None) == INV
+    assert cc(A, 1 << 31, 64, 64, 0.99, A, A, None) == UNS
+    qt = handle.ot_quantize_tokens
+    assert qt(A, 4, 64, 64, 8, A2, 7, A, None) == INV
+    assert qt(A, 4, 64, 64, 8, A2, 1, None, None) == INV
+    assert qt(A, 4, 12, 12, 8, A2, 1, A, None) == INV
+    assert qt(A, 1 << 31, 64, 64, 8, A2, 1, A, None) == UNS
+    qwf = handle.ot_quantize_weights
+    assert qwf(A, 16, 24, 8, A2, A, None) == INV
+    assert qwf(A, 16, 64, 8, A2, None, None) == INV
+    pt = handle.ot_linear_per_token
+    assert pt(A, 4, 64, A2, A, None, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV  # s_tok
+    assert pt(A, 4, 64, A2, A, A, None, 16, 8, 8, A, 16, 0, None, 0, None) == INV  # bias
+    assert pt(A, 4, 64, A2, A, A, A, 16, 8, 8, A, 8, 0, None, 0, None) == INV     # ldy < N
+    dp = handle.ot_derive_params
+    assert dp(A, A, 0, 8, 1, A, A, A, None) == INV
+    assert dp(A, A, 64, 8, 1, A, None, A, None) == INV
+    assert dp(A, A, 64, 1, 1, A, A, A, None) == INV
+
+
 def test_binding_refuses_host_tensors():
     import torch
     from paper_2406_18832_gb300 import binding
