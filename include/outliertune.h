@@ -15,7 +15,8 @@
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Work is enqueued asynchronously; outputs are valid once the
  *     stream has reached that point.  Nothing here synchronizes the stream
- *     except ot_get_device_status.
+ *     except ot_get_device_status and the first ot_linear_noalloc call on a
+ *     device.
  *   - Layouts are row-major.  X is [tokens, K] with row stride ldx elements,
  *     W is [N, K] (out x in, the nn.Linear layout that Eq. 6's W^T implies),
  *     Y is [M, N] with row stride ldy elements.
@@ -359,9 +360,10 @@ ot_status ot_linear_quantize_next(const void *q_f16, int64_t M, int64_t K, const
  * fixed 24 MiB array inside the library (a static device array that every
  * GPU loading the library holds until the process exits).  Nothing here
  * calls cudaMalloc, cudaFree or any allocating routine.
- *   - The first call on a device looks up the array's device address and
- *     zero-fills it on `stream`; make that first call before any stream
- *     capture.
+ *   - The first call on a device looks up the array's device address,
+ *     zero-fills it on `stream` and waits for that fill (it synchronizes
+ *     `stream` once); make that first call before any stream capture.  Later
+ *     calls, from any thread or stream, find the array already cleared.
  *   - Every call shares the array and it keeps the last call's contents, so
  *     calls that overlap on the GPU (on different streams, or from several
  *     threads) race and may corrupt each other's results: serialize them.

@@ -1154,8 +1154,10 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratch
 // Device address of g_noalloc_scratch on the current device.  In host code
 // the array's name is only a stand-in, so the address comes from
 // cudaGetSymbolAddress, once per device, with that device current; the first
-// use on a device also zero-fills the array on `st` (the stream-K flags and
-// epoch counters start at zero; the kernels keep them consistent after that).
+// use on a device also zero-fills the array (the stream-K flags and epoch
+// counters start at zero; the kernels keep them consistent after that) and
+// waits for the fill on `st`, so a call from another thread or stream that
+// finds the address cached never runs ahead of the fill.
 cudaError_t noalloc_scratch(void **ptr, cudaStream_t st) {
     static std::mutex mu;
     static void *addr[64] = {nullptr};
@@ -1169,6 +1171,8 @@ cudaError_t noalloc_scratch(void **ptr, cudaStream_t st) {
         e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
         if (e != cudaSuccess) return e;
         e = cudaMemsetAsync(p, 0, kNoAllocScratchBytes, st);
+        if (e != cudaSuccess) return e;
+        e = cudaStreamSynchronize(st);
         if (e != cudaSuccess) return e;
         addr[dev] = p;
     }
