@@ -29,6 +29,10 @@ and the token-wise clipping calibration of bias-free models (Appendix D):
   calibrate_clipped    - per-channel order statistics at quantile alpha
 and the epilogue that writes the next linear's codes (fc1 -> ReLU -> fc2):
   epilogue_quantize    - round((fma(acc, sw, b') [ReLU] - z') * r')
+Threaded drivers (calibrate_mt, fold_mt, quantize_mt, matmul_mt,
+epilogue_mt) run the same C functions on disjoint row or channel ranges in
+parallel host threads, for full-size parity checks and the timed CPU
+baseline; their results are identical to the single-threaded calls.
 """
 from __future__ import annotations
 
@@ -306,3 +310,90 @@ def epilogue_quantize(acc: np.ndarray, sw: np.ndarray, bfold: np.ndarray, z_next
     _load().oracle_epilogue_quantize(_ptr(acc), M, N, _ptr(_f32(sw)), _ptr(_f32(bfold)), 1 if relu else 0,
                                      _ptr(_f32(z_next)), _ptr(_f32(r_next)), bits_next, _ptr(q))
     return q
+
+
+# ---------------------------------------------------------------------------
+# Threaded drivers: the same C functions run on disjoint row (or channel)
+# ranges in parallel threads (ctypes releases the GIL during each call).
+# Every output element is computed by exactly the code above, so results are
+# identical to the single-threaded calls; only the wall time changes.
+# ---------------------------------------------------------------------------
+def host_threads() -> int:
+    """Cores this process may run on."""
+    return len(os.sched_getaffinity(0))
+
+
+def _ranges(n: int, parts: int):
+    parts = max(1, min(parts, n))
+    return [(n * i // parts, n * (i + 1) // parts) for i in range(parts)]
+
+
+def _run_parallel(fn, ranges, threads):
+    from concurrent.futures import ThreadPoolExecutor
+    if len(ranges) <= 1:
+        return [fn(*r) for r in ranges]
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        return list(ex.map(lambda r: fn(*r), ranges))
+
+
+def calibrate_mt(x: np.ndarray, mn: np.ndarray | None = None, mx: np.ndarray | None = None,
+                 threads: int | None = None):
+    """calibrate() with the channels split over threads (each channel's min /
+    max is one thread's sequential scan over the tokens, as in calibrate)."""
+    x = _f16(x)
+    T, K = x.shape
+    threads = threads or host_threads()
+    reset = mn is None
+    mn = np.empty(K, np.float32) if reset else _f32(mn).copy()
+    mx = np.empty(K, np.float32) if reset else _f32(mx).copy()
+    lib = _load()
+    base = x.ctypes.data
+
+    def part(k0, k1):
+        lib.oracle_calibrate(ctypes.c_void_p(base + 2 * k0), T, k1 - k0, K,
+                             ctypes.c_void_p(mn.ctypes.data + 4 * k0), ctypes.c_void_p(mx.ctypes.data + 4 * k0),
+                             1 if reset else 0)
+    _run_parallel(part, _ranges(K, 4 * threads), threads)
+    return mn, mx
+
+
+def fold_mt(w: np.ndarray, b: np.ndarray | None, z: np.ndarray, s: np.ndarray, bits_w: int,
+            threads: int | None = None):
+    """fold() with the output channels (rows of W) split over threads; every
+    row's codes, scale and folded bias depend on that row alone."""
+    w = _f16(w)
+    threads = threads or host_threads()
+    parts = _run_parallel(lambda n0, n1: fold(w[n0:n1], None if b is None else b[n0:n1], z, s, bits_w),
+                          _ranges(w.shape[0], 4 * threads), threads)
+    return tuple(np.concatenate([p[i] for p in parts]) for i in range(3))
+
+
+def quantize_mt(x: np.ndarray, z: np.ndarray, r: np.ndarray, bits_a: int, threads: int | None = None):
+    """quantize() with the tokens split over threads."""
+    x = _f16(x)
+    threads = threads or host_threads()
+    parts = _run_parallel(lambda m0, m1: quantize(x[m0:m1], z, r, bits_a), _ranges(x.shape[0], threads), threads)
+    return np.concatenate(parts) if parts else np.empty((0, x.shape[1]), np.int8)
+
+
+def matmul_mt(q: np.ndarray, qw: np.ndarray, threads: int | None = None) -> np.ndarray:
+    """matmul() with the tokens (or, for few tokens, the output channels) split
+    over threads; each accumulator is one thread's k-ascending int64 sum."""
+    q = np.ascontiguousarray(q, dtype=np.int8)
+    qw = np.ascontiguousarray(qw, dtype=np.int8)
+    threads = threads or host_threads()
+    M, N = q.shape[0], qw.shape[0]
+    if M >= threads:
+        parts = _run_parallel(lambda m0, m1: matmul(q[m0:m1], qw), _ranges(M, 4 * threads), threads)
+        return np.concatenate(parts)
+    parts = _run_parallel(lambda n0, n1: matmul(q, qw[n0:n1]), _ranges(N, 4 * threads), threads)
+    return np.concatenate(parts, axis=1)
+
+
+def epilogue_mt(acc: np.ndarray, sw: np.ndarray, bfold: np.ndarray, relu: bool = False,
+                threads: int | None = None) -> np.ndarray:
+    """epilogue() with the tokens split over threads."""
+    threads = threads or host_threads()
+    parts = _run_parallel(lambda m0, m1: epilogue(acc[m0:m1], sw, bfold, relu), _ranges(acc.shape[0], threads),
+                          threads)
+    return np.concatenate(parts)

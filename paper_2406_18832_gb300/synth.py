@@ -114,15 +114,13 @@ def outlier_params(cfg: int, li: int, layer: Layer, device="cpu"):
     return idx, mult, off
 
 
-def activations(cfg: int, li: int, layer: Layer, tokens: int, stream: int, device="cpu",
-                chunk: int = 8192):
-    """fp16 X[tokens, K]: N(0,1) (or ReLU'd exponential) with outlier channels.
-
-    stream 3 = calibration tokens, stream 4 = runtime tokens.
-    """
+def activation_chunks(cfg: int, li: int, layer: Layer, tokens: int, stream: int, device="cpu",
+                      chunk: int = 8192):
+    """The rows of activations(...) as consecutive fp16 blocks of `chunk`
+    tokens (the same values, drawn block by block from one generator), so a
+    large calibration set can be streamed without holding all of it."""
     idx, mult, off = outlier_params(cfg, li, layer, device)
     g = _gen(device, seed_of(cfg, li, stream))
-    out = torch.empty(tokens, layer.K, dtype=torch.float16, device=device)
     for t0 in range(0, tokens, chunk):
         t1 = min(tokens, t0 + chunk)
         if layer.post_relu:
@@ -134,7 +132,20 @@ def activations(cfg: int, li: int, layer: Layer, tokens: int, stream: int, devic
             base = torch.randn(t1 - t0, layer.K, generator=g, device=device)
         if idx.numel():
             base[:, idx] = base[:, idx] * mult + off
-        out[t0:t1] = base.to(torch.float16)
+        yield base.to(torch.float16)
+
+
+def activations(cfg: int, li: int, layer: Layer, tokens: int, stream: int, device="cpu",
+                chunk: int = 8192):
+    """fp16 X[tokens, K]: N(0,1) (or ReLU'd exponential) with outlier channels.
+
+    stream 3 = calibration tokens, stream 4 = runtime tokens.
+    """
+    out = torch.empty(tokens, layer.K, dtype=torch.float16, device=device)
+    t0 = 0
+    for blk in activation_chunks(cfg, li, layer, tokens, stream, device, chunk):
+        out[t0:t0 + blk.shape[0]] = blk
+        t0 += blk.shape[0]
     return out
 
 
