@@ -1,18 +1,23 @@
 """Benchmark of the per-channel quantized linear (OutlierTune, arXiv 2406.18832)
 on GB300.
 
-Workload: the four OPT-6.7B-shaped linears (QKV 4096->12288, out 4096->4096,
-fc1 4096->16384, fc2 16384->4096) at a prefill of 2048 tokens, W8A8, with
-synthetic LayerNorm-like activations carrying 0.5% fixed outlier channels.
-Offline per layer (not in the step, measured separately): calibration over
-65536 tokens and the weight fold.  One step = for every layer, the
-symmetrize+quantize kernel then the tcgen05 GEMM with its fused epilogue.
+Headline workload: the OPT-66B-shaped FFN linears (fc1 9216->36864, fc2
+36864->9216) at a prefill of 4096 tokens, W8A8, with synthetic LayerNorm-like
+activations carrying 1% fixed outlier channels (x U[30, 100], offsets
+U[-40, 40]).  Offline per layer (not in the step, measured separately):
+calibration over 65,536 tokens and the weight fold.  One step = for each of
+the two layers, the symmetrize+quantize kernel then the tcgen05 GEMM with its
+fused epilogue.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
 Prints one JSON line.  The value is exact int8 tera-operations per second
-(2*M*N*K per linear) over the whole step.  --impl reference times the CPU
-oracle on a bounded sample of the same workload on the host cores.
+(2*M*N*K per linear) over the whole step.  Beside it: the OPT-6.7B step at
+2048 tokens, the OPT-30B block, decode-sized and swept token counts (each
+against cuBLAS fp16 of the same shapes), the fused LayerNorm, the per-token
+path, asymmetric weights and the clipping calibration.  --impl reference
+times the CPU oracle on a bounded sample of the headline workload on the host
+cores.
 """
 from __future__ import annotations
 
@@ -29,9 +34,11 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-WORKLOAD_CFG = 2          # OPT-6.7B-shaped linears
-TOKENS = 2048
+WORKLOAD_CFG = 4          # OPT-66B-shaped fc1 / fc2
+WORKLOAD_NAME = "opt-66b-ffn-prefill-4096"
+TOKENS = 4096
 BITS = (8, 8)
+STEP6_CFG, STEP6_TOKENS = 2, 2048   # the OPT-6.7B step beside the headline
 METRIC = "W8A8 linear TOPS & % INT8 peak; quantize GB/s % HBM; vs cuBLAS FP16"
 L2_BYTES = 129 * 2 ** 20
 
@@ -51,9 +58,9 @@ def _env_rank():
         int(os.environ.get("LOCAL_RANK", "0"))
 
 
-def _workload_desc():
+def _workload_desc(cfg: int = WORKLOAD_CFG):
     from paper_2406_18832_gb300 import synth
-    c = synth.CONFIGS[WORKLOAD_CFG]
+    c = synth.CONFIGS[cfg]
     return c, [(l.name, l.K, l.N) for l in c.layers]
 
 
@@ -135,9 +142,10 @@ class ClockSampler:
 
 
 def _traffic_record():
-    """DRAM bytes per GEMM launch from the committed ncu summary, if the GEMM
-    source is unchanged since it was captured (else None)."""
-    path = os.path.join(ROOT, "profiles", "linear_kernel_traffic.txt")
+    """DRAM bytes per GEMM launch of the headline workload from the committed
+    ncu summary, if the GEMM source is unchanged since it was captured and the
+    summary is of this workload (else None)."""
+    path = os.path.join(ROOT, "profiles", "linear_pair_kernel_traffic_opt66b_ffn_m4096.txt")
     src = os.path.join(ROOT, "paper_2406_18832_gb300", "csrc", "gemm.cu")
     try:
         sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
@@ -147,7 +155,7 @@ def _traffic_record():
             if "=" in line and not line.startswith("#"):
                 k, v = line.split("=", 1)
                 vals[k.strip()] = v.strip()
-        if vals.get("gemm_cu_sha256_16") != sha:
+        if vals.get("gemm_cu_sha256_16") != sha or vals.get("workload") != WORKLOAD_NAME:
             return None
         return float(vals["dram_bytes_per_launch"])
     except Exception:
@@ -157,30 +165,20 @@ def _traffic_record():
 # ----------------------------------------------------------------------------
 # the CUDA path
 # ----------------------------------------------------------------------------
-def run_ours(args):
+def _build_layers(dev, cfg_index, tokens, bits, t_cal=None):
+    """Calibrated and folded QuantizedLinear per layer of a config, with its
+    runtime activations; calibration and fold are timed (offline steps)."""
     import torch
-    import torch.distributed as dist
 
-    from paper_2406_18832_gb300 import QuantizedLinear, binding, synth
-
-    rank, world, local = _env_rank()
-    if world > 1:
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    binding.load()
-    peaks = _peaks()
-    cfg, layer_shapes = _workload_desc()
-    bits_a, bits_w = BITS
-
-    # ---- offline: inputs, calibration, fold (each rank its own replica) ----
+    from paper_2406_18832_gb300 import QuantizedLinear, synth
+    cfg = synth.CONFIGS[cfg_index]
+    bits_a, bits_w = bits
     layers, xs = [], []
     calib_ms, calib_bytes, fold_ms = [], 0, []
     for li, layer in enumerate(cfg.layers):
-        w, b = synth.weights(WORKLOAD_CFG, li, layer, device=dev)
-        t_cal = 8192 if args.profile else cfg.T_cal
-        xc = synth.activations(WORKLOAD_CFG, li, layer, t_cal, 3, device=dev)
-        x = synth.activations(WORKLOAD_CFG, li, layer, TOKENS, 4, device=dev)
+        w, b = synth.weights(cfg_index, li, layer, device=dev)
+        xc = synth.activations(cfg_index, li, layer, t_cal or cfg.T_cal, 3, device=dev)
+        x = synth.activations(cfg_index, li, layer, tokens, 4, device=dev)
         ql = QuantizedLinear(layer.K, layer.N, bits_a, bits_w, relu=layer.relu_out, device=dev)
         # calibration: warm once, then time one pass over the calibration tokens
         ql.calibrate(xc)
@@ -202,21 +200,89 @@ def run_ours(args):
         layers.append((ql, w, b))
         xs.append(x)
     torch.cuda.empty_cache()
+    return layers, xs, calib_ms, calib_bytes, fold_ms
+
+
+def _timed_steps(layers, xs, qbufs, ybufs, steps, stream):
+    """Run `steps` steps (quantize then linear per layer) with CUDA events
+    around every launch; returns total ms and per-layer lists of GEMM and
+    quantize ms."""
+    import torch
+    nl = len(layers)
+    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(nl)] for _ in range(steps)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for k in range(steps):
+        for i, (ql, _, _) in enumerate(layers):
+            events[k][i][0].record(stream)
+            ql.quantize(xs[i], qbufs[i])
+            events[k][i][1].record(stream)
+            ql.linear(qbufs[i], ybufs[i])
+            events[k][i][2].record(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    gemm_ms = [[events[k][i][1].elapsed_time(events[k][i][2]) for k in range(steps)] for i in range(nl)]
+    quant_ms = [[events[k][i][0].elapsed_time(events[k][i][1]) for k in range(steps)] for i in range(nl)]
+    return t0.elapsed_time(t1), gemm_ms, quant_ms
+
+
+def _cublas_ms(xs, ws, ybufs, reps):
+    """cuBLAS fp16 GEMM (torch.matmul) of each layer's shape, ms per call."""
+    import torch
+    out = []
+    for x, w, y in zip(xs, ws, ybufs):
+        def f():
+            torch.matmul(x, w.t(), out=y)
+        for _ in range(3):
+            f()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            f()
+        e1.record()
+        torch.cuda.synchronize()
+        out.append(e0.elapsed_time(e1) / reps)
+    return out
+
+
+def _quant_stats(layer_shapes, tokens, quant_ms, steps):
+    """Quantize throughput on the algorithmic bytes (fp16 X in, int8 codes
+    out, z and r) and on the bytes the kernel moves (fp16 codes out)."""
+    alg = sum(3 * tokens * K + 8 * K for _, K, _ in layer_shapes)
+    moved = sum(4 * tokens * K + 8 * K for _, K, _ in layer_shapes)
+    t = sum(sum(v) for v in quant_ms) / steps
+    return alg, moved, t
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2406_18832_gb300 import binding
+
+    rank, world, local = _env_rank()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    binding.load()
+    peaks = _peaks()
+    cfg, layer_shapes = _workload_desc()
+    bits_a, bits_w = BITS
+
+    # ---- offline: inputs, calibration, fold (each rank its own replica) ----
+    layers, xs, calib_ms, calib_bytes, fold_ms = _build_layers(dev, WORKLOAD_CFG, TOKENS, BITS,
+                                                               8192 if args.profile else None)
     qbufs = [torch.empty(TOKENS, l.K, dtype=torch.float16, device=dev) for l in cfg.layers]
     ybufs = [torch.empty(TOKENS, l.N, dtype=torch.float16, device=dev) for l in cfg.layers]
     ops_step = _ops_per_step(layer_shapes, TOKENS)
     stream = torch.cuda.current_stream()
 
-    def step(evs=None):
+    def step():
         for i, (ql, _, _) in enumerate(layers):
-            if evs is not None:
-                evs[i][0].record(stream)
             ql.quantize(xs[i], qbufs[i])
-            if evs is not None:
-                evs[i][1].record(stream)
             ql.linear(qbufs[i], ybufs[i])
-            if evs is not None:
-                evs[i][2].record(stream)
 
     for _ in range(args.warmup):
         step()
@@ -237,24 +303,13 @@ def run_ours(args):
             print(json.dumps({"profile_run": True, "steps": args.steps}), flush=True)
         return
 
-    nl = len(layers)
-    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(nl)]
-              for _ in range(args.steps)]
-    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(torch.cuda.current_device() if world == 1 else local) as clk:
-        t0.record(stream)
-        for k in range(args.steps):
-            step(events[k])
-        t1.record(stream)
-        torch.cuda.synchronize()
+        total_ms, gemm_ms, quant_ms = _timed_steps(layers, xs, qbufs, ybufs, args.steps, stream)
     if world > 1:
         dist.barrier()
-    total_ms = t0.elapsed_time(t1)
-    gemm_ms = [[events[k][i][1].elapsed_time(events[k][i][2]) for k in range(args.steps)] for i in range(nl)]
-    quant_ms = [[events[k][i][0].elapsed_time(events[k][i][1]) for k in range(args.steps)] for i in range(nl)]
     total_ms = max_over_ranks(total_ms, dev)
     ms_per_step = total_ms / args.steps
     value = job_value(ops_step, world, args.steps, total_ms)
@@ -263,17 +318,20 @@ def run_ours(args):
     gemm_ops = [2 * TOKENS * K * N for _, K, N in layer_shapes]
     gemm_time = sum(sum(v) for v in gemm_ms)
     gemm_tops = sum(o * args.steps for o in gemm_ops) / (gemm_time * 1e-3) / 1e12
+    cub = _cublas_ms(xs, [w for _, w, _ in layers], ybufs, max(5, min(50, args.steps)))
     per_layer = []
     for i, (name, K, N) in enumerate(layer_shapes):
         g = statistics.median(gemm_ms[i])
         q = statistics.median(quant_ms[i])
-        qbytes = TOKENS * K * 4 + 8 * K
         per_layer.append({"layer": name, "K": K, "N": N, "gemm_us": round(g * 1e3, 2),
                           "gemm_tops": round(gemm_ops[i] / (g * 1e-3) / 1e12, 1),
-                          "quant_us": round(q * 1e3, 2), "quant_gbs": round(qbytes / (q * 1e-3) / 1e9, 1)})
-    qbytes_total = sum(TOKENS * K * 4 + 8 * K for _, K, _ in layer_shapes)
-    quant_time = sum(sum(v) for v in quant_ms) / args.steps
-    quant_gbs = qbytes_total / (quant_time * 1e-3) / 1e9
+                          "gemm_frac_peak": round(gemm_ops[i] / (g * 1e-3) / 1e12 / peaks["bf16"], 4),
+                          "cublas_fp16_us": round(cub[i] * 1e3, 2),
+                          "cublas_fp16_tflops": round(gemm_ops[i] / (cub[i] * 1e-3) / 1e12, 1),
+                          "quant_us": round(q * 1e3, 2),
+                          "quant_gbs_algorithmic": round((3 * TOKENS * K + 8 * K) / (q * 1e-3) / 1e9, 1),
+                          "quant_gbs_moved": round((4 * TOKENS * K + 8 * K) / (q * 1e-3) / 1e9, 1)})
+    q_alg, q_moved, quant_time = _quant_stats(layer_shapes, TOKENS, quant_ms, args.steps)
     clocks = clk.summary()
     long_run = total_ms > 4000.0
     peak = peaks["bf16_sus"] if long_run else peaks["bf16"]
@@ -281,25 +339,9 @@ def run_ours(args):
                 "achieved": round(gemm_tops, 1), "peak": peak, "unit": "TFLOP/s",
                 "frac": round(gemm_tops / peak, 4), "traffic": _traffic_record(),
                 "peak_source": f"{peaks['source']} bf16 dense {'sustained' if long_run else 'burst'} "
-                               "(fp16 dense runs at the bf16 rate)"}
+                               "(fp16 dense runs at the bf16 rate)",
+                "algorithmic": "2 M N K ops per launch (M = 4096; fc1 and fc2: 2.78 T each)"}
 
-    # ---- comparators: cuBLAS fp16 GEMM of the same shapes, cuBLASLt int8 ----
-    reps = max(10, min(200, args.steps))
-    cub = []
-    for i, (ql, w, b) in enumerate(layers):
-        def f():
-            torch.matmul(xs[i], w.t(), out=ybufs[i])
-        for _ in range(3):
-            f()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for _ in range(reps):
-            f()
-        e1.record()
-        torch.cuda.synchronize()
-        cub.append(e0.elapsed_time(e1) / reps)
-    cub_step_ms = sum(cub)
     int8_tops = None
     try:
         _, K0, N0 = layer_shapes[0]
@@ -310,23 +352,110 @@ def run_ours(args):
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
-        for _ in range(5):
+        for _ in range(3):
             torch._int_mm(a8, b8)
         e1.record()
         torch.cuda.synchronize()
-        int8_tops = 2 * TOKENS * K0 * N0 / (e0.elapsed_time(e1) / 5 * 1e-3) / 1e12
+        int8_tops = 2 * TOKENS * K0 * N0 / (e0.elapsed_time(e1) / 3 * 1e-3) / 1e12
         del a8, b8
     except Exception:
         int8_tops = None
 
     # ---- end to end through the public API, host buffers in and out ----
-    e2e_steps = max(3, min(100, args.steps))
+    e2e_steps = max(3, min(50, args.steps))
+    e2e_ms, h2d, d2h = _e2e(layers, xs, qbufs, ybufs, e2e_steps)
+
+    # ---- host copies for the CPU oracle baseline (rank 0, one replica) ----
+    host = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        host = [dict(w=w.cpu().numpy(), b=b.cpu().numpy(), x=x[:1024].cpu().numpy(), relu=ql.relu,
+                     xc=None) for (ql, w, b), x in zip(layers, xs)]
+        from paper_2406_18832_gb300 import synth
+        for li, layer in enumerate(cfg.layers):
+            host[li]["xc"] = synth.activations(WORKLOAD_CFG, li, layer, 8192, 3, device=dev).cpu().numpy()
+
+    weights_fp16 = sum(2 * K * N for _, K, N in layer_shapes)
+    weights_int8 = sum(ql.weight_bytes() for ql, _, _ in layers)
+    del layers, xs, qbufs, ybufs
+    torch.cuda.empty_cache()
+
+    step6 = bench_step6(dev, peaks, max(5, min(200, args.steps)), args.warmup)
+    block = None if args.no_block else bench_block(dev)
+    decode = bench_decode(dev, peaks)
+    lnq = bench_layernorm(dev, peaks)
+    qsweep = bench_quantize_sweep(dev, peaks)
+    sweep = bench_token_sweep(dev, peaks)
+    per_tok = bench_per_token(dev, peaks)
+    clip = bench_clipping(dev, peaks, step6.pop("_calib_ms0"))
+
+    cpu = None
+    if host is not None:
+        cpu = cpu_baseline(host, budget_s=args.cpu_budget)
+
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "int8 codes exact on the f16 tensor pipe (fp32 chunk sums, int32 totals)",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_NAME, "tokens": TOKENS, "bits_a": bits_a, "bits_w": bits_w,
+                   "layers": [{"name": n, "K": K, "N": N} for n, K, N in layer_shapes],
+                   "calibration_tokens": cfg.T_cal, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2: one step streams 680 MB of int8 weights and 1.3 GB of "
+                         "activations, codes and outputs through the 129 MB L2"},
+        "roofline": roofline,
+        "gpu_launches": args.steps * 2 * len(layer_shapes),
+        "e2e": {"value": round(ops_step / (e2e_ms * 1e-3) / 1e12 * world, 2), "unit": "TOPS",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
+                "copies": "pinned host buffers; host->device, layers and device->host on three streams"},
+        "clocks": clocks,
+        "quantize": {"gbs_algorithmic": round(q_alg / (quant_time * 1e-3) / 1e9, 1),
+                     "frac_algorithmic": round(q_alg / (quant_time * 1e-3) / 1e9 / peaks["hbm"], 4),
+                     "gbs_moved": round(q_moved / (quant_time * 1e-3) / 1e9, 1),
+                     "frac_moved": round(q_moved / (quant_time * 1e-3) / 1e9 / peaks["hbm"], 4),
+                     "hbm_peak_gbs": peaks["hbm"], "bytes_algorithmic_per_step": q_alg,
+                     "bytes_moved_per_step": q_moved,
+                     "note": "algorithmic: fp16 X in + int8 codes out + z, r; moved: the fp16 codes the "
+                             "prefill GEMM reads", "sweep": qsweep},
+        "calibrate": {"gbs": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9, 1),
+                      "frac": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9 / peaks["hbm"], 4),
+                      "tokens": cfg.T_cal, "ms_per_layer": [round(v, 3) for v in calib_ms]},
+        "fold_ms_per_layer": [round(v, 3) for v in fold_ms],
+        "cublas_fp16": {"ms_per_step": round(sum(cub), 4),
+                        "tflops": round(ops_step / (sum(cub) * 1e-3) / 1e12, 1),
+                        "ours_over_cublas": round(sum(cub) / ms_per_step, 4),
+                        "gemm_only_over_cublas": round(sum(cub) / (gemm_time / args.steps), 4)},
+        "int8_peak": {"cublaslt_int8_tops": None if int8_tops is None else round(int8_tops, 1),
+                      "frac_of_cublaslt_int8": None if not int8_tops else round(gemm_tops / int8_tops, 2),
+                      "note": "GB300 (sm_103a) has no tcgen05 int8 MMA; cuBLASLt int8 (torch._int_mm) of the "
+                              "fc1 shape, measured in this run"},
+        "per_layer": per_layer,
+        "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
+                   "ratio": round(weights_fp16 / weights_int8, 3)},
+        "opt67b_step": step6,
+        "block": block,
+        "decode": decode,
+        "token_sweep": sweep,
+        "per_token": per_tok,
+        "layernorm_quantize": lnq,
+        "clipping_calibration": clip,
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _e2e(layers, xs, qbufs, ybufs, steps):
+    """ms per step through the public API (QuantizedLinear.forward) with the
+    inputs copied in from pinned host memory and the outputs copied back: the
+    copies run on their own streams, so a layer's input copy overlaps the
+    previous layer and its output copy the next."""
+    import torch
     hx = [x.cpu().pin_memory() for x in xs]
     hy = [torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in ybufs]
     dx = [torch.empty_like(x) for x in xs]
-
-    # three streams: host->device copies, the layers, device->host copies; a
-    # layer's input copy overlaps the previous layer, its output copy the next
     s_c = torch.cuda.current_stream()
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
     ev_in = [torch.cuda.Event() for _ in layers]
@@ -352,79 +481,50 @@ def run_ours(args):
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    for _ in range(e2e_steps):
+    for _ in range(steps):
         e2e_step()
     s_c.wait_stream(s_in)
     s_c.wait_stream(s_out)
     e1.record()
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
     h2d = sum(x.numel() * 2 for x in xs)
     d2h = sum(y.numel() * 2 for y in ybufs)
+    return e0.elapsed_time(e1) / steps, h2d, d2h
 
-    block = None if args.no_block else bench_block(dev)
-    decode = bench_decode(dev, peaks)
-    asym = bench_asym(dev, layers, xs, ops_step, ms_per_step)
-    lnq = bench_layernorm(dev, peaks)
-    qsweep = bench_quantize_sweep(dev, peaks)
-    large = bench_large_gemm(dev, peaks)
-    sweep = bench_token_sweep(dev, peaks)
-    clip = bench_clipping(dev, peaks, calib_ms, calib_bytes)
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(budget_s=args.cpu_budget, layers=layers)
-
-    weights_fp16 = sum(2 * K * N for _, K, N in layer_shapes)
-    weights_int8 = sum(ql.weight_bytes() for ql, _, _ in layers)
-    line = {
-        "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None,
-        "dtype": "int8 codes exact on the f16 tensor pipe (fp32 chunk sums, int32 totals)",
-        "data": "synthetic",
-        "config": {"workload": "opt-6.7b-linears-prefill", "tokens": TOKENS, "bits_a": bits_a, "bits_w": bits_w,
-                   "layers": [{"name": n, "K": K, "N": N} for n, K, N in layer_shapes],
-                   "calibration_tokens": cfg.T_cal, "parallelism": f"replicas x{world}",
-                   "l2": "inputs larger than L2: one step streams 201 MB of int8 weights and 470 MB of "
-                         "activations and outputs through the 129 MB L2"},
-        "roofline": roofline,
-        "gpu_launches": args.steps * 2 * len(layers),
-        "e2e": {"value": round(ops_step / (e2e_ms * 1e-3) / 1e12 * world, 2), "unit": "TOPS",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
-                "copies": "pinned host buffers; host->device, layers and device->host on three streams"},
-        "clocks": clocks,
-        "quantize": {"gbs": round(quant_gbs, 1), "hbm_peak_gbs": peaks["hbm"],
-                     "frac": round(quant_gbs / peaks["hbm"], 4),
-                     "bytes_per_step": qbytes_total, "note": "fp16 X in + fp16 codes out + z, r",
-                     "sweep": qsweep},
-        "calibrate": {"gbs": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9, 1),
-                      "frac": round(calib_bytes / (sum(calib_ms) * 1e-3) / 1e9 / peaks["hbm"], 4),
-                      "tokens": cfg.T_cal, "ms_per_layer": [round(v, 3) for v in calib_ms]},
-        "fold_ms_per_layer": [round(v, 3) for v in fold_ms],
-        "cublas_fp16": {"ms_per_step": round(cub_step_ms, 4),
-                        "tflops": round(ops_step / (cub_step_ms * 1e-3) / 1e12, 1),
-                        "ours_over_cublas": round(cub_step_ms / ms_per_step, 4)},
-        "int8_peak": {"cublaslt_int8_tops": None if int8_tops is None else round(int8_tops, 1),
-                      "frac_of_cublaslt_int8": None if not int8_tops else round(gemm_tops / int8_tops, 2),
-                      "note": "GB300 has no tcgen05 int8 MMA; cuBLASLt int8 (torch._int_mm) of the QKV shape, "
-                              "measured in this run"},
-        "per_layer": per_layer,
-        "large_gemm": large,
-        "token_sweep": sweep,
-        "memory": {"weights_fp16_bytes": weights_fp16, "weights_int8_bytes": weights_int8,
-                   "ratio": round(weights_fp16 / weights_int8, 3)},
-        "block": block,
-        "decode": decode,
-        "asym_weights": asym,
-        "layernorm_quantize": lnq,
-        "clipping_calibration": clip,
-        "cpu_baseline": cpu,
-    }
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+def bench_step6(dev, peaks, steps, warmup):
+    """The OPT-6.7B step (QKV, out, fc1, fc2 at 2048 tokens, W8A8): quantize
+    then linear per layer, as the headline; with the same step on the paper's
+    "Int8" weights (per-output-channel zero points) beside it."""
+    import torch
+    cfg, shapes = _workload_desc(STEP6_CFG)
+    layers, xs, calib_ms, calib_bytes, _ = _build_layers(dev, STEP6_CFG, STEP6_TOKENS, BITS)
+    qbufs = [torch.empty(STEP6_TOKENS, l.K, dtype=torch.float16, device=dev) for l in cfg.layers]
+    ybufs = [torch.empty(STEP6_TOKENS, l.N, dtype=torch.float16, device=dev) for l in cfg.layers]
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        for i, (ql, _, _) in enumerate(layers):
+            ql.forward(xs[i], qbufs[i], ybufs[i])
+    torch.cuda.synchronize()
+    total_ms, gemm_ms, quant_ms = _timed_steps(layers, xs, qbufs, ybufs, steps, stream)
+    ops_step = _ops_per_step(shapes, STEP6_TOKENS)
+    ms = total_ms / steps
+    gemm_ops = [2 * STEP6_TOKENS * K * N for _, K, N in shapes]
+    gemm_tops = sum(o * steps for o in gemm_ops) / (sum(sum(v) for v in gemm_ms) * 1e-3) / 1e12
+    cub = _cublas_ms(xs, [w for _, w, _ in layers], ybufs, 50)
+    q_alg, q_moved, qt = _quant_stats(shapes, STEP6_TOKENS, quant_ms, steps)
+    asym = bench_asym(dev, layers, xs, ops_step, ms)
+    out = {"workload": "opt-6.7b-linears-prefill-2048", "tokens": STEP6_TOKENS, "ms_per_step": round(ms, 4),
+           "tops": round(ops_step / (ms * 1e-3) / 1e12, 1), "gemm_tflops": round(gemm_tops, 1),
+           "gemm_frac_peak": round(gemm_tops / peaks["bf16"], 4),
+           "per_layer_gemm_us": [round(statistics.median(v) * 1e3, 2) for v in gemm_ms],
+           "quantize_gbs_algorithmic": round(q_alg / (qt * 1e-3) / 1e9, 1),
+           "cublas_fp16_ms_per_step": round(sum(cub), 4),
+           "ours_over_cublas": round(sum(cub) / ms, 4), "asym_weights": asym,
+           "_calib_ms0": (calib_ms[0], STEP6_CFG)}
+    del layers, xs, qbufs, ybufs
+    torch.cuda.empty_cache()
+    return out
 
 
 def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 8192):
@@ -435,16 +535,16 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
     import torch
 
     from paper_2406_18832_gb300 import QuantizedLinear, synth
-    cfg = synth.CONFIGS[WORKLOAD_CFG]
+    cfg = synth.CONFIGS[STEP6_CFG]
     qls = []
     for li, (layer, (ql_sym, w, b)) in enumerate(zip(cfg.layers, layers)):
         ql = QuantizedLinear(layer.K, layer.N, ql_sym.bits_a, ql_sym.bits_w, relu=layer.relu_out, device=dev,
                              weights="asym")
-        ql.calibrate(synth.activations(WORKLOAD_CFG, li, layer, t_cal, 3, device=dev)).fold(w, b)
+        ql.calibrate(synth.activations(STEP6_CFG, li, layer, t_cal, 3, device=dev)).fold(w, b)
         qls.append(ql)
-    qb = [torch.empty(TOKENS, ql.K, dtype=torch.float16, device=dev) for ql in qls]
-    rb = [torch.empty(TOKENS, dtype=torch.int32, device=dev) for _ in qls]
-    yb = [torch.empty(TOKENS, ql.N, dtype=torch.float16, device=dev) for ql in qls]
+    qb = [torch.empty(STEP6_TOKENS, ql.K, dtype=torch.float16, device=dev) for ql in qls]
+    rb = [torch.empty(STEP6_TOKENS, dtype=torch.int32, device=dev) for _ in qls]
+    yb = [torch.empty(STEP6_TOKENS, ql.N, dtype=torch.float16, device=dev) for ql in qls]
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in qls]
     gemm_ms = [0.0] * len(qls)
 
@@ -474,7 +574,7 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
         torch.cuda.synchronize()
         for i in range(len(qls)):
             gemm_ms[i] += evs[i][1].elapsed_time(evs[i][2]) / 20
-    return {"workload": "opt-6.7b-linears-prefill, Int8 weights with zero points", "tokens": TOKENS,
+    return {"workload": "opt-6.7b-linears-prefill, Int8 weights with zero points", "tokens": STEP6_TOKENS,
             "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
             "over_symmetric_step": round(ms / ms_sym, 4),
             "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
@@ -510,13 +610,15 @@ def bench_token_sweep(dev, peaks, reps: int = 20):
                 for i in range(n):
                     binding.ot_linear(q, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
             ms = _graph_ms(calls, n)
+            ms16 = _fp16_gemm_ms(dev, M, N, K, n)
             ops = 2 * M * N * K
             t_roof = max(N * K / (peaks["hbm"] * 1e9), ops / (peaks["bf16"] * 1e12))
             out.append({"layer": layer.name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 2),
                         "tops": round(ops / (ms * 1e-3) / 1e12, 1),
                         "weight_gbs": round(N * K / (ms * 1e-3) / 1e9, 1),
                         "bound": "hbm" if N * K / (peaks["hbm"] * 1e9) > ops / (peaks["bf16"] * 1e12) else "tensor",
-                        "frac_roofline": round(t_roof / (ms * 1e-3), 4)})
+                        "frac_roofline": round(t_roof / (ms * 1e-3), 4),
+                        "cublas_fp16_us": round(ms16 * 1e3, 2), "speedup_vs_fp16": round(ms16 / ms, 3)})
             del q, y
         del qws
     del ws
@@ -525,51 +627,24 @@ def bench_token_sweep(dev, peaks, reps: int = 20):
             "per_point": out}
 
 
-def bench_large_gemm(dev, peaks, reps: int = 10):
-    """OPT-66B fc1 / fc2 (9216 <-> 36864) at 4096 tokens, W8A8: the linear
-    alone (codes resident) against a cuBLAS fp16 GEMM of the same shape.
-    Codes and weights are drawn directly (uniform in [-127, 127]); every
-    launch streams ~0.5 GB, above the L2."""
+def _fp16_gemm_ms(dev, M, N, K, reps):
+    """cuBLAS fp16 (torch.matmul) of [M, K] x [K, N] with fp16 weights W [N, K],
+    timed like the quantized linear beside it: `reps` consecutive calls that
+    rotate over enough weight copies to exceed 3x the L2, replayed from a CUDA
+    graph; ms per call."""
     import torch
+    g = torch.Generator(device=dev).manual_seed(5000 + M)
+    copies = max(2, -(-3 * L2_BYTES // (2 * N * K)))
+    ws = [(torch.randn(N, K, generator=g, device=dev) * 0.02).half() for _ in range(copies)]
+    x = torch.randn(M, K, generator=g, device=dev).half()
+    y = torch.empty(M, N, dtype=torch.float16, device=dev)
 
-    from paper_2406_18832_gb300 import binding
-    M = 4096
-    ws = torch.zeros(binding.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
-    g = torch.Generator(device=dev).manual_seed(66)
-    out = []
-    for name, K, N in (("fc1", 9216, 36864), ("fc2", 36864, 9216)):
-        q = torch.randint(-127, 128, (M, K), generator=g, device=dev, dtype=torch.int32).half()
-        qw = torch.randint(-127, 128, (N, K), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
-        sw = torch.rand(N, generator=g, device=dev) * 1e-5
-        bf = torch.zeros(N, device=dev)
-        y = torch.empty(M, N, dtype=torch.float16, device=dev)
-        x16 = torch.randn(M, K, generator=g, device=dev).half()
-        w16 = (torch.randn(N, K, generator=g, device=dev) * 0.02).half()
-
-        def med(fn):
-            for _ in range(2):
-                fn()
-            torch.cuda.synchronize()
-            ts = []
-            for _ in range(reps):
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record()
-                fn()
-                e1.record()
-                torch.cuda.synchronize()
-                ts.append(e0.elapsed_time(e1))
-            return statistics.median(ts)
-        ms = med(lambda: binding.ot_linear(q, qw, sw, bf, 8, 8, y, workspace=ws))
-        del y
-        ms16 = med(lambda: torch.matmul(x16, w16.t()))
-        ops = 2 * M * K * N
-        out.append({"layer": name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 1),
-                    "tops": round(ops / (ms * 1e-3) / 1e12, 1), "frac_peak": round(ops / (ms * 1e-3) / 1e12 / peaks["bf16"], 4),
-                    "cublas_fp16_us": round(ms16 * 1e3, 1), "cublas_fp16_tflops": round(ops / (ms16 * 1e-3) / 1e12, 1)})
-        del q, qw, x16, w16
-    del ws
-    torch.cuda.empty_cache()
-    return {"workload": "opt-66b fc1 / fc2 at 4096 tokens, W8A8", "kernel": "linear_pair_kernel", "per_layer": out}
+    def calls():
+        for i in range(reps):
+            torch.matmul(x, ws[i % copies].t(), out=y)
+    ms = _graph_ms(calls, reps)
+    del ws, x, y
+    return ms
 
 
 def bench_quantize_sweep(dev, peaks, reps: int = 20):
@@ -675,17 +750,18 @@ def bench_layernorm(dev, peaks, reps: int = 200):
             "unfused": "torch layer_norm (fp16 out) + quantize_kernel"}
 
 
-def bench_clipping(dev, peaks, calib_ms, calib_bytes, reps: int = 3):
-    """Token-wise clipping calibration (Appendix D) on the QKV calibration set
-    of the main workload (65,536 tokens x 4096, 512 MiB): per-channel order
-    statistics by a two-pass radix select, against the min/max calibration
-    of the main line (one pass)."""
+def bench_clipping(dev, peaks, minmax, reps: int = 3):
+    """Token-wise clipping calibration (Appendix D) on the OPT-6.7B QKV
+    calibration set (65,536 tokens x 4096, 512 MiB): per-channel order
+    statistics by a two-pass radix select, against the one-pass min / max
+    calibration of the same set (minmax = (ms, config) from the OPT-6.7B step)."""
     import torch
 
     from paper_2406_18832_gb300 import binding, synth
-    cfg = synth.CONFIGS[WORKLOAD_CFG]
+    minmax_ms, cfg_index = minmax
+    cfg = synth.CONFIGS[cfg_index]
     layer = cfg.layers[0]
-    x = synth.activations(WORKLOAD_CFG, 0, layer, cfg.T_cal, 3, device=dev)
+    x = synth.activations(cfg_index, 0, layer, cfg.T_cal, 3, device=dev)
     lo = torch.empty(layer.K, device=dev)
     hi = torch.empty(layer.K, device=dev)
     binding.ot_calibrate_clipped(x, 0.999, lo, hi)
@@ -703,7 +779,7 @@ def bench_clipping(dev, peaks, calib_ms, calib_bytes, reps: int = 3):
             "data_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
             "read_gbs": round(2 * nbytes / (ms * 1e-3) / 1e9, 1),
             "frac_hbm": round(2 * nbytes / (ms * 1e-3) / 1e9 / peaks["hbm"], 4),
-            "minmax_ms": round(calib_ms[0], 3), "note": "two passes over the data (radix select on fp16 keys)"}
+            "minmax_ms": round(minmax_ms, 3), "note": "two passes over the data (radix select on fp16 keys)"}
 
 
 def _graph_ms(calls, reps):
@@ -795,14 +871,17 @@ def bench_decode(dev, peaks, reps: int = 50):
                     binding.ot_linear_fused(x, z0, r1, 6, qws[i % copies], sw, bf, 6, qs, y, workspace=ws)
 
             ms_two, ms_fused = _graph_ms(two_calls, reps), _graph_ms(fused_calls, reps)
+            ms16 = _fp16_gemm_ms(dev, M, layer.N, layer.K, reps)
             res.append({"layer": layer.name, "K": layer.K, "N": layer.N, "tokens": M, "us": round(ms * 1e3, 2),
                         "weight_gbs": round(gbs, 1), "frac_hbm": round(gbs / peaks["hbm"], 4),
                         "eager_us": round(eager_ms * 1e3, 2), "quantize_then_linear_us": round(ms_two * 1e3, 2),
-                        "fused_us": round(ms_fused * 1e3, 2)})
+                        "fused_us": round(ms_fused * 1e3, 2), "cublas_fp16_us": round(ms16 * 1e3, 2),
+                        "speedup_vs_fp16": round(ms16 / ms, 3), "fused_speedup_vs_fp16": round(ms16 / ms_fused, 3)})
         del qws
     return {"workload": "opt-13b decode-sized linears, Int6", "kernel": "linear_gemv_kernel (mma.sync, TMA stream)",
             "bound": "hbm", "timing": "CUDA graph replay of consecutive calls (eager_us: one Python call each); "
-            "quantize_then_linear_us / fused_us: ot_quantize_act + ot_linear per call, or ot_linear_fused",
+            "quantize_then_linear_us / fused_us: ot_quantize_act + ot_linear per call, or ot_linear_fused; "
+            "cublas_fp16_us: torch.matmul fp16 of the same shape, fp16 weights, timed the same way",
             "l2": "consecutive calls read different weight copies, > 3x L2 in all",
             "per_shape": res}
 
@@ -870,87 +949,184 @@ def bench_block(dev, tokens: int = 4096, t_cal: int = 4096, reps: int = 20):
     return out
 
 
+def bench_per_token(dev, peaks, reps: int = 50):
+    """The per-token path (Eq. 3) the paper uses for the out and fc2 linears:
+    dynamic per-token scales and codes (one kernel), then the linear with the
+    per-token x per-channel epilogue, OPT-6.7B out (4096 -> 4096) and fc2
+    (16384 -> 4096) at 2048 tokens, W8A8, against the per-channel step of
+    the same shapes (static z, r) and cuBLAS fp16.  Consecutive calls replayed
+    from a CUDA graph."""
+    import torch
+
+    from paper_2406_18832_gb300 import binding, synth
+    c = synth.CONFIGS[STEP6_CFG]
+    M = STEP6_TOKENS
+    ws = torch.zeros(binding.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+    out = []
+    for li in (1, 3):
+        layer = c.layers[li]
+        K, N = layer.K, layer.N
+        w, b = synth.weights(STEP6_CFG, li, layer, device=dev)
+        x = synth.activations(STEP6_CFG, li, layer, M, 4, device=dev)
+        qw = torch.empty(N, K, dtype=torch.int8, device=dev)
+        sw = torch.empty(N, device=dev)
+        binding.ot_quantize_weights(w, 8, qw, sw)
+        bias = b.float()
+        q = torch.empty(M, K, dtype=torch.float16, device=dev)
+        s_tok = torch.empty(M, device=dev)
+        y = torch.empty(M, N, dtype=torch.float16, device=dev)
+
+        def tok_calls():
+            for _ in range(reps):
+                binding.ot_quantize_tokens(x, 8, q, s_tok)
+                binding.ot_linear_per_token(q, qw, sw, s_tok, bias, 8, 8, y, workspace=ws)
+
+        def quant_only():
+            for _ in range(reps):
+                binding.ot_quantize_tokens(x, 8, q, s_tok)
+        ms = _graph_ms(tok_calls, reps)
+        ms_q = _graph_ms(quant_only, reps)
+        ops = 2 * M * N * K
+        out.append({"layer": layer.name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 2),
+                    "tops": round(ops / (ms * 1e-3) / 1e12, 1), "quantize_tokens_us": round(ms_q * 1e3, 2),
+                    "quantize_tokens_gbs": round((3 * M * K + 4 * M) / (ms_q * 1e-3) / 1e9, 1)})
+        del w, b, x, qw, q, y
+    del ws
+    torch.cuda.empty_cache()
+    return {"workload": "opt-6.7b out and fc2 at 2048 tokens, per-token activations (Eq. 3), W8A8",
+            "timing": "CUDA graph replay; quantize_tokens reads each row twice (max, then codes; the second "
+                      "read mostly from L2); gbs on fp16 X in + int8 codes out + scales",
+            "per_layer": out}
+
+
 # ----------------------------------------------------------------------------
 # the CPU oracle (baseline leg and --impl reference)
 # ----------------------------------------------------------------------------
-def _oracle_layers(device_layers=None):
-    """Folded weights for every layer, computed by the oracle on the host."""
+def _oracle_fold_layers(host, bits, timings):
+    """Calibrate (on each layer's calibration sample), derive the parameters
+    and fold the whole layer with the oracle, timing each step."""
+    import oracle
+    out = []
+    for d in host:
+        t = time.perf_counter()
+        mn, mx = oracle.calibrate_mt(d["xc"])
+        timings["calibrate_s"] += time.perf_counter() - t
+        timings["calibrate_bytes"] += d["xc"].nbytes
+        t = time.perf_counter()
+        z, s, r = oracle.params(mn, mx, bits[0])
+        timings["params_s"] += time.perf_counter() - t
+        t = time.perf_counter()
+        qw, sw, bf = oracle.fold_mt(d["w"], d["b"], z, s, bits[1])
+        timings["fold_s"] += time.perf_counter() - t
+        timings["fold_weights"] += d["w"].size
+        out.append(dict(z=z, r=r, qw=qw, sw=sw, bf=bf, relu=d["relu"], K=d["w"].shape[1], N=d["w"].shape[0]))
+    return out
+
+
+def _oracle_tokens(ol, xs, rows, bits, timings):
+    """The online steps (quantize, int64 product, fp32-fma epilogue) of `rows`
+    tokens through every layer with the oracle's threaded drivers; returns ops."""
+    import oracle
+    ops = 0
+    for d, x in zip(ol, xs):
+        xr = x[rows]
+        t = time.perf_counter()
+        q = oracle.quantize_mt(xr, d["z"], d["r"], bits[0])
+        t1 = time.perf_counter()
+        acc = oracle.matmul_mt(q, d["qw"])
+        t2 = time.perf_counter()
+        oracle.epilogue_mt(acc, d["sw"], d["bf"], d["relu"])
+        t3 = time.perf_counter()
+        timings["quantize_s"] += t1 - t
+        timings["matmul_s"] += t2 - t1
+        timings["epilogue_s"] += t3 - t2
+        ops += 2 * len(rows) * d["N"] * d["K"]
+    return ops
+
+
+def _new_timings():
+    return dict(calibrate_s=0.0, calibrate_bytes=0, params_s=0.0, fold_s=0.0, fold_weights=0,
+                quantize_s=0.0, matmul_s=0.0, epilogue_s=0.0)
+
+
+def cpu_baseline(host, budget_s=12.0):
+    """Time the oracle, as it stands, per step of the headline workload on the
+    host cores (its C functions over row ranges in one thread per core):
+    calibration on 8192 tokens per layer, parameters, the fold of the whole
+    layers, then quantize / int64 product / epilogue of a token sample sized
+    to about `budget_s` seconds.  value = online ops / online seconds."""
+    import numpy as np
+
+    import oracle
+    tm = _new_timings()
+    ol = _oracle_fold_layers(host, BITS, tm)
+    xs = [d["x"] for d in host]
+    probe = _new_timings()
+    t = time.perf_counter()
+    _oracle_tokens(ol, xs, np.arange(16), BITS, probe)
+    per16 = time.perf_counter() - t
+    rows_n = int(max(16, min(xs[0].shape[0], budget_s / max(per16, 1e-6) * 16)) // 16 * 16)
+    ops = _oracle_tokens(ol, xs, np.arange(rows_n), BITS, tm)
+    online = tm["quantize_s"] + tm["matmul_s"] + tm["epilogue_s"]
+    cores = oracle.host_threads()
+    return {"value": round(ops / online / 1e12, 6), "unit": "TOPS", "cores": cores, "kind": "oracle",
+            "sample": f"{rows_n} of the {TOKENS} tokens through fc1 and fc2 (quantize, int64 product, fp32-fma "
+                      f"epilogue, {online:.1f} s); offline steps: calibration on 8192 tokens per layer, "
+                      f"parameters, the fold of both whole layers",
+            "per_step_s": {"calibrate": round(tm["calibrate_s"], 3), "params": round(tm["params_s"], 5),
+                           "fold": round(tm["fold_s"], 3), "quantize": round(tm["quantize_s"], 3),
+                           "matmul": round(tm["matmul_s"], 3), "epilogue": round(tm["epilogue_s"], 3)},
+            "calibrate_gbs": round(tm["calibrate_bytes"] / tm["calibrate_s"] / 1e9, 2),
+            "fold_mweights_per_s": round(tm["fold_weights"] / tm["fold_s"] / 1e6, 1),
+            "threads": "one per core of os.sched_getaffinity, rows (or channels) split evenly"}
+
+
+def run_reference(args):
+    """The CPU oracle on the headline workload (inputs drawn on the host), one
+    step = a bounded token sample through fc1 and fc2, sized so warm-up and
+    timed steps end within about two minutes."""
     import numpy as np
 
     import oracle
     from paper_2406_18832_gb300 import synth
-    cfg, _ = _workload_desc()
-    out = []
-    for li, layer in enumerate(cfg.layers):
-        w, b = synth.weights(WORKLOAD_CFG, li, layer)
-        xc = synth.activations(WORKLOAD_CFG, li, layer, 4096, 3)   # calibration sample (host)
-        mn, mx = oracle.calibrate(xc.numpy())
-        z, s, r = oracle.params(mn, mx, BITS[0])
-        qw, sw, bf = oracle.fold(w.numpy(), b.numpy(), z, s, BITS[1])
-        x = synth.activations(WORKLOAD_CFG, li, layer, 64, 4).numpy()
-        out.append(dict(qw=qw, sw=sw, bf=bf, z=z, r=r, x=x, K=layer.K, N=layer.N))
-    return out
-
-
-def _oracle_sample(ol, rows, cols):
-    import oracle
-    ops = 0
-    for d in ol:
-        x = d["x"][:rows]
-        q = oracle.quantize(x, d["z"], d["r"], BITS[0])
-        n = min(cols, d["N"])
-        acc = oracle.matmul(q, d["qw"][:n])
-        oracle.epilogue(acc, d["sw"][:n], d["bf"][:n])
-        ops += 2 * rows * n * d["K"]
-    return ops
-
-
-def cpu_baseline(budget_s=12.0, layers=None):
-    """Time the oracle (single-threaded C, as it stands) on a bounded sample of
-    the workload: `rows` tokens through the four layers, all output channels."""
-    ol = _oracle_layers()
-    t = time.perf_counter()
-    ops = _oracle_sample(ol, 1, 10 ** 9)
-    one = time.perf_counter() - t
-    rows = max(1, min(64, int(budget_s / max(one, 1e-6))))
-    t = time.perf_counter()
-    ops = _oracle_sample(ol, rows, 10 ** 9)
-    dt = time.perf_counter() - t
-    return {"value": round(ops / dt / 1e12, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
-            "sample": f"{rows} token(s) of the 2048 through all four layers (quantize, int64 product, "
-                      f"fp32-fma epilogue), every output channel; {dt:.1f} s",
-            "host_cores_available": len(os.sched_getaffinity(0))}
-
-
-def run_reference(args):
     rank, world, _ = _env_rank()
     if rank != 0:
         return
-    ol = _oracle_layers()
-    _, layer_shapes = _workload_desc()
-    # size one step so that warmup + steps fit in about two minutes of host time
+    cfg, layer_shapes = _workload_desc()
+    host = []
+    for li, layer in enumerate(cfg.layers):
+        w, b = synth.weights(WORKLOAD_CFG, li, layer)
+        host.append(dict(w=w.numpy(), b=b.numpy(), relu=layer.relu_out,
+                         xc=synth.activations(WORKLOAD_CFG, li, layer, 2048, 3).numpy(),
+                         x=synth.activations(WORKLOAD_CFG, li, layer, TOKENS, 4).numpy()))
+    setup = _new_timings()
+    ol = _oracle_fold_layers(host, BITS, setup)
+    xs = [d["x"] for d in host]
+    probe = _new_timings()
     t = time.perf_counter()
-    _oracle_sample(ol, 1, 256)
-    per256 = time.perf_counter() - t
-    budget_step = max(0.01, 120.0 / max(1, args.steps + args.warmup))
-    cols = int(max(16, min(16384, 256 * budget_step / max(per256, 1e-6))))
-    for _ in range(args.warmup):
-        _oracle_sample(ol, 1, cols)
+    _oracle_tokens(ol, xs, np.arange(8), BITS, probe)
+    per8 = time.perf_counter() - t
+    budget_step = max(0.05, 110.0 / max(1, args.steps + args.warmup))
+    rows_n = int(max(1, min(TOKENS, budget_step / max(per8, 1e-6) * 8)))
+    for k in range(args.warmup):
+        _oracle_tokens(ol, xs, (np.arange(rows_n) + k * rows_n) % TOKENS, BITS, _new_timings())
+    tm = _new_timings()
     t = time.perf_counter()
     ops = 0
-    for _ in range(args.steps):
-        ops += _oracle_sample(ol, 1, cols)
+    for k in range(args.steps):
+        ops += _oracle_tokens(ol, xs, (np.arange(rows_n) + (k + args.warmup) * rows_n) % TOKENS, BITS, tm)
     dt = time.perf_counter() - t
     value = ops / dt / 1e12
-    sample = (f"per step: 1 token through all four layers, first {cols} output channels of each "
-              f"(quantize, int64 product, fp32-fma epilogue)")
+    cores = oracle.host_threads()
+    sample = (f"per step: {rows_n} of the {TOKENS} tokens through fc1 and fc2 (quantize, int64 product, "
+              f"fp32-fma epilogue) on {cores} host threads; weights folded once before timing")
     line = {"metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64 (CPU oracle)", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": "opt-6.7b-linears-prefill", "tokens": TOKENS, "bits_a": BITS[0],
-                       "bits_w": BITS[1], "layers": [{"name": n, "K": K, "N": N} for n, K, N in layer_shapes]},
-            "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": 1, "kind": "oracle",
+            "config": {"workload": WORKLOAD_NAME, "tokens": TOKENS, "bits_a": BITS[0], "bits_w": BITS[1],
+                       "layers": [{"name": n, "K": K, "N": N} for n, K, N in layer_shapes]},
+            "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -959,8 +1135,8 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
