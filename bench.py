@@ -613,17 +613,44 @@ def bench_token_sweep(dev, peaks, reps: int = 20):
             ms16 = _fp16_gemm_ms(dev, M, N, K, n)
             ops = 2 * M * N * K
             t_roof = max(N * K / (peaks["hbm"] * 1e9), ops / (peaks["bf16"] * 1e12))
-            out.append({"layer": layer.name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 2),
-                        "tops": round(ops / (ms * 1e-3) / 1e12, 1),
-                        "weight_gbs": round(N * K / (ms * 1e-3) / 1e9, 1),
-                        "bound": "hbm" if N * K / (peaks["hbm"] * 1e9) > ops / (peaks["bf16"] * 1e12) else "tensor",
-                        "frac_roofline": round(t_roof / (ms * 1e-3), 4),
-                        "cublas_fp16_us": round(ms16 * 1e3, 2), "speedup_vs_fp16": round(ms16 / ms, 3)})
+            pt = {"layer": layer.name, "K": K, "N": N, "tokens": M, "us": round(ms * 1e3, 2),
+                  "tops": round(ops / (ms * 1e-3) / 1e12, 1),
+                  "weight_gbs": round(N * K / (ms * 1e-3) / 1e9, 1),
+                  "bound": "hbm" if N * K / (peaks["hbm"] * 1e9) > ops / (peaks["bf16"] * 1e12) else "tensor",
+                  "frac_roofline": round(t_roof / (ms * 1e-3), 4),
+                  "cublas_fp16_us": round(ms16 * 1e3, 2), "speedup_vs_fp16": round(ms16 / ms, 3)}
+            if M <= 128:
+                # int8 codes in, and the quantization inside the linear (fp16 X in), against
+                # the quantize kernel followed by the linear
+                q8 = q.to(torch.int8)
+                x = q.clone()
+                z0, r1 = torch.zeros(K, device=dev), torch.ones(K, device=dev)
+                qs = torch.empty_like(q)
+
+                def calls8():
+                    for i in range(n):
+                        binding.ot_linear(q8, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
+
+                def calls_fused():
+                    for i in range(n):
+                        binding.ot_linear_fused(x, z0, r1, 6, qws[i % copies], sw, bf, 6, qs, y, workspace=ws)
+
+                def calls_two():
+                    for i in range(n):
+                        binding.ot_quantize_act(x, z0, r1, 6, qs, binding.OT_CODE_F16)
+                        binding.ot_linear(qs, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
+                pt["int8_codes_us"] = round(_graph_ms(calls8, n) * 1e3, 2)
+                pt["fused_us"] = round(_graph_ms(calls_fused, n) * 1e3, 2)
+                pt["quantize_then_linear_us"] = round(_graph_ms(calls_two, n) * 1e3, 2)
+                del q8, x, qs
+            out.append(pt)
             del q, y
         del qws
     del ws
     torch.cuda.empty_cache()
     return {"workload": "opt-13b QKV and fc2, Int6, 1-4096 tokens", "timing": "CUDA graph replay, rotating weights",
+            "up_to_128_tokens": "int8_codes_us: ot_linear on int8 codes; fused_us: ot_linear_fused (fp16 X in, "
+                                "quantized inside the linear); quantize_then_linear_us: ot_quantize_act + ot_linear",
             "per_point": out}
 
 
@@ -703,7 +730,7 @@ def bench_layernorm(dev, peaks, reps: int = 200):
     import torch.nn.functional as F
 
     from paper_2406_18832_gb300 import binding
-    M, K, eps = TOKENS, 4096, 1e-5
+    M, K, eps = STEP6_TOKENS, 4096, 1e-5
     g = torch.Generator(device=dev).manual_seed(77)
     copies = -(-3 * L2_BYTES // (M * K * 2))
     hs = [torch.randn(M, K, generator=g, device=dev).half() for _ in range(copies)]

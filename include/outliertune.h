@@ -47,12 +47,14 @@ typedef enum {
     OT_ERR_TIMEOUT = 4       /* a bounded device-side wait gave up */
 } ot_status;
 
-/* Storage format of activation codes written by ot_quantize_act. */
+/* Storage format of activation codes (written by the quantize entry points,
+ * read by ot_linear / ot_linear_s32). */
 typedef enum {
-    OT_CODE_I8 = 0,   /* int8 codes, 1 byte per element */
-    OT_CODE_F16 = 1   /* the same integers stored exactly as fp16 (the operand
-                         format ot_linear reads: sm_103a has no integer tcgen05
-                         MMA, so the product runs on the fp16 tensor path) */
+    OT_CODE_I8 = 0,   /* int8 codes, 1 byte per element (the paper's storage) */
+    OT_CODE_F16 = 1   /* the same integers stored exactly as fp16: the operand
+                         format of the tensor cores (sm_103a has no integer
+                         tcgen05 MMA, so the product runs on the fp16 tensor
+                         path); the fastest input for more than 128 tokens */
 } ot_code_format;
 
 /* Human-readable name of a status code (static string, never NULL). */
@@ -128,8 +130,13 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  * (Eq. 6) and the folded bias (Eq. 7):
  *   acc[m,n] = sum_k q[m,k] * qw[n,k]            exact integer
  *   y[m,n]   = fp16( fma((float)acc[m,n], sw_n, b'_n) ), then ReLU if relu != 0
- *   q_f16   activation codes as fp16 integers [M, K] (OT_CODE_F16 output of
- *           ot_quantize_act), |q| <= qmax(bits_a); 16-byte aligned, K % 16 == 0
+ *   q       activation codes [M, K], dense, |q| <= qmax(bits_a); 16-byte
+ *           aligned, K % 16 == 0; q_format OT_CODE_I8 (int8, as ot_quantize_act
+ *           writes them with OT_CODE_I8) or OT_CODE_F16 (fp16 integers).  int8
+ *           codes are widened to fp16 inside the kernel (decode kernel for
+ *           M <= 16, the single-CTA tcgen05 kernel's token warps above); fp16
+ *           codes for M > 128 take the CTA-pair prefill kernel, which reads
+ *           them directly and is the fastest path at prefill sizes
  *   qw      int8 [N, K] from ot_fold_weights, |qw| <= qmax(bits_w); 16-byte aligned
  *   sw, b_fold  fp32 [N]
  *   y_f16   fp16 [M, N], row stride ldy >= N
@@ -151,10 +158,11 @@ ot_status ot_quantize_act(const void *x_f16, int64_t M, int64_t K, int64_t ldx,
  * chunks in int32.  Codes outside [-qmax, qmax] void that guarantee.
  * K * qmax_a * qmax_w must be < 2^31 (K <= 133144 for W8A8).
  */
-ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
-                    const float *sw, const float *b_fold, int64_t N, int bits_a,
-                    int bits_w, void *y_f16, int64_t ldy, int relu,
-                    void *workspace, size_t workspace_bytes, void *stream);
+ot_status ot_linear(const void *q, int q_format, int64_t M, int64_t K,
+                    const int8_t *qw, const float *sw, const float *b_fold,
+                    int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy,
+                    int relu, void *workspace, size_t workspace_bytes,
+                    void *stream);
 
 /*
  * ot_linear_workspace_size -- bytes of scratch that let ot_linear /
@@ -311,18 +319,24 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
                          size_t workspace_bytes, void *stream);
 
 /*
- * ot_linear_fused -- ot_quantize_act followed by ot_linear in one call (the
- * activation quantization of Eq. 6-7 fused in front of the product, as
- * Section 3.2 fuses it with the operation producing X): q = codes of X
- * (fp16 integers), y = fp16(fma(sum_k q qw, sw_n, b'_n)), ReLU if relu.
- * The linear is launched as a programmatic dependent of the quantization, so
- * its weight stream and set-up overlap the quantization and only its reads of
- * the codes wait for it.
+ * ot_linear_fused -- the per-channel quantization of X (Eq. 6-7) and the
+ * linear in one call: q = codes of X, y = fp16(fma(sum_k q qw, sw_n, b'_n)),
+ * ReLU if relu; the result is bit-identical to ot_quantize_act followed by
+ * ot_linear.
+ *   - M <= 128: the linear's own token producer reads fp16 X and quantizes
+ *     each tile in shared memory before the tensor cores read it (the
+ *     quantization inside the GEMM's operand producer): one kernel, and the
+ *     codes never reach HBM; q_f16 is not written.
+ *   - M > 128: the quantize kernel writes the codes to q_f16, and the linear
+ *     is launched as its programmatic dependent, so the linear's weight loads
+ *     and set-up overlap the quantization and only its reads of the codes wait
+ *     for it (at prefill sizes each token tile is read by every weight tile,
+ *     so quantizing once beats quantizing in every CTA).
  * x_f16 fp16 [M, ldx] (ldx >= K, ldx % 8 == 0, 16-byte aligned); z, r fp32 [K]
  * (16-byte aligned); q_f16: caller scratch fp16 [M, K], dense, 16-byte
- * aligned, receives the codes (valid after the stream synchronizes); the
- * remaining arguments as ot_linear.  Same validation and errors as the two
- * calls; M == 0 launches nothing.
+ * aligned, whose contents are unspecified afterwards; the remaining arguments
+ * as ot_linear.  Same validation and errors as the two calls; M == 0
+ * launches nothing.
  */
 ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z,
                           const float *r, int bits_a, const int8_t *qw, const float *sw,
@@ -380,10 +394,12 @@ ot_status ot_linear_noalloc(const void *q_f16, int64_t M, int64_t K,
  * ot_linear_s32 -- the same integer product as ot_linear, written out as the
  * int32 accumulators acc[m,n] (dense [M, N]) instead of the scaled fp16
  * output; the accumulators of Eq. 6 before external scaling, for checking.
+ * q and q_format as in ot_linear.
  */
-ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw,
-                        int64_t N, int bits_a, int bits_w, int32_t *acc,
-                        void *workspace, size_t workspace_bytes, void *stream);
+ot_status ot_linear_s32(const void *q, int q_format, int64_t M, int64_t K,
+                        const int8_t *qw, int64_t N, int bits_a, int bits_w,
+                        int32_t *acc, void *workspace, size_t workspace_bytes,
+                        void *stream);
 
 /*
  * ot_get_device_status -- synchronize `stream`, then return and clear the

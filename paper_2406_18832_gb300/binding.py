@@ -30,8 +30,8 @@ _SIGNATURES = {
     "ot_derive_params": ([_P, _P, _I64, _I, _I, _P, _P, _P, _P], _I),
     "ot_fold_weights": ([_P, _P, _I, _I, _P, _P, _I64, _I64, _I, _P, _P, _P, _P, _P, _P, _P], _I),
     "ot_quantize_act": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _I, _P], _I),
-    "ot_linear": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P], _I),
-    "ot_linear_s32": ([_P, _I64, _I64, _P, _I64, _I, _I, _P, _P, ctypes.c_size_t, _P], _I),
+    "ot_linear": ([_P, _I, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P, ctypes.c_size_t, _P], _I),
+    "ot_linear_s32": ([_P, _I, _I64, _I64, _P, _I64, _I, _I, _P, _P, ctypes.c_size_t, _P], _I),
     "ot_linear_workspace_size": ([_P], _I),
     "ot_linear_noalloc": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _P, _I64, _I, _P], _I),
     "ot_quantize_tokens": ([_P, _I64, _I64, _I64, _I, _P, _I, _P, _P], _I),
@@ -245,7 +245,8 @@ def ot_layernorm_quantize(h, gamma_r, beta_r, eps: float, bits_a: int, q, q_form
 
 def ot_linear_fused(x, z, r, bits_a: int, qw, sw, b_fold, bits_w: int, q, y, relu: bool = False, workspace=None,
                     stream=None):
-    """Quantize x into q (fp16 codes [M, K]) and run the linear into y [M, N] in one call."""
+    """Quantize x and run the linear into y [M, N] in one call; q is fp16 scratch [M, K] (written only
+    above 128 tokens, where the codes go through HBM)."""
     M, K, ldx = _rows(x, "x")
     _dense(q, "q")
     _dense(qw, "qw")
@@ -316,7 +317,15 @@ def _ws_args(workspace, device, stream):
     return _dev(workspace, "workspace"), workspace.numel() * workspace.element_size()
 
 
+def _codes(q):
+    """(pointer, ot_code_format) of an activation-code tensor: int8 or fp16 codes."""
+    if q.dtype == torch.int8:
+        return _dev(q, "q", torch.int8), OT_CODE_I8
+    return _dev(q, "q", torch.float16), OT_CODE_F16
+
+
 def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False, workspace=None, stream=None):
+    """y = fp16(fma(sum_k q qw, sw, b')); q holds int8 or fp16 codes (its dtype picks the format)."""
     _dense(q, "q")
     _dense(qw, "qw")
     M, K = q.shape
@@ -324,9 +333,9 @@ def ot_linear(q, qw, sw, b_fold, bits_a: int, bits_w: int, y, relu: bool = False
     ym, yn, ldy = _rows(y, "y")
     if ym != M or yn != N:
         raise ValueError("y must be [M, N]")
-    pq = _dev(q, "q", torch.float16)
+    pq, fmt = _codes(q)
     wp, wb = _ws_args(workspace, q.device, stream)
-    _check(load().ot_linear(pq, M, K, _dev(qw, "qw", torch.int8), _dev(sw, "sw", torch.float32),
+    _check(load().ot_linear(pq, fmt, M, K, _dev(qw, "qw", torch.int8), _dev(sw, "sw", torch.float32),
                             _dev(b_fold, "b_fold", torch.float32), N, bits_a, bits_w,
                             _dev(y, "y", torch.float16), ldy, 1 if relu else 0, wp, wb, _stream(stream)),
            "ot_linear")
@@ -392,9 +401,9 @@ def ot_linear_s32(q, qw, bits_a: int, bits_w: int, acc, workspace=None, stream=N
     _dense(acc, "acc")
     M, K = q.shape
     N = qw.shape[0]
-    pq = _dev(q, "q", torch.float16)
+    pq, fmt = _codes(q)
     wp, wb = _ws_args(workspace, q.device, stream)
-    _check(load().ot_linear_s32(pq, M, K, _dev(qw, "qw", torch.int8), N, bits_a, bits_w,
+    _check(load().ot_linear_s32(pq, fmt, M, K, _dev(qw, "qw", torch.int8), N, bits_a, bits_w,
                                 _dev(acc, "acc", torch.int32), wp, wb, _stream(stream)),
            "ot_linear_s32")
 

@@ -186,16 +186,18 @@ ot_status ot_linear_workspace_size(size_t *bytes) {
     return OT_OK;
 }
 
-ot_status ot_linear(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, const float *sw, const float *b_fold,
-                    int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy, int relu, void *workspace,
-                    size_t workspace_bytes, void *stream) {
-    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
+ot_status ot_linear(const void *q, int q_format, int64_t M, int64_t K, const int8_t *qw, const float *sw,
+                    const float *b_fold, int64_t N, int bits_a, int bits_w, void *y_f16, int64_t ldy, int relu,
+                    void *workspace, size_t workspace_bytes, void *stream) {
+    if (q_format != OT_CODE_I8 && q_format != OT_CODE_F16) return OT_ERR_INVALID_ARG;
+    ot_status v = linear_common(q, M, K, qw, N, bits_a, bits_w, y_f16);
     if (v != OT_OK) return v;
     if (!sw || !b_fold || ldy < N || (y_f16 && !aligned(y_f16, 2))) return OT_ERR_INVALID_ARG;
     if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
     if (ldy > kIntMax) return OT_ERR_UNSUPPORTED;
-    ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+    ot::LinearArgs a{q, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
                      workspace, workspace ? workspace_bytes : 0};
+    a.q_fmt = q_format == OT_CODE_I8 ? ot::kCodesI8 : ot::kCodesF16;
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
@@ -246,6 +248,17 @@ ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, 
     if (ldy > kIntMax || (M + 63) / 64 > 65535) return OT_ERR_UNSUPPORTED;
     if (M == 0) return OT_OK;
     const cudaStream_t st = as_stream(stream);
+    if (M <= ot::kFusedInKernelMaxTokens) {
+        // the linear's token producer quantizes X itself (no codes in HBM)
+        ot::LinearArgs a{x_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
+                         workspace, workspace ? workspace_bytes : 0};
+        a.q_fmt = ot::kActF16;
+        a.xz = z;
+        a.xr = r;
+        a.ldx = ldx;
+        a.qmax_in = (int)qmax_of(bits_a);
+        return from_cuda(ot::launch_linear(a, st));
+    }
     cudaError_t e = ot::launch_quantize(x_f16, M, K, ldx, z, r, bits_a, q_f16, OT_CODE_F16, st);
     if (e != cudaSuccess) return from_cuda(e);
     ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
@@ -287,14 +300,17 @@ ot_status ot_linear_noalloc(const void *q_f16, int64_t M, int64_t K, const int8_
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 
-ot_status ot_linear_s32(const void *q_f16, int64_t M, int64_t K, const int8_t *qw, int64_t N, int bits_a,
-                        int bits_w, int32_t *acc, void *workspace, size_t workspace_bytes, void *stream) {
-    ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, acc);
+ot_status ot_linear_s32(const void *q, int q_format, int64_t M, int64_t K, const int8_t *qw, int64_t N,
+                        int bits_a, int bits_w, int32_t *acc, void *workspace, size_t workspace_bytes,
+                        void *stream) {
+    if (q_format != OT_CODE_I8 && q_format != OT_CODE_F16) return OT_ERR_INVALID_ARG;
+    ot_status v = linear_common(q, M, K, qw, N, bits_a, bits_w, acc);
     if (v != OT_OK) return v;
     if (acc && !aligned(acc, 4)) return OT_ERR_INVALID_ARG;
     if (workspace && !aligned(workspace, 16)) return OT_ERR_INVALID_ARG;
-    ot::LinearArgs a{q_f16, qw, nullptr, nullptr, acc, M, N, K, N, bits_a, bits_w, 0, true,
+    ot::LinearArgs a{q, qw, nullptr, nullptr, acc, M, N, K, N, bits_a, bits_w, 0, true,
                      workspace, workspace ? workspace_bytes : 0};
+    a.q_fmt = q_format == OT_CODE_I8 ? ot::kCodesI8 : ot::kCodesF16;
     return from_cuda(ot::launch_linear(a, as_stream(stream)));
 }
 

@@ -58,14 +58,27 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemAccCol = 256;   // A buffers at columns [0, 32*kStages), accumulators from 256
 static_assert(32 * kStages <= (int)kTmemAccCol, "TMEM A buffers overlap the accumulators");
 
-template <int BN>
+// Token operand of linear_kernel (its MMA's B): fp16 codes copied by TMA as
+// they are (kTokF16); int8 codes copied into a staging buffer and widened to
+// fp16 by four token warps (kTokI8); or fp16 activations copied by TMA and
+// quantized in place by the token warps, per channel with z and r (kTokX:
+// the quantization of Eq. 6 / Eq. 7 inside the GEMM's operand producer).
+constexpr int kTokF16 = 0, kTokI8 = 1, kTokX = 2;
+constexpr int kWarpTok0 = 16;  // token warps 16-19 (kTok != kTokF16: 20 warps)
+template <int kTok>
+__host__ __device__ constexpr int lin_threads() { return kTok == kTokF16 ? kThreads : kThreads + 128; }
+
+template <int BN, int kTok>
 struct alignas(1024) Smem {
     uint8_t b[kStages][BN * 128];   // activation codes, 128-byte swizzled rows
     uint8_t w[kStages][kBM * kBK];  // int8 weight codes, 64-byte swizzled rows
+    uint8_t bs[kTok == kTokI8 ? kStages : 1][kTok == kTokI8 ? BN * 64 : 16];  // int8 codes as copied (kTokI8)
     uint64_t full[kStages];         // TMA landed (tx bytes)
     uint64_t empty[kStages];        // stage free: MMA done with b[] + 4 converter warps done with w[]
+                                    // (+ kTokI8: 4 token warps done with bs[])
     uint64_t afull[kStages];        // TMEM A buffer written (4 converter warps)
     uint64_t aempty[kStages];       // TMEM A buffer consumed (MMA commit)
+    uint64_t bfull[kStages];        // kTok != kTokF16: b[] holds fp16 codes (4 token warps)
     uint64_t accfull[2];            // chunk accumulator complete (MMA commit)
     uint64_t accempty[2];           // chunk accumulator drained (8 epilogue warps)
     uint64_t drain;                 // teardown: all issued MMAs complete
@@ -84,21 +97,6 @@ __device__ __forceinline__ void wait_teardown(uint32_t bar, uint32_t parity) {
             return;
         }
     }
-}
-
-// 4 signed int8 codes -> two fp16x2 words (exact).  Each byte b is biased to
-// u = b + 128 and placed under the fp16 exponent of 1024 (bit pattern
-// 0x6400 | u = 1024 + u, unit spacing in [1024, 2048)); subtracting 1152
-// leaves b exactly.
-__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
-    const uint32_t u = w ^ 0x80808080u;
-    const uint32_t a = __byte_perm(u, 0x64646464u, 0x4140);
-    const uint32_t b = __byte_perm(u, 0x64646464u, 0x4342);
-    const __half2 bias = __half2half2(__ushort_as_half(0x6480));  // 1152
-    const __half2 ha = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
-    const __half2 hb = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
-    lo = *reinterpret_cast<const uint32_t *>(&ha);
-    hi = *reinterpret_cast<const uint32_t *>(&hb);
 }
 
 // Work of one worker (a CTA pair of linear_pair_kernel, a CTA of
@@ -186,23 +184,25 @@ __device__ __forceinline__ uint64_t ld_acquire_u64(const unsigned long long *p) 
     return v;
 }
 
-template <int BN, bool kS32, bool kAsym, bool kQOut>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int BN, bool kS32, bool kAsym, bool kQOut, int kTok>
+__global__ void __launch_bounds__(lin_threads<kTok>(), 1)
     linear_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                   const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
                   int N, int K, int ldy, int kcb, int relu, const float *__restrict__ s_tok,
                   const int32_t *__restrict__ zc, const int32_t *__restrict__ rowsum,
                   const float *__restrict__ zq, const float *__restrict__ rq, int qmax_out,
-                  int32_t *__restrict__ ws, int ws_pairs) {
+                  int32_t *__restrict__ ws, int ws_pairs, const float *__restrict__ xz,
+                  const float *__restrict__ xr, int qmax_in) {
     extern __shared__ uint8_t smem_raw[];
-    Smem<BN> &S = *reinterpret_cast<Smem<BN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem<BN, kTok> &S =
+        *reinterpret_cast<Smem<BN, kTok> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
     const int m_tiles = (M + BN - 1) / BN;
     const int n_tiles = (N + kBM - 1) / kBM;
     const int num_tiles = m_tiles * n_tiles;
     const int nkb = (K + kBK - 1) / kBK;
     volatile int *abort = &S.abort;
-    constexpr uint32_t kTxBytes = BN * 128 + kBM * kBK;
+    constexpr uint32_t kTxBytes = (kTok == kTokI8 ? BN * 64 : BN * 128) + kBM * kBK;
     // With a workspace (the prefill kernel's layout, ws_pairs pairs of slots)
     // the CTAs split tiles along K like the pairs of linear_pair_kernel.
     PairSched sch;
@@ -211,9 +211,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_u32(&S.full[s]), 1);
-            mbar_init(smem_u32(&S.empty[s]), 1 + 4);
+            mbar_init(smem_u32(&S.empty[s]), 1 + 4 + (kTok == kTokI8 ? 4 : 0));
             mbar_init(smem_u32(&S.afull[s]), 4);
             mbar_init(smem_u32(&S.aempty[s]), 1);
+            mbar_init(smem_u32(&S.bfull[s]), 4);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&S.accfull[b]), 1);
@@ -239,83 +240,92 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = S.tmem_base;
 
     // the TMA and MMA roles run their loops with the whole warp and issue from one elected lane
-    if (warp == kWarpTma) {
-        // weights of the first tile into L2 while a programmatic predecessor
-        // may still be writing the codes; then wait for it
-        if (sch.count > 0 && elect_one()) {
-            int u, pk0, pk1;
-            sch.piece(0, u, pk0, pk1);
-            for (int kb = pk0; kb < pk1 && kb < pk0 + kStages; ++kb)
-                tma_prefetch_l2_2d(&tm_w, kb * kBK, (u / m_tiles) * kBM);
-        }
-        __syncwarp();
-        grid_dep_wait();
-        uint32_t it = 0;
-        bool ok = true;
-        for (int p = 0; p < sch.count && ok; ++p) {
-            int u, pk0, pk1;
-            sch.piece(p, u, pk0, pk1);
-            const int m0 = (u % m_tiles) * BN, n0 = (u / m_tiles) * kBM;
-            for (int kb = pk0; kb < pk1; ++kb, ++it) {
-                const int s = it % kStages;
-                const uint32_t ph = (it / kStages) & 1;
-                if (!(ok = mbar_wait_warp(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status))) break;
-                if (elect_one()) {
-                    mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
-                    tma_load_2d(smem_u32(S.b[s]), &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
-                    tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
-                }
-                __syncwarp();
+    // registers: 512 threads x 128 at launch (kTokF16); with the token warps
+    // 640 x 96, then per warpgroup 48 / 72 / 144 / 144 / 72
+    if (warp < 4) {
+        if constexpr (kTok != kTokF16) regs_dec<48>();
+        if (warp == kWarpTma) {
+            // weights of the first tile into L2 while a programmatic predecessor
+            // may still be writing the codes; then wait for it
+            if (sch.count > 0 && elect_one()) {
+                int u, pk0, pk1;
+                sch.piece(0, u, pk0, pk1);
+                for (int kb = pk0; kb < pk1 && kb < pk0 + kStages; ++kb)
+                    tma_prefetch_l2_2d(&tm_w, kb * kBK, (u / m_tiles) * kBM);
             }
-        }
-        // teardown: every load issued must have landed before the CTA exits
-        if (lane == 0) {
-            const uint32_t issued = it;
-            for (uint32_t j = issued > (uint32_t)kStages ? issued - kStages : 0; j < issued; ++j)
-                wait_teardown(smem_u32(&S.full[j % kStages]), (j / kStages) & 1);
-        }
-        __syncwarp();
-    } else if (warp == kWarpMma) {
-        const uint32_t idesc = idesc_f16_f32(kBM, BN);
-        uint32_t it = 0, g = 0;
-        bool ok = true;
-        for (int p = 0; p < sch.count && ok; ++p) {
-            int u, pk0, pk1;
-            sch.piece(p, u, pk0, pk1);
-            for (int kb0 = pk0; kb0 < pk1 && ok; kb0 += kcb, ++g) {
-                const int buf = g & 1;
-                if (!(ok = mbar_wait_warp(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
-                tc_fence_after();
-                const uint32_t d = tmem + kTmemAccCol + buf * BN;
-                const int kb1 = min(pk1, kb0 + kcb);
-                for (int kb = kb0; kb < kb1; ++kb, ++it) {
+            __syncwarp();
+            grid_dep_wait();
+            uint32_t it = 0;
+            bool ok = true;
+            for (int p = 0; p < sch.count && ok; ++p) {
+                int u, pk0, pk1;
+                sch.piece(p, u, pk0, pk1);
+                const int m0 = (u % m_tiles) * BN, n0 = (u / m_tiles) * kBM;
+                for (int kb = pk0; kb < pk1; ++kb, ++it) {
                     const int s = it % kStages;
                     const uint32_t ph = (it / kStages) & 1;
-                    if (!(ok = mbar_wait_warp(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
-                    if (!(ok = mbar_wait_warp(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
-                    tc_fence_after();
-                    const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status))) break;
                     if (elect_one()) {
-#pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk)
-                            mma_f16_ts(d, tmem + s * 32 + kk * 8, bdesc + (uint64_t)((kk * 32) >> 4), idesc,
-                                       (kb != kb0 || kk != 0) ? 1u : 0u);
-                        mma_commit(smem_u32(&S.empty[s]));
-                        mma_commit(smem_u32(&S.aempty[s]));
+                        mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
+                        tma_load_2d(smem_u32(kTok == kTokI8 ? S.bs[s % (kTok == kTokI8 ? kStages : 1)] : S.b[s]),
+                                    &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
+                        tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
                     }
                     __syncwarp();
                 }
-                if (ok && elect_one()) mma_commit(smem_u32(&S.accfull[buf]));
-                __syncwarp();
             }
+            // teardown: every load issued must have landed before the CTA exits
+            if (lane == 0) {
+                const uint32_t issued = it;
+                for (uint32_t j = issued > (uint32_t)kStages ? issued - kStages : 0; j < issued; ++j)
+                    wait_teardown(smem_u32(&S.full[j % kStages]), (j / kStages) & 1);
+            }
+            __syncwarp();
+        } else if (warp == kWarpMma) {
+            const uint32_t idesc = idesc_f16_f32(kBM, BN);
+            uint32_t it = 0, g = 0;
+            bool ok = true;
+            for (int p = 0; p < sch.count && ok; ++p) {
+                int u, pk0, pk1;
+                sch.piece(p, u, pk0, pk1);
+                for (int kb0 = pk0; kb0 < pk1 && ok; kb0 += kcb, ++g) {
+                    const int buf = g & 1;
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status))) break;
+                    tc_fence_after();
+                    const uint32_t d = tmem + kTmemAccCol + buf * BN;
+                    const int kb1 = min(pk1, kb0 + kcb);
+                    for (int kb = kb0; kb < kb1; ++kb, ++it) {
+                        const int s = it % kStages;
+                        const uint32_t ph = (it / kStages) & 1;
+                        // the token warps and the converters both start after the stage's copies landed
+                        const uint32_t bbar = kTok == kTokF16 ? smem_u32(&S.full[s]) : smem_u32(&S.bfull[s]);
+                        if (!(ok = mbar_wait_warp(bbar, ph, abort, &g_status))) break;
+                        if (!(ok = mbar_wait_warp(smem_u32(&S.afull[s]), ph, abort, &g_status))) break;
+                        tc_fence_after();
+                        const uint64_t bdesc = smem_desc_sw128(smem_u32(S.b[s]));
+                        if (elect_one()) {
+    #pragma unroll
+                            for (int kk = 0; kk < kBK / 16; ++kk)
+                                mma_f16_ts(d, tmem + s * 32 + kk * 8, bdesc + (uint64_t)((kk * 32) >> 4), idesc,
+                                           (kb != kb0 || kk != 0) ? 1u : 0u);
+                            mma_commit(smem_u32(&S.empty[s]));
+                            mma_commit(smem_u32(&S.aempty[s]));
+                        }
+                        __syncwarp();
+                    }
+                    if (ok && elect_one()) mma_commit(smem_u32(&S.accfull[buf]));
+                    __syncwarp();
+                }
+            }
+            // teardown: all issued MMAs complete before TMEM is freed
+            if (elect_one()) {
+                mma_commit(smem_u32(&S.drain));
+                wait_teardown(smem_u32(&S.drain), 0);
+            }
+            __syncwarp();
         }
-        // teardown: all issued MMAs complete before TMEM is freed
-        if (elect_one()) {
-            mma_commit(smem_u32(&S.drain));
-            wait_teardown(smem_u32(&S.drain), 0);
-        }
-        __syncwarp();
-    } else if (warp >= kWarpConv0 && warp < kWarpConv0 + 4) {
+    } else if (warp < kWarpEpi0) {
+        if constexpr (kTok != kTokF16) regs_dec<72>();
         const int q = warp & 3;
         const int row = q * 32 + lane;           // weight row of the tile = TMEM lane
         const uint32_t sw64 = (row >> 1) & 3;    // 64-byte swizzle phase of this row
@@ -335,24 +345,92 @@ __global__ void __launch_bounds__(kThreads, 1)
                     raw[c] = *reinterpret_cast<const uint4 *>(S.w[s] + row * 64 + ((c ^ sw64) << 4));
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.empty[s]));
-                uint32_t a[32];
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    i8x4_to_f16x4(raw[c].x, a[8 * c + 0], a[8 * c + 1]);
-                    i8x4_to_f16x4(raw[c].y, a[8 * c + 2], a[8 * c + 3]);
-                    i8x4_to_f16x4(raw[c].z, a[8 * c + 4], a[8 * c + 5]);
-                    i8x4_to_f16x4(raw[c].w, a[8 * c + 6], a[8 * c + 7]);
-                }
                 if (!(ok = mbar_wait(smem_u32(&S.aempty[s]), ph ^ 1, abort, &g_status))) break;
                 tc_fence_after();
-                tmem_st32(tmem + lane_base + s * 32, a);
+                // the row's 64 fp16 values, two per 32-bit TMEM column, k ascending, in two halves
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    uint32_t a[16];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const uint4 r4 = raw[2 * half + c];
+                        i8x4_to_f16x4(r4.x, a[8 * c + 0], a[8 * c + 1]);
+                        i8x4_to_f16x4(r4.y, a[8 * c + 2], a[8 * c + 3]);
+                        i8x4_to_f16x4(r4.z, a[8 * c + 4], a[8 * c + 5]);
+                        i8x4_to_f16x4(r4.w, a[8 * c + 6], a[8 * c + 7]);
+                    }
+                    tmem_st16(tmem + lane_base + s * 32 + half * 16, a);
+                }
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.afull[s]));
             }
         }
-    } else if (warp >= kWarpEpi0) {
+    } else if (kTok != kTokF16 && warp >= kWarpTok0) {
+        if constexpr (kTok != kTokF16) regs_dec<72>();
+        // token warps: thread t takes the 16-byte chunk cl (8 channels) of rows
+        // r0, r0 + 16, ... of each k-block; r & 7 is the same for all of them,
+        // so the chunk's place under the 128-byte swizzle, cl ^ (r & 7), is fixed
+        const int t = (int)threadIdx.x - kWarpTok0 * 32;
+        const int cl = t & 7, r0 = t >> 3;
+        const int cp = (cl ^ (r0 & 7)) << 4;
+        uint32_t it = 0;
+        bool ok = true;
+        for (int p = 0; p < sch.count && ok; ++p) {
+            int u, pk0, pk1;
+            sch.piece(p, u, pk0, pk1);
+            for (int kb = pk0; kb < pk1; ++kb, ++it) {
+                const int s = it % kStages;
+                const uint32_t ph = (it / kStages) & 1;
+                float2 nz[4], rr[4];
+                if constexpr (kTok == kTokX) {
+                    // channels past K (zero-filled by the copy) get z = r = 0: code 0
+                    const int k0 = kb * kBK + cl * 8;
+                    float4 z0 = make_float4(0.f, 0.f, 0.f, 0.f), z1 = z0, q0 = z0, q1 = z0;
+                    if (k0 < K) {
+                        z0 = __ldg(reinterpret_cast<const float4 *>(xz + k0));
+                        z1 = __ldg(reinterpret_cast<const float4 *>(xz + k0) + 1);
+                        q0 = __ldg(reinterpret_cast<const float4 *>(xr + k0));
+                        q1 = __ldg(reinterpret_cast<const float4 *>(xr + k0) + 1);
+                    }
+                    nz[0] = make_float2(-z0.x, -z0.y); nz[1] = make_float2(-z0.z, -z0.w);
+                    nz[2] = make_float2(-z1.x, -z1.y); nz[3] = make_float2(-z1.z, -z1.w);
+                    rr[0] = make_float2(q0.x, q0.y); rr[1] = make_float2(q0.z, q0.w);
+                    rr[2] = make_float2(q1.x, q1.y); rr[3] = make_float2(q1.z, q1.w);
+                }
+                if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
+                uint8_t *bt = S.b[s] + cp;
+                if constexpr (kTok == kTokI8) {
+                    uint2 v[BN / 16];
+#pragma unroll
+                    for (int i = 0; i < BN / 16; ++i)
+                        v[i] = *reinterpret_cast<const uint2 *>(S.bs[s % (kTok == kTokI8 ? kStages : 1)] +
+                                                                (r0 + 16 * i) * 64 + cl * 8);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&S.empty[s]));  // staging read
+#pragma unroll
+                    for (int i = 0; i < BN / 16; ++i)
+                        *reinterpret_cast<uint4 *>(bt + (r0 + 16 * i) * 128) = i8x8_to_f16x8(v[i]);
+                } else {
+#pragma unroll
+                    for (int i0 = 0; i0 < BN / 16; i0 += 4) {
+                        uint4 v[4];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) v[i] = *reinterpret_cast<const uint4 *>(bt + (r0 + 16 * (i0 + i)) * 128);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            *reinterpret_cast<uint4 *>(bt + (r0 + 16 * (i0 + i)) * 128) =
+                                quantize_f16x8(v[i], nz, rr, qmax_in);
+                    }
+                }
+                fence_proxy_async_smem();  // these stores before the tensor core's reads of b[]
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&S.bfull[s]));
+            }
+        }
+    } else {
+        if constexpr (kTok != kTokF16) regs_inc<144>();
         constexpr int CPW = BN / 2;              // accumulator columns per epilogue warp
         constexpr int PIECE = CPW < 32 ? CPW : 32;
         const int e = warp - kWarpEpi0;
@@ -988,21 +1066,29 @@ bool make_tmap_3d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, uin
 
 int pair_max_clusters();
 
-template <int BN, bool kS32, bool kAsym, bool kQOut>
+template <int BN, bool kS32, bool kAsym, bool kQOut, int kTok>
 cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
+    // token tiles: BN rows x 64 channels of fp16 codes or fp16 activations
+    // (128-byte swizzle, the MMA's layout) or of int8 codes (unswizzled, widened
+    // by the token warps); weights: 128 rows x 64 int8 (64-byte swizzle)
     CUtensorMap tm_q, tm_w;
-    if (!make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
-                      (uint64_t)a.K * 2, kBK, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
-                      kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
+    const bool qmap = kTok == kTokI8
+                          ? make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.q, (uint64_t)a.K, (uint64_t)a.M,
+                                         (uint64_t)a.K, kBK, BN, CU_TENSOR_MAP_SWIZZLE_NONE)
+                          : make_tmap_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
+                                         (uint64_t)(kTok == kTokX ? a.ldx : a.K) * 2, kBK, BN,
+                                         CU_TENSOR_MAP_SWIZZLE_128B);
+    if (!qmap || !make_tmap_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N,
+                               (uint64_t)a.K, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
         return cudaErrorInvalidValue;
     // at least 120 KB so two CTAs never share an SM (each takes all 512 TMEM columns)
-    const size_t smem = sizeof(Smem<BN>) + 1024 > 120 * 1024 ? sizeof(Smem<BN>) + 1024 : 120 * 1024;
+    using SmemT = Smem<BN, kTok>;
+    const size_t smem = sizeof(SmemT) + 1024 > 120 * 1024 ? sizeof(SmemT) + 1024 : 120 * 1024;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32, kAsym, kQOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)smem);
+        attr_err = cudaFuncSetAttribute(linear_kernel<BN, kS32, kAsym, kQOut, kTok>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int64_t tiles = ((a.M + BN - 1) / BN) * ((a.N + kBM - 1) / kBM);
@@ -1019,9 +1105,9 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
                          whole - shared >= kStreamKMinSaving && tiles * nkb < ((int64_t)1 << 30);
     const int grid = streamk ? workers : (int)(tiles < num_sms() ? tiles : num_sms());
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
-    return launch_kernel(linear_kernel<BN, kS32, kAsym, kQOut>, dim3(grid), dim3(kThreads), smem, st, a.pdl, tm_q, tm_w,
-                         a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, a.s_tok, a.zc,
-                         a.rowsum, a.zq, a.rq, a.qmax_out, ws, pairs);
+    return launch_kernel(linear_kernel<BN, kS32, kAsym, kQOut, kTok>, dim3(grid), dim3(lin_threads<kTok>()), smem,
+                         st, a.pdl, tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb,
+                         a.relu, a.s_tok, a.zc, a.rowsum, a.zq, a.rq, a.qmax_out, ws, pairs, a.xz, a.xr, a.qmax_in);
 }
 
 // Clusters of the pair kernel that fit on the device at once (one per two SMs).
@@ -1034,7 +1120,8 @@ int pair_max_clusters() {
     if (dev_cached == dev) return value;
     const size_t smem = sizeof(SmemPair) + 1024;
     int n = 0;
-    if (cudaFuncSetAttribute(linear_pair_kernel<false, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+    if (cudaFuncSetAttribute(linear_pair_kernel<false, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) ==
         cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 256);
@@ -1098,9 +1185,20 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
 // M <= 16 goes to the decode kernel (gemv.cu) before this dispatch.
 template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
-    if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut>(a, kcb, st);
-    if (a.M <= 128 || a.K % 128 != 0) return run_linear<128, kS32, kAsym, kQOut>(a, kcb, st);
+    if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
+    if (a.M <= 128 || a.K % 128 != 0) return run_linear<128, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
     return run_linear_pair<kS32, kAsym, kQOut>(a, kcb, st);
+}
+
+// int8 codes (any M > 16) and fp16 activations quantized in the kernel
+// (16 < M <= 128) go to linear_kernel with its token warps.
+template <int kTok>
+cudaError_t dispatch_tok(const LinearArgs &a, int kcb, cudaStream_t st) {
+    if (a.out_s32)
+        return a.M <= 64 ? run_linear<64, true, false, false, kTok>(a, kcb, st)
+                         : run_linear<128, true, false, false, kTok>(a, kcb, st);
+    return a.M <= 64 ? run_linear<64, false, false, false, kTok>(a, kcb, st)
+                     : run_linear<128, false, false, false, kTok>(a, kcb, st);
 }
 
 }  // namespace
@@ -1193,6 +1291,8 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
         d.workspace_bytes = room ? a.workspace_bytes - off : 0;
         return launch_linear_gemv(d, kcb, st);
     }
+    if (a.q_fmt == kCodesI8) return dispatch_tok<kTokI8>(a, kcb, st);
+    if (a.q_fmt == kActF16) return dispatch_tok<kTokX>(a, kcb, st);
     if (a.out_s32) return dispatch_bn<true, false, false>(a, kcb, st);
     if (a.zq) return dispatch_bn<false, false, true>(a, kcb, st);
     return a.zc ? dispatch_bn<false, true, false>(a, kcb, st) : dispatch_bn<false, false, false>(a, kcb, st);

@@ -66,7 +66,11 @@ constexpr int kGvWBox = kGvRows * 128;           // weight box: 128 rows x 128 b
 constexpr int kGvWBytes = 2 * kGvWBox;            // weights of a stage (two boxes)
 constexpr int kGvMaxStages = 8;
 constexpr int kGvSmemBudget = 224 * 1024;
-constexpr int kGvHeader = 256;                    // barriers, counters, flags
+constexpr int kGvHeader = 384;                    // barriers, counters, flags
+// Token box of a stage: fp16 codes (kGvF16) as copied; int8 codes (kGvI8),
+// widened when the fragments are read; or fp16 activations (kGvX) that the
+// CTA's warps quantize in place (z, r per channel) before any warp reads them.
+constexpr int kGvF16 = 0, kGvI8 = 1, kGvX = 2;
 constexpr int kGvPdlUnits = 2;                    // units whose weights load before a programmatic wait
 constexpr int kGvSlotInts = kGvRows * 32;         // workspace ints per split tile (32 tokens x 128 rows)
 
@@ -80,6 +84,8 @@ struct GvParams {
     unsigned long long *flags;     // [grid] launch epoch once a CTA's slot is complete
     unsigned long long *ctl;       // {epoch of the last launch, CTAs done with this one}
     int pdl;                       // launched as a programmatic dependent of the codes' producer
+    const float *xz, *xr;          // kGvX: z, r [K]
+    int qmax_in;                   // kGvX: qmax of the codes
     int *status;        // device status word
     int M, N, K, ldy, kcb, relu;
     int nks;            // units per tile
@@ -88,17 +94,6 @@ struct GvParams {
     int grid;
     int whole;          // ranges of whole tiles (no workspace)
 };
-
-__device__ __forceinline__ void i8x4_to_f16x4_gv(uint32_t w, uint32_t &lo, uint32_t &hi) {
-    const uint32_t u = w ^ 0x80808080u;
-    const uint32_t a = __byte_perm(u, 0x64646464u, 0x4140);
-    const uint32_t b = __byte_perm(u, 0x64646464u, 0x4342);
-    const __half2 bias = __half2half2(__ushort_as_half(0x6480));  // 1152
-    const __half2 ha = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
-    const __half2 hb = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
-    lo = *reinterpret_cast<const uint32_t *>(&ha);
-    hi = *reinterpret_cast<const uint32_t *>(&hb);
-}
 
 __device__ __forceinline__ void mma_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
     asm volatile(
@@ -150,8 +145,8 @@ __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32
     }
 }
 
-// TN token groups of 8 (the MMA's n8).
-template <int TN, bool kS32>
+// TN token groups of 8 (the MMA's n8); kTokG: the token box's format.
+template <int TN, bool kS32, int kTokG>
 __global__ void __launch_bounds__(kGvThreads, 1)
     linear_gemv_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_a,
                        const GvParams p) {
@@ -163,6 +158,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     unsigned *loads = done + kGvMaxStages;                                // units loaded into a slot, ever
     volatile int *abort = reinterpret_cast<volatile int *>(loads + kGvMaxStages);
     unsigned long long *epoch_s = reinterpret_cast<unsigned long long *>(base + 192);  // this launch's epoch
+    uint64_t *qready = reinterpret_cast<uint64_t *>(base + 256);  // kGvX: the slot's codes are quantized
     int32_t(*red)[kGvRows + 1] = reinterpret_cast<int32_t(*)[kGvRows + 1]>(base + kGvHeader);  // [TN*8]
     uint8_t *ring = base + ((kGvHeader + p.red_bytes + 1023) & ~1023);
 
@@ -172,7 +168,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     const int M = p.M, N = p.N, K = p.K, nks = p.nks;
     const int64_t tile0 = u_begin / nks;
     const int ks0 = (int)(u_begin - tile0 * nks);
-    const uint32_t abytes = (uint32_t)M * kGvKS * 2;  // activation box
+    const uint32_t abytes = (uint32_t)M * kGvKS * (kTokG == kGvI8 ? 1 : 2);  // token box
     uint64_t pol_w = 0, pol_a = 0;
 
     // Load unit (tile, ks) into `slot`, completing on full[slot]: the weight
@@ -204,6 +200,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         tma_prefetch_desc(&tm_a);
         for (int s = 0; s < S; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&qready[s]), kGvWarps);
             done[s] = 0;
             loads[s] = 0;
         }
@@ -256,7 +253,8 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     // swizzles (16-byte chunk c stored at c ^ (row % 8)) fall in different bank halves.
     const int sg = (r >> 1) + 4 * (r & 1);
     const int w_off = (kw >> 7) * kGvWBox + (32 * rp + sg) * 128 + ((((kw & 127) >> 4) + t) ^ sg) * 16;
-    const int a_off = kGvWBytes + r * (2 * kGvKS) + 2 * (kw + 16 * t);
+    constexpr int kEl = kTokG == kGvI8 ? 1 : 2;  // bytes per token value in the box
+    const int a_off = kGvWBytes + r * (kEl * kGvKS) + kEl * (kw + 16 * t);
 
     float acc[2][TN][4];
 #pragma unroll
@@ -291,7 +289,36 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         const int64_t seg_begin = u, seg_end = min(u_end, u + (nks - ks));
         const int mine = (int)(seg_end - u);
         for (; u < seg_end; ++u, ++ks) {
-            const bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[slot]), phase, abort, p.status));
+            bool ok;
+            if constexpr (kTokG == kGvX) {
+                // thread j quantizes the 16-byte chunk j (8 channels of one token) of the
+                // box; z, r are fetched before the wait; channels past K get code 0
+                const int j = threadIdx.x;
+                const int k0 = ks * kGvKS + (j & 31) * 8;
+                float2 nz[4], rq[4];
+                float4 z0 = make_float4(0.f, 0.f, 0.f, 0.f), z1 = z0, q0 = z0, q1 = z0;
+                if (j < M * 32 && k0 < K) {
+                    z0 = __ldg(reinterpret_cast<const float4 *>(p.xz + k0));
+                    z1 = __ldg(reinterpret_cast<const float4 *>(p.xz + k0) + 1);
+                    q0 = __ldg(reinterpret_cast<const float4 *>(p.xr + k0));
+                    q1 = __ldg(reinterpret_cast<const float4 *>(p.xr + k0) + 1);
+                }
+                nz[0] = make_float2(-z0.x, -z0.y); nz[1] = make_float2(-z0.z, -z0.w);
+                nz[2] = make_float2(-z1.x, -z1.y); nz[3] = make_float2(-z1.z, -z1.w);
+                rq[0] = make_float2(q0.x, q0.y); rq[1] = make_float2(q0.z, q0.w);
+                rq[2] = make_float2(q1.x, q1.y); rq[3] = make_float2(q1.z, q1.w);
+                ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[slot]), phase, abort, p.status));
+                if (ok && j < M * 32) {
+                    uint4 *c = reinterpret_cast<uint4 *>(ring + (size_t)slot * p.stage_bytes + kGvWBytes +
+                                                         (j >> 5) * (2 * kGvKS) + (j & 31) * 16);
+                    *c = quantize_f16x8(*c, nz, rq, p.qmax_in);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&qready[slot]));
+                ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&qready[slot]), phase, abort, p.status)) && ok;
+            } else {
+                ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[slot]), phase, abort, p.status));
+            }
             // past K the boxes hold zeros; skip windows that lie wholly past it
             if (ok && kw < K - ks * kGvKS) {
                 if (in_chunk == p.kcb) {
@@ -311,8 +338,14 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 for (int tn = 0; tn < TN; ++tn) {
                     uint4 lo = make_uint4(0, 0, 0, 0), hi = make_uint4(0, 0, 0, 0);
                     if (tgv[tn] && tok[tn]) {
-                        lo = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * (2 * kGvKS));
-                        hi = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * (2 * kGvKS) + 16);
+                        if constexpr (kTokG == kGvI8) {
+                            const uint4 v = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * kGvKS);
+                            lo = i8x8_to_f16x8(make_uint2(v.x, v.y));
+                            hi = i8x8_to_f16x8(make_uint2(v.z, v.w));
+                        } else {
+                            lo = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * (2 * kGvKS));
+                            hi = *reinterpret_cast<const uint4 *>(st + a_off + tn * 8 * (2 * kGvKS) + 16);
+                        }
                     }
                     x[tn][0] = lo.x; x[tn][1] = lo.y; x[tn][2] = lo.z; x[tn][3] = lo.w;
                     x[tn][4] = hi.x; x[tn][5] = hi.y; x[tn][6] = hi.z; x[tn][7] = hi.w;
@@ -325,8 +358,8 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                     const uint32_t w1[4] = {wv[g][1].x, wv[g][1].y, wv[g][1].z, wv[g][1].w};
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        i8x4_to_f16x4_gv(w0[j], a[j][0], a[j][2]);
-                        i8x4_to_f16x4_gv(w1[j], a[j][1], a[j][3]);
+                        i8x4_to_f16x4(w0[j], a[j][0], a[j][2]);
+                        i8x4_to_f16x4(w1[j], a[j][1], a[j][3]);
                     }
 #pragma unroll
                     for (int tn = 0; tn < TN; ++tn) {
@@ -426,26 +459,27 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     }
 }
 
-template <int TN, bool kS32>
+template <int TN, bool kS32, int kTokG>
 cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvParams &base, cudaStream_t st,
                      bool pdl) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_gemv_kernel<TN, kS32>,
+        attr_err = cudaFuncSetAttribute(linear_gemv_kernel<TN, kS32, kTokG>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kGvSmemBudget);
     });
     if (attr_err != cudaSuccess) return attr_err;
     GvParams p = base;
     p.red_bytes = (TN * 8 * (kGvRows + 1) * 4 + 127) / 128 * 128;
-    p.stage_bytes = (kGvWBytes + p.M * kGvKS * 2 + 1023) & ~1023;
+    p.stage_bytes = (kGvWBytes + p.M * kGvKS * (kTokG == kGvI8 ? 1 : 2) + 1023) & ~1023;
     const int ring_off = (kGvHeader + p.red_bytes + 1023) & ~1023;
     const int room = kGvSmemBudget - 1024 - ring_off;
     p.stages = room / p.stage_bytes;
     if (p.stages > kGvMaxStages) p.stages = kGvMaxStages;
     if (p.stages < 2) return cudaErrorInvalidConfiguration;
     const size_t smem = 1024 + ring_off + (size_t)p.stages * p.stage_bytes;
-    return launch_kernel(linear_gemv_kernel<TN, kS32>, dim3(p.grid), dim3(kGvThreads), smem, st, pdl, tm_w, tm_a, p);
+    return launch_kernel(linear_gemv_kernel<TN, kS32, kTokG>, dim3(p.grid), dim3(kGvThreads), smem, st, pdl, tm_w,
+                         tm_a, p);
 }
 
 }  // namespace
@@ -458,11 +492,14 @@ size_t gemv_workspace_bytes() {
 cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     // weights: boxes of 128 rows x 128 int8 (128-byte swizzle); codes: boxes of
     // all M tokens x 256 fp16 (no swizzle); both zero-filled outside the arrays
+    // (int8 codes: boxes of all M tokens x 256 int8; fp16 activations: rows of ldx elements)
     CUtensorMap tm_w, tm_a;
+    const bool i8 = a.q_fmt == kCodesI8;
+    const uint64_t arow = i8 ? (uint64_t)a.K : (uint64_t)(a.q_fmt == kActF16 ? a.ldx : a.K) * 2;
     if (!tensor_map_2d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K,
                        128, kGvRows, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !tensor_map_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, (uint64_t)a.K, (uint64_t)a.M,
-                       (uint64_t)a.K * 2, kGvKS, (uint32_t)a.M, CU_TENSOR_MAP_SWIZZLE_NONE))
+        !tensor_map_2d(&tm_a, i8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q,
+                       (uint64_t)a.K, (uint64_t)a.M, arow, kGvKS, (uint32_t)a.M, CU_TENSOR_MAP_SWIZZLE_NONE))
         return cudaErrorInvalidValue;
     GvParams p{};
     p.sw = a.sw;
@@ -474,6 +511,9 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     p.rq = a.rq;
     p.qmax_out = a.qmax_out;
     p.pdl = a.pdl ? 1 : 0;
+    p.xz = a.xz;
+    p.xr = a.xr;
+    p.qmax_in = a.qmax_in;
     p.out = a.out;
     p.status = device_status_word();
     if (!p.status) return cudaErrorUnknown;
@@ -510,9 +550,18 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
         p.grid = (int)(p.ntiles < sms ? p.ntiles : sms);
     }
     const bool d = a.pdl;
-    if (a.M <= 8) return a.out_s32 ? run_gemv<1, true>(tm_w, tm_a, p, st, d) : run_gemv<1, false>(tm_w, tm_a, p, st, d);
-    if (a.M <= 16) return a.out_s32 ? run_gemv<2, true>(tm_w, tm_a, p, st, d) : run_gemv<2, false>(tm_w, tm_a, p, st, d);
-    return cudaErrorInvalidValue;  // more than 16 tokens go to the tcgen05 kernels
+    if (a.M > 16) return cudaErrorInvalidValue;  // more than 16 tokens go to the tcgen05 kernels
+    const bool one = a.M <= 8;
+    if (a.q_fmt == kActF16)
+        return one ? run_gemv<1, false, kGvX>(tm_w, tm_a, p, st, d) : run_gemv<2, false, kGvX>(tm_w, tm_a, p, st, d);
+    if (i8) {
+        if (a.out_s32)
+            return one ? run_gemv<1, true, kGvI8>(tm_w, tm_a, p, st, d) : run_gemv<2, true, kGvI8>(tm_w, tm_a, p, st, d);
+        return one ? run_gemv<1, false, kGvI8>(tm_w, tm_a, p, st, d) : run_gemv<2, false, kGvI8>(tm_w, tm_a, p, st, d);
+    }
+    if (a.out_s32)
+        return one ? run_gemv<1, true, kGvF16>(tm_w, tm_a, p, st, d) : run_gemv<2, true, kGvF16>(tm_w, tm_a, p, st, d);
+    return one ? run_gemv<1, false, kGvF16>(tm_w, tm_a, p, st, d) : run_gemv<2, false, kGvF16>(tm_w, tm_a, p, st, d);
 }
 
 }  // namespace ot

@@ -54,6 +54,59 @@ __device__ __forceinline__ float2 f2_fma(float2 a, float2 b, float2 c) {
 }
 
 // ---------------------------------------------------------------------------
+// integer codes held exactly in fp16
+// ---------------------------------------------------------------------------
+// 4 signed int8 codes -> two fp16x2 words (exact).  Each byte b is biased to
+// u = b + 128 and placed under the fp16 exponent of 1024 (bit pattern
+// 0x6400 | u = 1024 + u, unit spacing in [1024, 2048)); subtracting 1152
+// leaves b exactly.
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t u = w ^ 0x80808080u;
+    const uint32_t a = __byte_perm(u, 0x64646464u, 0x4140);
+    const uint32_t b = __byte_perm(u, 0x64646464u, 0x4342);
+    const __half2 bias = __half2half2(__ushort_as_half(0x6480));  // 1152
+    const __half2 ha = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
+    const __half2 hb = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
+    lo = *reinterpret_cast<const uint32_t *>(&ha);
+    hi = *reinterpret_cast<const uint32_t *>(&hb);
+}
+
+// 8 int8 codes (two words, k ascending) -> 8 fp16 codes (four fp16x2 words).
+__device__ __forceinline__ uint4 i8x8_to_f16x8(uint2 v) {
+    uint4 o;
+    i8x4_to_f16x4(v.x, o.x, o.y);
+    i8x4_to_f16x4(v.y, o.z, o.w);
+    return o;
+}
+
+// Two integers |c| <= 128 as an fp16x2 word: 1152 + c lies in [1024, 2048),
+// where fp16 has unit spacing, so its bit pattern is 0x6400 | (128 + c);
+// subtracting 1152 in fp16 is exact.
+__device__ __forceinline__ uint32_t f16x2_of_codes(int c0, int c1) {
+    const uint32_t bits = (uint32_t)(0x6480 + c0) | ((uint32_t)(0x6480 + c1) << 16);
+    const __half2 v = __hsub2(*reinterpret_cast<const __half2 *>(&bits), __half2half2(__ushort_as_half(0x6480)));
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// Per-channel code of Eq. 6 / Eq. 7 for 8 consecutive channels held as fp16
+// x (one 16-byte word): c = clamp(round_half_even((x - z) * r), -qmax, qmax),
+// the subtraction and the product each rounded to fp32 (two values per
+// f32x2 instruction; cvt.rni maps NaN to 0), returned as fp16 codes.
+// nz holds -z (x - z == x + (-z) exactly).
+__device__ __forceinline__ uint4 quantize_f16x8(uint4 xv, const float2 (&nz)[4], const float2 (&r)[4], int qmax) {
+    const __half2 *h = reinterpret_cast<const __half2 *>(&xv);
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const float2 u = f2_mul(f2_add(__half22float2(h[j]), nz[j]), r[j]);
+        const int c0 = max(-qmax, min(qmax, __float2int_rn(u.x)));
+        const int c1 = max(-qmax, min(qmax, __float2int_rn(u.y)));
+        o[j] = f16x2_of_codes(c0, c1);
+    }
+    return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// ---------------------------------------------------------------------------
 // mbarrier
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {

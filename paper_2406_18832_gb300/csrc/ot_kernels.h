@@ -55,7 +55,17 @@ struct LinearArgs {
     int qmax_out;             // with zq: the next layer's qmax
     bool pdl;                 // launched as a programmatic dependent of the kernel that wrote q (weights are
                               // read before that kernel ends, codes only after)
+    int q_fmt = 0;            // kCodesF16: q holds fp16 codes; kCodesI8: int8 codes; kActF16: fp16
+                              // activations [M, ldx] that the kernel quantizes with xz, xr, qmax_in
+    const float *xz = nullptr, *xr = nullptr;  // kActF16: z, r [K]
+    int64_t ldx = 0;          // kActF16: row stride of q
+    int qmax_in = 0;          // kActF16: qmax of the codes
 };
+constexpr int kCodesF16 = 0, kCodesI8 = 1, kActF16 = 2;
+// ot_linear_fused quantizes inside the linear's token producer up to this
+// many tokens (decode kernel and linear_kernel); above it the prefill kernel
+// reads codes written by the quantize kernel.
+constexpr int64_t kFusedInKernelMaxTokens = 128;
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();
 // Fixed scratch of ot_linear_noalloc (a static device array in gemm.cu).

@@ -60,8 +60,8 @@ def test_status_strings_and_version(lib):
 def _linear_args(handle):
     P, I64, I = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
     S = ctypes.c_size_t
-    handle.ot_linear.argtypes = [P, I64, I64, P, P, P, I64, I, I, P, I64, I, P, S, P]
-    handle.ot_linear_s32.argtypes = [P, I64, I64, P, I64, I, I, P, P, S, P]
+    handle.ot_linear.argtypes = [P, I, I64, I64, P, P, P, I64, I, I, P, I64, I, P, S, P]
+    handle.ot_linear_s32.argtypes = [P, I, I64, I64, P, I64, I, I, P, P, S, P]
     handle.ot_quantize_act.argtypes = [P, I64, I64, I64, P, P, I, P, I, P]
     handle.ot_calibrate.argtypes = [P, I64, I64, I64, P, P, I, P]
     handle.ot_fold_weights.argtypes = [P, P, I, I, P, P, I64, I64, I, P, P, P, P, P, P, P]
@@ -84,23 +84,27 @@ def test_validation_rejects_bad_arguments_before_launch(lib):
     _linear_args(handle)
     INV, UNS = 1, 2
     # K not a multiple of 16
-    assert handle.ot_linear(A, 4, 24, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 24, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
     # bits outside [2, 8]
-    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 9, 8, A, 16, 0, None, 0, None) == INV
-    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 8, 1, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, A2, A, A, 16, 9, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, A2, A, A, 16, 8, 1, A, 16, 0, None, 0, None) == INV
     # misaligned operands
-    assert handle.ot_linear(A + 2, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
-    assert handle.ot_linear(A, 4, 64, A2 + 8, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A + 2, 1, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, A2 + 8, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
     # null pointers, ldy < N, negative sizes
-    assert handle.ot_linear(A, 4, 64, None, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
-    assert handle.ot_linear(A, 4, 64, A2, None, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
-    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 8, 8, A, 8, 0, None, 0, None) == INV
-    assert handle.ot_linear(A, -1, 64, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, None, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, A2, None, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, A2, A, A, 16, 8, 8, A, 8, 0, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, -1, 64, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
     # K beyond the int32 accumulator for W8A8 (K * 127 * 127 >= 2^31)
-    assert handle.ot_linear(A, 4, 133152, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == UNS
-    assert handle.ot_linear_s32(A, 4, 24, A2, 16, 8, 8, A, None, 0, None) == INV
+    assert handle.ot_linear(A, 1, 4, 133152, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == UNS
+    assert handle.ot_linear_s32(A, 1, 4, 24, A2, 16, 8, 8, A, None, 0, None) == INV
+    # code format other than OT_CODE_I8 / OT_CODE_F16; int8 codes keep the same checks
+    assert handle.ot_linear(A, 7, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear(A + 8, 0, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, None, 0, None) == INV
+    assert handle.ot_linear_s32(A, 0, 4, 24, A2, 16, 8, 8, A, None, 0, None) == INV
     # workspace must be 16-byte aligned
-    assert handle.ot_linear(A, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, A + 8, 1 << 20, None) == INV
+    assert handle.ot_linear(A, 1, 4, 64, A2, A, A, 16, 8, 8, A, 16, 0, A + 8, 1 << 20, None) == INV
     # quantize: bad format, unaligned z, ldx < K
     assert handle.ot_quantize_act(A, 4, 64, 64, A, A, 8, A2, 7, None) == INV
     assert handle.ot_quantize_act(A, 4, 64, 64, A + 4, A, 8, A2, 1, None) == INV

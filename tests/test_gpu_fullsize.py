@@ -14,8 +14,10 @@ Per layer, on the GPU and in the oracle:
     weight tile (first and last channel of each, and of each 32-lane quarter),
     so every (token tile, weight tile) pair -- stream-K split tiles included,
     whose accumulators hold every k-range -- contributes outputs.
-The oracle runs its C functions over row ranges in host threads (identical
-arithmetic, bit-identical results)."""
+The int8-code input and the fused call (quantization inside the linear up to
+128 tokens) must give the same bits as the checked output.  The oracle runs
+its C functions over row ranges in host threads (identical arithmetic,
+bit-identical results)."""
 import numpy as np
 import pytest
 import torch
@@ -117,6 +119,21 @@ def _check_tokens(cfg, li, layer, ql, o, M, bits, full: bool):
     assert_f16_close(gy, oy, what=f"y M={M}")
     # one fp32 fma rounded once to fp16 on both sides: bit-identical
     assert np.array_equal(gy.view(np.uint16), oy.view(np.uint16)), f"fp16 outputs M={M}"
+
+    # the same layer from int8 codes, and with the quantization inside the
+    # linear (ot_linear_fused): the same bits as the checked output
+    q8 = torch.empty(M, layer.K, dtype=torch.int8, device=dev)
+    binding.ot_quantize_act(x, ql.z, ql.r, bits_a, q8, binding.OT_CODE_I8)
+    y8 = torch.empty_like(y)
+    binding.ot_linear(q8, ql.qw, ql.sw, ql.b_fold, bits_a, bits_w, y8, relu=layer.relu_out)
+    yf = torch.empty_like(y)
+    binding.ot_linear_fused(x, ql.z, ql.r, bits_a, ql.qw, ql.sw, ql.b_fold, bits_w, torch.empty_like(q), yf,
+                            relu=layer.relu_out)
+    torch.cuda.synchronize()
+    assert binding.ot_get_device_status() == binding.OT_OK
+    assert np.array_equal(q8.cpu().numpy(), oq), f"int8 codes M={M}"
+    assert torch.equal(y8, y), f"int8-code linear M={M}"
+    assert torch.equal(yf, y), f"fused linear M={M}"
 
 
 # (config, layer, bits, token counts, token counts checked in full)
