@@ -635,12 +635,18 @@ def bench_token_sweep(dev, peaks, reps: int = 20):
                     for i in range(n):
                         binding.ot_linear_fused(x, z0, r1, 6, qws[i % copies], sw, bf, 6, qs, y, workspace=ws)
 
+                def calls_producer():
+                    for i in range(n):
+                        binding.ot_linear_fused(x, z0, r1, 6, qws[i % copies], sw, bf, 6, qs, y, workspace=ws,
+                                                mode=binding.OT_FUSE_PRODUCER)
+
                 def calls_two():
                     for i in range(n):
                         binding.ot_quantize_act(x, z0, r1, 6, qs, binding.OT_CODE_F16)
                         binding.ot_linear(qs, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
                 pt["int8_codes_us"] = round(_graph_ms(calls8, n) * 1e3, 2)
                 pt["fused_us"] = round(_graph_ms(calls_fused, n) * 1e3, 2)
+                pt["fused_in_producer_us"] = round(_graph_ms(calls_producer, n) * 1e3, 2)
                 pt["quantize_then_linear_us"] = round(_graph_ms(calls_two, n) * 1e3, 2)
                 del q8, x, qs
             out.append(pt)
@@ -649,8 +655,10 @@ def bench_token_sweep(dev, peaks, reps: int = 20):
     del ws
     torch.cuda.empty_cache()
     return {"workload": "opt-13b QKV and fc2, Int6, 1-4096 tokens", "timing": "CUDA graph replay, rotating weights",
-            "up_to_128_tokens": "int8_codes_us: ot_linear on int8 codes; fused_us: ot_linear_fused (fp16 X in, "
-                                "quantized inside the linear); quantize_then_linear_us: ot_quantize_act + ot_linear",
+            "up_to_128_tokens": "int8_codes_us: ot_linear on int8 codes; fused_us: ot_linear_fused (default: the "
+                                "quantize kernel, the linear its programmatic dependent); fused_in_producer_us: "
+                                "ot_linear_fused with the quantization in the linear's token producer; "
+                                "quantize_then_linear_us: ot_quantize_act + ot_linear",
             "per_point": out}
 
 

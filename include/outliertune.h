@@ -318,31 +318,43 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
                          void *y_f16, int64_t ldy, int relu, void *workspace,
                          size_t workspace_bytes, void *stream);
 
+/* How ot_linear_fused joins the activation quantization to the product. */
+typedef enum {
+    OT_FUSE_AUTO = 0,      /* the faster form for the call (measured on GB300:
+                              OT_FUSE_PDL at every token count) */
+    OT_FUSE_PRODUCER = 1,  /* the linear's token producer quantizes X itself
+                              (M <= 128 only) */
+    OT_FUSE_PDL = 2        /* the quantize kernel writes the codes, the linear
+                              runs as its programmatic dependent */
+} ot_fuse_mode;
+
 /*
  * ot_linear_fused -- the per-channel quantization of X (Eq. 6-7) and the
  * linear in one call: q = codes of X, y = fp16(fma(sum_k q qw, sw_n, b'_n)),
  * ReLU if relu; the result is bit-identical to ot_quantize_act followed by
- * ot_linear.
- *   - M <= 128: the linear's own token producer reads fp16 X and quantizes
- *     each tile in shared memory before the tensor cores read it (the
- *     quantization inside the GEMM's operand producer): one kernel, and the
- *     codes never reach HBM; q_f16 is not written.
- *   - M > 128: the quantize kernel writes the codes to q_f16, and the linear
- *     is launched as its programmatic dependent, so the linear's weight loads
- *     and set-up overlap the quantization and only its reads of the codes wait
- *     for it (at prefill sizes each token tile is read by every weight tile,
- *     so quantizing once beats quantizing in every CTA).
+ * ot_linear, in either form:
+ *   - OT_FUSE_PDL: the quantize kernel writes the codes to q_f16 and the
+ *     linear is launched as its programmatic dependent, so the linear's
+ *     weight loads and set-up overlap the quantization and only its reads of
+ *     the codes wait for it.
+ *   - OT_FUSE_PRODUCER (M <= 128): the linear's own token producer reads fp16
+ *     X with z and r and quantizes each tile in shared memory before the
+ *     tensor cores read it (the quantization inside the GEMM's operand
+ *     producer; one kernel, q_f16 not written).  Each token tile is then
+ *     quantized once per weight tile instead of once in all, which on GB300
+ *     costs more than the HBM round trip of the codes it saves.
  * x_f16 fp16 [M, ldx] (ldx >= K, ldx % 8 == 0, 16-byte aligned); z, r fp32 [K]
  * (16-byte aligned); q_f16: caller scratch fp16 [M, K], dense, 16-byte
- * aligned, whose contents are unspecified afterwards; the remaining arguments
- * as ot_linear.  Same validation and errors as the two calls; M == 0
- * launches nothing.
+ * aligned, whose contents are unspecified afterwards; mode an ot_fuse_mode
+ * (OT_ERR_UNSUPPORTED for OT_FUSE_PRODUCER with M > 128); the remaining
+ * arguments as ot_linear.  Same validation and errors as the two calls;
+ * M == 0 launches nothing.
  */
 ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z,
                           const float *r, int bits_a, const int8_t *qw, const float *sw,
                           const float *b_fold, int64_t N, int bits_w, void *q_f16, void *y_f16,
-                          int64_t ldy, int relu, void *workspace, size_t workspace_bytes,
-                          void *stream);
+                          int64_t ldy, int relu, int mode, void *workspace,
+                          size_t workspace_bytes, void *stream);
 
 /*
  * ot_linear_quantize_next -- a linear whose output is the input of the next

@@ -18,6 +18,7 @@ from . import build as _build
 
 OT_OK, OT_ERR_INVALID_ARG, OT_ERR_UNSUPPORTED, OT_ERR_CUDA, OT_ERR_TIMEOUT = range(5)
 OT_CODE_I8, OT_CODE_F16 = 0, 1
+OT_FUSE_AUTO, OT_FUSE_PRODUCER, OT_FUSE_PDL = 0, 1, 2
 
 _lock = threading.Lock()
 _handle = None
@@ -47,7 +48,7 @@ _SIGNATURES = {
     "ot_calibrate_clipped": ([_P, _I64, _I64, _I64, ctypes.c_double, _P, _P, _P], _I),
     "ot_linear_quantize_next": ([_P, _I64, _I64, _P, _P, _P, _I64, _I, _I, _I, _P, _P, _I, _P, _I64, _P,
                                  ctypes.c_size_t, _P], _I),
-    "ot_linear_fused": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _P, _P, _I64, _I, _P, _P, _I64, _I, _P,
+    "ot_linear_fused": ([_P, _I64, _I64, _I64, _P, _P, _I, _P, _P, _P, _I64, _I, _P, _P, _I64, _I, _I, _P,
                          ctypes.c_size_t, _P], _I),
     "ot_get_device_status": ([_P], _I),
     "ot_selftest_wait_timeout": ([_I64, _P], _I),
@@ -244,9 +245,9 @@ def ot_layernorm_quantize(h, gamma_r, beta_r, eps: float, bits_a: int, q, q_form
 
 
 def ot_linear_fused(x, z, r, bits_a: int, qw, sw, b_fold, bits_w: int, q, y, relu: bool = False, workspace=None,
-                    stream=None):
-    """Quantize x and run the linear into y [M, N] in one call; q is fp16 scratch [M, K] (written only
-    above 128 tokens, where the codes go through HBM)."""
+                    stream=None, mode: int = OT_FUSE_AUTO):
+    """Quantize x and run the linear into y [M, N] in one call; q is fp16 scratch [M, K]; mode is an
+    ot_fuse_mode (OT_FUSE_PRODUCER: quantized inside the linear, up to 128 tokens)."""
     M, K, ldx = _rows(x, "x")
     _dense(q, "q")
     _dense(qw, "qw")
@@ -261,7 +262,7 @@ def ot_linear_fused(x, z, r, bits_a: int, qw, sw, b_fold, bits_w: int, q, y, rel
                                   _dev(r, "r", torch.float32), bits_a, _dev(qw, "qw", torch.int8),
                                   _dev(sw, "sw", torch.float32), _dev(b_fold, "b_fold", torch.float32), N, bits_w,
                                   _dev(q, "q", torch.float16), _dev(y, "y", torch.float16), ldy, 1 if relu else 0,
-                                  wp, wb, _stream(stream)), "ot_linear_fused")
+                                  mode, wp, wb, _stream(stream)), "ot_linear_fused")
 
 
 def ot_linear_quantize_next(q, qw, sw, b_fold, bits_a: int, bits_w: int, z_next, r_next, bits_next: int, q_next,

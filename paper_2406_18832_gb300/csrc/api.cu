@@ -236,8 +236,9 @@ ot_status ot_linear_asym(const void *q_f16, int64_t M, int64_t K, const int8_t *
 
 ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, const float *z, const float *r,
                           int bits_a, const int8_t *qw, const float *sw, const float *b_fold, int64_t N, int bits_w,
-                          void *q_f16, void *y_f16, int64_t ldy, int relu, void *workspace, size_t workspace_bytes,
-                          void *stream) {
+                          void *q_f16, void *y_f16, int64_t ldy, int relu, int mode, void *workspace,
+                          size_t workspace_bytes, void *stream) {
+    if (mode != OT_FUSE_AUTO && mode != OT_FUSE_PRODUCER && mode != OT_FUSE_PDL) return OT_ERR_INVALID_ARG;
     if (ldx < K || ldx % 8 != 0) return OT_ERR_INVALID_ARG;
     ot_status v = linear_common(q_f16, M, K, qw, N, bits_a, bits_w, y_f16);
     if (v != OT_OK) return v;
@@ -248,7 +249,8 @@ ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, 
     if (ldy > kIntMax || (M + 63) / 64 > 65535) return OT_ERR_UNSUPPORTED;
     if (M == 0) return OT_OK;
     const cudaStream_t st = as_stream(stream);
-    if (M <= ot::kFusedInKernelMaxTokens) {
+    if (mode == OT_FUSE_PRODUCER && M > ot::kFusedInKernelMaxTokens) return OT_ERR_UNSUPPORTED;
+    if (mode == OT_FUSE_PRODUCER) {
         // the linear's token producer quantizes X itself (no codes in HBM)
         ot::LinearArgs a{x_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
                          workspace, workspace ? workspace_bytes : 0};

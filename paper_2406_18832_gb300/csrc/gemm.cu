@@ -73,6 +73,7 @@ struct alignas(1024) Smem {
     uint8_t b[kStages][BN * 128];   // activation codes, 128-byte swizzled rows
     uint8_t w[kStages][kBM * kBK];  // int8 weight codes, 64-byte swizzled rows
     uint8_t bs[kTok == kTokI8 ? kStages : 1][kTok == kTokI8 ? BN * 64 : 16];  // int8 codes as copied (kTokI8)
+    alignas(16) float zr[kTok == kTokX ? kStages : 1][2][64];  // kTokX: the k-block's z and r, copied with the tiles
     uint64_t full[kStages];         // TMA landed (tx bytes)
     uint64_t empty[kStages];        // stage free: MMA done with b[] + 4 converter warps done with w[]
                                     // (+ kTokI8: 4 token warps done with bs[])
@@ -266,10 +267,18 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
                     const uint32_t ph = (it / kStages) & 1;
                     if (!(ok = mbar_wait_warp(smem_u32(&S.empty[s]), ph ^ 1, abort, &g_status))) break;
                     if (elect_one()) {
-                        mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes);
+                        // kTokX: the k-block's z and r (channels below K only; K % 16 == 0, so the
+                        // byte count stays a multiple of 64)
+                        const uint32_t zr_bytes = kTok == kTokX ? (uint32_t)min(kBK, K - kb * kBK) * 4 : 0;
+                        mbar_arrive_expect_tx(smem_u32(&S.full[s]), kTxBytes + 2 * zr_bytes);
                         tma_load_2d(smem_u32(kTok == kTokI8 ? S.bs[s % (kTok == kTokI8 ? kStages : 1)] : S.b[s]),
                                     &tm_q, smem_u32(&S.full[s]), kb * kBK, m0);
                         tma_load_2d(smem_u32(S.w[s]), &tm_w, smem_u32(&S.full[s]), kb * kBK, n0);
+                        if constexpr (kTok == kTokX) {
+                            const int zs = s % (kTok == kTokX ? kStages : 1);
+                            bulk_load(smem_u32(S.zr[zs][0]), xz + kb * kBK, zr_bytes, smem_u32(&S.full[s]));
+                            bulk_load(smem_u32(S.zr[zs][1]), xr + kb * kBK, zr_bytes, smem_u32(&S.full[s]));
+                        }
                     }
                     __syncwarp();
                 }
@@ -383,23 +392,25 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
             for (int kb = pk0; kb < pk1; ++kb, ++it) {
                 const int s = it % kStages;
                 const uint32_t ph = (it / kStages) & 1;
+                if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
                 float2 nz[4], rr[4];
                 if constexpr (kTok == kTokX) {
-                    // channels past K (zero-filled by the copy) get z = r = 0: code 0
-                    const int k0 = kb * kBK + cl * 8;
+                    // channels past K (zero-filled by the copy; their z, r not copied) get z = r = 0: code 0
                     float4 z0 = make_float4(0.f, 0.f, 0.f, 0.f), z1 = z0, q0 = z0, q1 = z0;
-                    if (k0 < K) {
-                        z0 = __ldg(reinterpret_cast<const float4 *>(xz + k0));
-                        z1 = __ldg(reinterpret_cast<const float4 *>(xz + k0) + 1);
-                        q0 = __ldg(reinterpret_cast<const float4 *>(xr + k0));
-                        q1 = __ldg(reinterpret_cast<const float4 *>(xr + k0) + 1);
+                    if (kb * kBK + cl * 8 < K) {
+                        const int zs = s % (kTok == kTokX ? kStages : 1);
+                        const float4 *zp = reinterpret_cast<const float4 *>(S.zr[zs][0] + cl * 8);
+                        const float4 *rp = reinterpret_cast<const float4 *>(S.zr[zs][1] + cl * 8);
+                        z0 = zp[0];
+                        z1 = zp[1];
+                        q0 = rp[0];
+                        q1 = rp[1];
                     }
                     nz[0] = make_float2(-z0.x, -z0.y); nz[1] = make_float2(-z0.z, -z0.w);
                     nz[2] = make_float2(-z1.x, -z1.y); nz[3] = make_float2(-z1.z, -z1.w);
                     rr[0] = make_float2(q0.x, q0.y); rr[1] = make_float2(q0.z, q0.w);
                     rr[2] = make_float2(q1.x, q1.y); rr[3] = make_float2(q1.z, q1.w);
                 }
-                if (!(ok = mbar_wait(smem_u32(&S.full[s]), ph, abort, &g_status))) break;
                 uint8_t *bt = S.b[s] + cp;
                 if constexpr (kTok == kTokI8) {
                     uint2 v[BN / 16];

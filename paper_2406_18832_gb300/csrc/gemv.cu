@@ -173,9 +173,14 @@ __global__ void __launch_bounds__(kGvThreads, 1)
 
     // Load unit (tile, ks) into `slot`, completing on full[slot]: the weight
     // boxes, then (load_codes) the codes box.
+    // kGvX: the slice's z and r follow the activation box (channels below K only)
+    const uint32_t zr_off = kGvWBytes + abytes;
+    auto zr_bytes = [&](int ks) -> uint32_t {
+        return kTokG == kGvX ? (uint32_t)min(kGvKS, K - ks * kGvKS) * 4 : 0u;
+    };
     auto load_weights = [&](int slot, int64_t tile, int ks) {
         const uint32_t bar = smem_u32(&full[slot]);
-        mbar_arrive_expect_tx(bar, kGvWBytes + abytes);
+        mbar_arrive_expect_tx(bar, kGvWBytes + abytes + 2 * zr_bytes(ks));
         const uint32_t st = smem_u32(ring + (size_t)slot * p.stage_bytes);
         tma_load_2d_hint(st, &tm_w, bar, ks * kGvKS, (int32_t)(tile * kGvRows), pol_w);
         tma_load_2d_hint(st + kGvWBox, &tm_w, bar, ks * kGvKS + 128, (int32_t)(tile * kGvRows), pol_w);
@@ -184,6 +189,10 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     auto load_codes = [&](int slot, int ks) {
         const uint32_t st = smem_u32(ring + (size_t)slot * p.stage_bytes);
         tma_load_2d_hint(st + kGvWBytes, &tm_a, smem_u32(&full[slot]), ks * kGvKS, 0, pol_a);
+        if constexpr (kTokG == kGvX) {
+            bulk_load(st + zr_off, p.xz + ks * kGvKS, zr_bytes(ks), smem_u32(&full[slot]));
+            bulk_load(st + zr_off + kGvKS * 4, p.xr + ks * kGvKS, zr_bytes(ks), smem_u32(&full[slot]));
+        }
     };
     auto load_unit = [&](int slot, int64_t tile, int ks) {
         load_weights(slot, tile, ks);
@@ -292,25 +301,26 @@ __global__ void __launch_bounds__(kGvThreads, 1)
             bool ok;
             if constexpr (kTokG == kGvX) {
                 // thread j quantizes the 16-byte chunk j (8 channels of one token) of the
-                // box; z, r are fetched before the wait; channels past K get code 0
+                // box with the slice's z, r copied beside it; channels past K get code 0
                 const int j = threadIdx.x;
-                const int k0 = ks * kGvKS + (j & 31) * 8;
-                float2 nz[4], rq[4];
-                float4 z0 = make_float4(0.f, 0.f, 0.f, 0.f), z1 = z0, q0 = z0, q1 = z0;
-                if (j < M * 32 && k0 < K) {
-                    z0 = __ldg(reinterpret_cast<const float4 *>(p.xz + k0));
-                    z1 = __ldg(reinterpret_cast<const float4 *>(p.xz + k0) + 1);
-                    q0 = __ldg(reinterpret_cast<const float4 *>(p.xr + k0));
-                    q1 = __ldg(reinterpret_cast<const float4 *>(p.xr + k0) + 1);
-                }
-                nz[0] = make_float2(-z0.x, -z0.y); nz[1] = make_float2(-z0.z, -z0.w);
-                nz[2] = make_float2(-z1.x, -z1.y); nz[3] = make_float2(-z1.z, -z1.w);
-                rq[0] = make_float2(q0.x, q0.y); rq[1] = make_float2(q0.z, q0.w);
-                rq[2] = make_float2(q1.x, q1.y); rq[3] = make_float2(q1.z, q1.w);
                 ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[slot]), phase, abort, p.status));
                 if (ok && j < M * 32) {
-                    uint4 *c = reinterpret_cast<uint4 *>(ring + (size_t)slot * p.stage_bytes + kGvWBytes +
-                                                         (j >> 5) * (2 * kGvKS) + (j & 31) * 16);
+                    uint8_t *stg = ring + (size_t)slot * p.stage_bytes;
+                    float4 z0 = make_float4(0.f, 0.f, 0.f, 0.f), z1 = z0, q0 = z0, q1 = z0;
+                    if (ks * kGvKS + (j & 31) * 8 < K) {
+                        const float4 *zp = reinterpret_cast<const float4 *>(stg + zr_off + (j & 31) * 32);
+                        const float4 *rp = reinterpret_cast<const float4 *>(stg + zr_off + kGvKS * 4 + (j & 31) * 32);
+                        z0 = zp[0];
+                        z1 = zp[1];
+                        q0 = rp[0];
+                        q1 = rp[1];
+                    }
+                    float2 nz[4], rq[4];
+                    nz[0] = make_float2(-z0.x, -z0.y); nz[1] = make_float2(-z0.z, -z0.w);
+                    nz[2] = make_float2(-z1.x, -z1.y); nz[3] = make_float2(-z1.z, -z1.w);
+                    rq[0] = make_float2(q0.x, q0.y); rq[1] = make_float2(q0.z, q0.w);
+                    rq[2] = make_float2(q1.x, q1.y); rq[3] = make_float2(q1.z, q1.w);
+                    uint4 *c = reinterpret_cast<uint4 *>(stg + kGvWBytes + (j >> 5) * (2 * kGvKS) + (j & 31) * 16);
                     *c = quantize_f16x8(*c, nz, rq, p.qmax_in);
                 }
                 __syncwarp();
@@ -471,7 +481,8 @@ cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvP
     if (attr_err != cudaSuccess) return attr_err;
     GvParams p = base;
     p.red_bytes = (TN * 8 * (kGvRows + 1) * 4 + 127) / 128 * 128;
-    p.stage_bytes = (kGvWBytes + p.M * kGvKS * (kTokG == kGvI8 ? 1 : 2) + 1023) & ~1023;
+    p.stage_bytes = (kGvWBytes + p.M * kGvKS * (kTokG == kGvI8 ? 1 : 2) + (kTokG == kGvX ? 2 * kGvKS * 4 : 0) + 1023) &
+                    ~1023;
     const int ring_off = (kGvHeader + p.red_bytes + 1023) & ~1023;
     const int room = kGvSmemBudget - 1024 - ring_off;
     p.stages = room / p.stage_bytes;

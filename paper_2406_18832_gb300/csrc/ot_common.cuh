@@ -275,6 +275,15 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void *tmap, uint
         : "memory");
 }
 
+// Plain (untiled) bulk copy of `bytes` from global to shared memory,
+// completing on `bar` as transaction bytes; both addresses 16-byte aligned,
+// bytes a multiple of 16.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
 // Programmatic dependent launch.  A kernel launched with programmatic stream
 // serialization may start while the kernel before it in the stream is still
 // running; grid_dep_wait() returns once that kernel has completed and its

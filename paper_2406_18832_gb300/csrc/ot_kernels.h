@@ -62,9 +62,9 @@ struct LinearArgs {
     int qmax_in = 0;          // kActF16: qmax of the codes
 };
 constexpr int kCodesF16 = 0, kCodesI8 = 1, kActF16 = 2;
-// ot_linear_fused quantizes inside the linear's token producer up to this
-// many tokens (decode kernel and linear_kernel); above it the prefill kernel
-// reads codes written by the quantize kernel.
+// Largest token count for which the linear's token producer can quantize X
+// itself (decode kernel and linear_kernel); above it only the prefill kernel,
+// reading codes written by the quantize kernel, runs.
 constexpr int64_t kFusedInKernelMaxTokens = 128;
 // Workspace bytes that enable stream-K scheduling of the prefill kernel on this device.
 size_t linear_workspace_bytes();

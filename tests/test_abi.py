@@ -70,7 +70,7 @@ def _linear_args(handle):
     handle.ot_quantize_act_rowsum.argtypes = [P, I64, I64, I64, P, P, I, P, I, P, P]
     handle.ot_fold_weights_asym.argtypes = [P, P, I, I, P, P, I64, I64, I, P, P, P, P, P, P, P, P]
     handle.ot_linear_quantize_next.argtypes = [P, I64, I64, P, P, P, I64, I, I, I, P, P, I, P, I64, P, S, P]
-    handle.ot_linear_fused.argtypes = [P, I64, I64, I64, P, P, I, P, P, P, I64, I, P, P, I64, I, P, S, P]
+    handle.ot_linear_fused.argtypes = [P, I64, I64, I64, P, P, I, P, P, P, I64, I, P, P, I64, I, I, P, S, P]
 
 
 # Fake, 256-byte-aligned addresses: every call below must be rejected on the
@@ -132,12 +132,15 @@ def test_validation_rejects_bad_arguments_before_launch(lib):
     assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, A, A + 2, 8, A, 16, None, 0, None) == INV
     assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, A, A, 9, A, 16, None, 0, None) == INV
     assert qn(A, 4, 64, A2, A, A, 16, 8, 8, 1, A, A, 8, A, 15, None, 0, None) == INV
-    # fused quantize + linear: ldx < K, null z, unaligned x, null code buffer
+    # fused quantize + linear: ldx < K, null z, unaligned x, null code buffer, unknown mode,
+    # the in-producer form above 128 tokens
     fz = handle.ot_linear_fused
-    assert fz(A, 4, 64, 56, A, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, None, 0, None) == INV
-    assert fz(A, 4, 64, 64, None, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, None, 0, None) == INV
-    assert fz(A + 8, 4, 64, 64, A, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, None, 0, None) == INV
-    assert fz(A, 4, 64, 64, A, A, 8, A2, A, A, 16, 8, None, A, 16, 0, None, 0, None) == INV
+    assert fz(A, 4, 64, 56, A, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, 0, None, 0, None) == INV
+    assert fz(A, 4, 64, 64, None, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, 0, None, 0, None) == INV
+    assert fz(A + 8, 4, 64, 64, A, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, 0, None, 0, None) == INV
+    assert fz(A, 4, 64, 64, A, A, 8, A2, A, A, 16, 8, None, A, 16, 0, 0, None, 0, None) == INV
+    assert fz(A, 4, 64, 64, A, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, 3, None, 0, None) == INV
+    assert fz(A, 129, 64, 64, A, A, 8, A2, A, A, 16, 8, A2, A, 16, 0, 1, None, 0, None) == UNS
 
 
 def test_validation_of_the_layernorm_calibration_and_per_token_entry_points(lib):

@@ -129,11 +129,17 @@ def _check_tokens(cfg, li, layer, ql, o, M, bits, full: bool):
     yf = torch.empty_like(y)
     binding.ot_linear_fused(x, ql.z, ql.r, bits_a, ql.qw, ql.sw, ql.b_fold, bits_w, torch.empty_like(q), yf,
                             relu=layer.relu_out)
+    yp = None
+    if M <= 128:
+        yp = torch.empty_like(y)
+        binding.ot_linear_fused(x, ql.z, ql.r, bits_a, ql.qw, ql.sw, ql.b_fold, bits_w, torch.empty_like(q), yp,
+                                relu=layer.relu_out, mode=binding.OT_FUSE_PRODUCER)
     torch.cuda.synchronize()
     assert binding.ot_get_device_status() == binding.OT_OK
     assert np.array_equal(q8.cpu().numpy(), oq), f"int8 codes M={M}"
     assert torch.equal(y8, y), f"int8-code linear M={M}"
     assert torch.equal(yf, y), f"fused linear M={M}"
+    assert yp is None or torch.equal(yp, y), f"linear quantizing in its producer M={M}"
 
 
 # (config, layer, bits, token counts, token counts checked in full)

@@ -1,8 +1,9 @@
 """ot_linear_fused: the activation quantization (Eq. 6-7) and the linear in one
-call.  Up to 128 tokens the linear's token producer quantizes X in shared
-memory (decode kernel for M <= 16, the single-CTA tcgen05 kernel's token
-warps for 16 < M <= 128); above, the quantize kernel writes the codes and
-the prefill linear runs as its programmatic dependent.  Against the oracle
+call, in both forms: the quantize kernel followed by the linear as its
+programmatic dependent (OT_FUSE_PDL, the default), and up to 128 tokens the
+linear's token producer quantizing X in shared memory (OT_FUSE_PRODUCER:
+decode kernel for M <= 16, the single-CTA tcgen05 kernel's token warps for
+16 < M <= 128).  Against the oracle
 bit for bit on every kernel of the path, with and without the stream-K
 workspace, with a strided X, channel counts that end inside a 64-wide
 k-block, NaN and infinite inputs, under CUDA-graph capture, and in
@@ -73,16 +74,18 @@ def test_linear_fused_bit_exact(M, N, K, bits):
     xd = x.to(DEV)[:, :K]
     for relu in (False, True):
         q_o, _, y_o = oracle.linear(np.ascontiguousarray(xs.numpy()), qw, sw, bf, z, r, bits, relu)
-        for workspace in (False, ws, ws):
-            q = torch.full((M, K), 5.0, dtype=torch.float16, device=DEV)
-            y = torch.full((M, N), 7.0, dtype=torch.float16, device=DEV)
-            B.ot_linear_fused(xd, _dev(z), _dev(r), bits, _dev(qw), _dev(sw), _dev(bf), bits, q, y, relu=relu,
-                              workspace=workspace)
-            torch.cuda.synchronize()
-            assert B.ot_get_device_status() == B.OT_OK
-            if M > 128:  # the codes go through the caller's buffer only at prefill sizes
-                assert np.array_equal(q.cpu().numpy().astype(np.int64), q_o.astype(np.int64))
-            assert np.array_equal(y.cpu().numpy().view(np.uint16), y_o.view(np.uint16))
+        modes = (B.OT_FUSE_AUTO, B.OT_FUSE_PDL) + ((B.OT_FUSE_PRODUCER,) if M <= 128 else ())
+        for mode in modes:
+            for workspace in (False, ws, ws):
+                q = torch.full((M, K), 5.0, dtype=torch.float16, device=DEV)
+                y = torch.full((M, N), 7.0, dtype=torch.float16, device=DEV)
+                B.ot_linear_fused(xd, _dev(z), _dev(r), bits, _dev(qw), _dev(sw), _dev(bf), bits, q, y, relu=relu,
+                                  workspace=workspace, mode=mode)
+                torch.cuda.synchronize()
+                assert B.ot_get_device_status() == B.OT_OK
+                if mode != B.OT_FUSE_PRODUCER:  # the in-producer form writes no codes
+                    assert np.array_equal(q.cpu().numpy().astype(np.int64), q_o.astype(np.int64))
+                assert np.array_equal(y.cpu().numpy().view(np.uint16), y_o.view(np.uint16)), f"mode {mode}"
 
 
 @pytest.mark.parametrize("M", [1, 16, 64, 512])
@@ -99,12 +102,15 @@ def test_linear_fused_back_to_back_one_code_buffer(M):
     args = [_dev(a) for a in (z, r, qw, sw, bf)]
     xd = [x.to(DEV) for x in xs]
     torch.cuda.synchronize()
-    for x, y in zip(xd, ys):
-        B.ot_linear_fused(x, args[0], args[1], 8, args[2], args[3], args[4], 8, q, y)
-    torch.cuda.synchronize()
-    for x, y in zip(xs, ys):
-        _, _, y_o = oracle.linear(x.numpy(), qw, sw, bf, z, r, 8)
-        assert np.array_equal(y.cpu().numpy().view(np.uint16), y_o.view(np.uint16))
+    for mode in (B.OT_FUSE_PDL,) + ((B.OT_FUSE_PRODUCER,) if M <= 128 else ()):
+        for x, y in zip(xd, ys):
+            y.fill_(0)
+        for x, y in zip(xd, ys):
+            B.ot_linear_fused(x, args[0], args[1], 8, args[2], args[3], args[4], 8, q, y, mode=mode)
+        torch.cuda.synchronize()
+        for x, y in zip(xs, ys):
+            _, _, y_o = oracle.linear(x.numpy(), qw, sw, bf, z, r, 8)
+            assert np.array_equal(y.cpu().numpy().view(np.uint16), y_o.view(np.uint16))
 
 
 @pytest.mark.parametrize("M", [4, 96, 400])
