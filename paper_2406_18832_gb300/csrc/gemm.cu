@@ -354,22 +354,19 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
                     raw[c] = *reinterpret_cast<const uint4 *>(S.w[s] + row * 64 + ((c ^ sw64) << 4));
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.empty[s]));
+                // the row's 64 fp16 values, two per 32-bit TMEM column, k ascending; widened
+                // before waiting for the TMEM buffer, so only the store follows the wait
+                uint32_t a[32];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    i8x4_to_f16x4(raw[c].x, a[8 * c + 0], a[8 * c + 1]);
+                    i8x4_to_f16x4(raw[c].y, a[8 * c + 2], a[8 * c + 3]);
+                    i8x4_to_f16x4(raw[c].z, a[8 * c + 4], a[8 * c + 5]);
+                    i8x4_to_f16x4(raw[c].w, a[8 * c + 6], a[8 * c + 7]);
+                }
                 if (!(ok = mbar_wait(smem_u32(&S.aempty[s]), ph ^ 1, abort, &g_status))) break;
                 tc_fence_after();
-                // the row's 64 fp16 values, two per 32-bit TMEM column, k ascending, in two halves
-#pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    uint32_t a[16];
-#pragma unroll
-                    for (int c = 0; c < 2; ++c) {
-                        const uint4 r4 = raw[2 * half + c];
-                        i8x4_to_f16x4(r4.x, a[8 * c + 0], a[8 * c + 1]);
-                        i8x4_to_f16x4(r4.y, a[8 * c + 2], a[8 * c + 3]);
-                        i8x4_to_f16x4(r4.z, a[8 * c + 4], a[8 * c + 5]);
-                        i8x4_to_f16x4(r4.w, a[8 * c + 6], a[8 * c + 7]);
-                    }
-                    tmem_st16(tmem + lane_base + s * 32 + half * 16, a);
-                }
+                tmem_st32(tmem + lane_base + s * 32, a);
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
@@ -858,6 +855,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                 __syncwarp();
                 // the group's last weights are in registers: the stage may be refilled
                 if (lane == 0 && last) mbar_arrive(smem_u32(&S.wempty[wst]));
+                // the row's 64 fp16 values, two per 32-bit TMEM column, k ascending; widened
+                // before waiting for the A stage, so only the TMEM store follows the wait
+                uint32_t h[32];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    i8x4_to_f16x4(raw[c].x, h[8 * c + 0], h[8 * c + 1]);
+                    i8x4_to_f16x4(raw[c].y, h[8 * c + 2], h[8 * c + 3]);
+                    i8x4_to_f16x4(raw[c].z, h[8 * c + 4], h[8 * c + 5]);
+                    i8x4_to_f16x4(raw[c].w, h[8 * c + 6], h[8 * c + 7]);
+                }
                 // A stage sa was last read by the MMA of k-block it - kAStages
                 if (it >= (uint32_t)kAStages) {
                     const uint32_t prev = it - kAStages;
@@ -865,20 +872,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                         break;
                     tc_fence_after();
                 }
-                // the row's 64 fp16 values, two per 32-bit TMEM column, k ascending, in two halves
-#pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    uint32_t h[16];
-#pragma unroll
-                    for (int c = 0; c < 2; ++c) {
-                        const uint4 r4 = raw[2 * half + c];
-                        i8x4_to_f16x4(r4.x, h[8 * c + 0], h[8 * c + 1]);
-                        i8x4_to_f16x4(r4.y, h[8 * c + 2], h[8 * c + 3]);
-                        i8x4_to_f16x4(r4.z, h[8 * c + 4], h[8 * c + 5]);
-                        i8x4_to_f16x4(r4.w, h[8 * c + 6], h[8 * c + 7]);
-                    }
-                    tmem_st16(a_tm + sa * 32 + half * 16, h);
-                }
+                tmem_st32(a_tm + sa * 32, h);
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
