@@ -44,7 +44,9 @@ typedef enum {
     OT_ERR_INVALID_ARG = 1,  /* null pointer, bad size, alignment or bits */
     OT_ERR_UNSUPPORTED = 2,  /* valid request this build does not run (e.g. K too large) */
     OT_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed */
-    OT_ERR_TIMEOUT = 4       /* a bounded device-side wait gave up */
+    OT_ERR_TIMEOUT = 4,      /* a bounded device-side wait gave up */
+    OT_ERR_BOUNDS = 5        /* debug builds only (OT_DEBUG): a kernel's index
+                                check failed and the access was skipped */
 } ot_status;
 
 /* Storage format of activation codes (written by the quantize entry points,
@@ -62,6 +64,12 @@ const char *ot_status_string(ot_status st);
 
 /* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
 int ot_version(void);
+
+/* 1 when the library was compiled with OT_DEBUG (kernels check their global
+ * indices against the sizes they were given, skip an access that fails and
+ * report it through ot_get_device_status as OT_ERR_BOUNDS), else 0.  The paper
+ * has no counterpart: it stands in for a memory checker. */
+int ot_debug_build(void);
 
 /*
  * ot_calibrate -- per-channel running min / max of calibration activations
@@ -416,8 +424,9 @@ ot_status ot_linear_s32(const void *q, int q_format, int64_t M, int64_t K,
 /*
  * ot_get_device_status -- synchronize `stream`, then return and clear the
  * device status word of the current device: OT_ERR_TIMEOUT if a bounded
- * device wait gave up since the last call, else OT_OK (or OT_ERR_CUDA if the
- * synchronization itself failed).
+ * device wait gave up since the last call; in a debug build OT_ERR_BOUNDS if
+ * an index check failed since the last call; else OT_OK (or OT_ERR_CUDA if
+ * the synchronization itself failed).
  */
 ot_status ot_get_device_status(void *stream);
 

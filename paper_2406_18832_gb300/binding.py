@@ -16,17 +16,19 @@ import torch
 
 from . import build as _build
 
-OT_OK, OT_ERR_INVALID_ARG, OT_ERR_UNSUPPORTED, OT_ERR_CUDA, OT_ERR_TIMEOUT = range(5)
+OT_OK, OT_ERR_INVALID_ARG, OT_ERR_UNSUPPORTED, OT_ERR_CUDA, OT_ERR_TIMEOUT, OT_ERR_BOUNDS = range(6)
 OT_CODE_I8, OT_CODE_F16 = 0, 1
 OT_FUSE_AUTO, OT_FUSE_PRODUCER, OT_FUSE_PDL = 0, 1, 2
 
 _lock = threading.Lock()
-_handle = None
+_handle = None          # the library the functions below call
+_handles = {}           # loaded libraries by variant ("release", "debug")
 
 _P, _I64, _I, _F = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float
 _SIGNATURES = {
     "ot_status_string": ([_I], ctypes.c_char_p),
     "ot_version": ([], _I),
+    "ot_debug_build": ([], _I),
     "ot_calibrate": ([_P, _I64, _I64, _I64, _P, _P, _I, _P], _I),
     "ot_derive_params": ([_P, _P, _I64, _I, _I, _P, _P, _P, _P], _I),
     "ot_fold_weights": ([_P, _P, _I, _I, _P, _P, _I64, _I64, _I, _P, _P, _P, _P, _P, _P, _P], _I),
@@ -65,21 +67,40 @@ def library_path() -> str:
     return _build.LIB_PATH
 
 
+def _open(variant: str) -> ctypes.CDLL:
+    lib = _handles.get(variant)
+    if lib is None:
+        path = _build.LIB_PATH_DEBUG if variant == "debug" else _build.LIB_PATH
+        if not os.path.exists(path):
+            raise RuntimeError(f"CUDA library not built: {path} is missing "
+                               "(run __graft_entry__.build() or python -m paper_2406_18832_gb300.build)")
+        lib = ctypes.CDLL(path)
+        for name, (args, res) in _SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        _handles[variant] = lib
+    return lib
+
+
 def load() -> ctypes.CDLL:
-    """Load lib/libot_gb300.so (built by paper_2406_18832_gb300.build)."""
+    """The library the functions of this module call: lib/libot_gb300.so
+    (built by paper_2406_18832_gb300.build) unless select() chose another."""
     global _handle
     with _lock:
         if _handle is None:
-            path = _build.LIB_PATH
-            if not os.path.exists(path):
-                raise RuntimeError(f"CUDA library not built: {path} is missing "
-                                   "(run __graft_entry__.build() or python -m paper_2406_18832_gb300.build)")
-            lib = ctypes.CDLL(path)
-            for name, (args, res) in _SIGNATURES.items():
-                fn = getattr(lib, name)
-                fn.argtypes = args
-                fn.restype = res
-            _handle = lib
+            _handle = _open("release")
+    return _handle
+
+
+def select(variant: str = "release") -> ctypes.CDLL:
+    """Route this module's calls to the release library or to the debug build
+    (lib/libot_gb300_debug.so: kernels check their indices, OT_DEBUG)."""
+    global _handle
+    if variant not in ("release", "debug"):
+        raise ValueError("variant must be 'release' or 'debug'")
+    with _lock:
+        _handle = _open(variant)
     return _handle
 
 

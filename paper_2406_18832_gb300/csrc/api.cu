@@ -46,11 +46,20 @@ const char *ot_status_string(ot_status st) {
         case OT_ERR_UNSUPPORTED: return "OT_ERR_UNSUPPORTED: request outside what this build runs";
         case OT_ERR_CUDA: return "OT_ERR_CUDA: a CUDA call or kernel launch failed";
         case OT_ERR_TIMEOUT: return "OT_ERR_TIMEOUT: a bounded device wait gave up";
+        case OT_ERR_BOUNDS: return "OT_ERR_BOUNDS: a kernel index check failed (debug build)";
     }
     return "unknown ot_status";
 }
 
 int ot_version(void) { return kVersion; }
+
+int ot_debug_build(void) {
+#ifdef OT_DEBUG
+    return 1;
+#else
+    return 0;
+#endif
+}
 
 ot_status ot_calibrate(const void *x_f16, int64_t T, int64_t K, int64_t ldx, float *ch_min, float *ch_max,
                        int reset, void *stream) {
@@ -324,6 +333,15 @@ ot_status ot_selftest_wait_timeout(int64_t limit_ns, void *stream) {
 ot_status ot_get_device_status(void *stream) {
     int v = 0;
     if (ot::read_clear_status(&v, as_stream(stream)) != cudaSuccess) return OT_ERR_CUDA;
+#ifdef OT_DEBUG
+    // the first failed index check of each file's kernels (source line, 0 = none)
+    unsigned lines[4] = {0, 0, 0, 0};
+    if (ot::dbg_read_clear_gemm(&lines[0]) != cudaSuccess || ot::dbg_read_clear_gemv(&lines[1]) != cudaSuccess ||
+        ot::dbg_read_clear_quant(&lines[2]) != cudaSuccess || ot::dbg_read_clear_fold(&lines[3]) != cudaSuccess)
+        return OT_ERR_CUDA;
+    for (unsigned l : lines)
+        if (l != 0) return OT_ERR_BOUNDS;
+#endif
     return v == OT_ERR_TIMEOUT ? OT_ERR_TIMEOUT : OT_OK;
 }
 

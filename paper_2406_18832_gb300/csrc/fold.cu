@@ -8,6 +8,8 @@
 
 namespace ot {
 
+OT_DEBUG_UNIT(fold)
+
 namespace {
 
 constexpr int kFoldThreads = 256;
@@ -66,7 +68,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_codes_kernel(const __half *
             uint2 o;
             o.x = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
             o.y = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
-            *reinterpret_cast<uint2 *>(qw + n * K + k) = o;
+            if (OT_DCHECK(k + 8 <= K)) *reinterpret_cast<uint2 *>(qw + n * K + k) = o;
         }
         __syncthreads();
     }
@@ -155,7 +157,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_codes_asym_kernel(const __h
             uint2 o;
             o.x = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
             o.y = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
-            *reinterpret_cast<uint2 *>(qw + n * K + k) = o;
+            if (OT_DCHECK(k + 8 <= K)) *reinterpret_cast<uint2 *>(qw + n * K + k) = o;
         }
         __syncthreads();
     }

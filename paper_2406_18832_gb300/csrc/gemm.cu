@@ -45,6 +45,7 @@ namespace ot {
 
 // Device status word of this library (OT_OK or OT_ERR_TIMEOUT), one per device.
 __device__ int g_status;
+OT_DEBUG_UNIT(gemm)
 
 namespace {
 
@@ -495,8 +496,9 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
             if (pk1 < nkb) {
                 // partial piece: publish the int32 sums for the CTA that ends this tile
                 int32_t *slot = ws + (size_t)blockIdx.x * pair_slot_ints();
+                if (OT_DCHECK(blockIdx.x < 2u * (unsigned)ws_pairs && col0 + CPW <= 256))
 #pragma unroll
-                for (int j = 0; j < CPW; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
+                    for (int j = 0; j < CPW; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.pub));
@@ -536,7 +538,7 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
 #pragma unroll
                     for (int j = 0; j < CPW; ++j) {
                         const int m = m0 + col0 + j;
-                        if (m < M) o[(int64_t)m * N + n] = tot[j];
+                        if (m < M && OT_DCHECK((int64_t)m * N + n < (int64_t)M * N)) o[(int64_t)m * N + n] = tot[j];
                     }
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
@@ -561,9 +563,11 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
                         if constexpr (kQOut) {
                             // the next layer's code round((v - z') * r'), as an fp16 integer
                             const int c = __float2int_rn(__fmul_rn(__fsub_rn(v, zqn), rqn));
-                            if (m < M) o[(int64_t)m * ldy + n] = __int2half_rn(max(-qmax_out, min(qmax_out, c)));
+                            if (m < M && OT_DCHECK((int64_t)m * ldy + n < (int64_t)(M - 1) * ldy + N))
+                                o[(int64_t)m * ldy + n] = __int2half_rn(max(-qmax_out, min(qmax_out, c)));
                         } else {
-                            if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                            if (m < M && OT_DCHECK((int64_t)m * ldy + n < (int64_t)(M - 1) * ldy + N))
+                                o[(int64_t)m * ldy + n] = __float2half_rn(v);
                         }
                     }
                 }
@@ -942,8 +946,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             if (pk1 < nkb) {
                 // partial piece: publish the int32 sums for the pair that ends this tile
                 int32_t *slot = slots + ((size_t)cluster * 2 + rank) * pair_slot_ints();
+                if (OT_DCHECK(cluster < nclusters && col0 + kPairHalf <= 256))
 #pragma unroll
-                for (int j = 0; j < kPairHalf; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
+                    for (int j = 0; j < kPairHalf; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.pub));
@@ -983,7 +988,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 #pragma unroll
                     for (int j = 0; j < kPairHalf; ++j) {
                         const int m = m0 + col0 + j;
-                        if (m < M) o[(int64_t)m * N + n] = tot[j];
+                        if (m < M && OT_DCHECK((int64_t)m * N + n < (int64_t)M * N)) o[(int64_t)m * N + n] = tot[j];
                     }
                 } else {
                     const float scale = __ldg(sw + n), bias = __ldg(bfold + n);
@@ -1008,9 +1013,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                         if constexpr (kQOut) {
                             // the next layer's code round((v - z') * r'), as an fp16 integer
                             const int c = __float2int_rn(__fmul_rn(__fsub_rn(v, zqn), rqn));
-                            if (m < M) o[(int64_t)m * ldy + n] = __int2half_rn(max(-qmax_out, min(qmax_out, c)));
+                            if (m < M && OT_DCHECK((int64_t)m * ldy + n < (int64_t)(M - 1) * ldy + N))
+                                o[(int64_t)m * ldy + n] = __int2half_rn(max(-qmax_out, min(qmax_out, c)));
                         } else {
-                            if (m < M) o[(int64_t)m * ldy + n] = __float2half_rn(v);
+                            if (m < M && OT_DCHECK((int64_t)m * ldy + n < (int64_t)(M - 1) * ldy + N))
+                                o[(int64_t)m * ldy + n] = __float2half_rn(v);
                         }
                     }
                 }

@@ -54,6 +54,8 @@
 
 namespace ot {
 
+OT_DEBUG_UNIT(gemv)
+
 namespace {
 
 constexpr int kGvRows = 128;                      // weight rows per tile (16 MMA n8 groups)
@@ -124,7 +126,7 @@ __device__ __forceinline__ uint64_t ld_acquire_flag(const unsigned long long *f)
 template <bool kS32>
 __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32_t s) {
     if constexpr (kS32) {
-        reinterpret_cast<int32_t *>(p.out)[(int64_t)m * p.N + n] = s;
+        if (OT_DCHECK(m < p.M && n < p.N)) reinterpret_cast<int32_t *>(p.out)[(int64_t)m * p.N + n] = s;
     } else {
         const float scale = __ldg(p.sw + n);
         const float sc = p.s_tok ? __fmul_rn(__ldg(p.s_tok + m), scale) : scale;  // per-token path (Eq. 3)
@@ -141,7 +143,8 @@ __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32
         } else {
             o = __float2half_rn(v);
         }
-        reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = o;
+        if (OT_DCHECK(m < p.M && n < p.N && p.N <= p.ldy))
+            reinterpret_cast<__half *>(p.out)[(int64_t)m * p.ldy + n] = o;
     }
 }
 
@@ -415,9 +418,10 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         } else if (seg_begin != tile * nks) {
             // a later part of a tile that an earlier CTA finishes: publish it
             int32_t *part = p.part + (size_t)blockIdx.x * kGvSlotInts;
+            const bool in_ws = OT_DCHECK((int)blockIdx.x < p.grid && M * kGvRows <= kGvSlotInts);
             for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
                 const int m = idx / kGvRows, c = idx % kGvRows;
-                __stcg(part + idx, red[m][c]);
+                if (in_ws) __stcg(part + idx, red[m][c]);
                 red[m][c] = 0;
             }
             __threadfence();

@@ -27,6 +27,34 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 
+// ---------------------------------------------------------------------------
+// Debug builds (-DOT_DEBUG): index checks in place of a memory checker.
+// OT_DCHECK(cond) is true in release builds; in debug builds a false
+// condition records the source line in the translation unit's debug word
+// (first failure wins) and returns false, so the guarded access is skipped.
+// Each .cu file that uses it declares OT_DEBUG_UNIT(name) once, which also
+// defines the host reader ot::dbg_read_clear_<name> (ot_get_device_status
+// polls them and returns OT_ERR_BOUNDS).
+// ---------------------------------------------------------------------------
+#ifdef OT_DEBUG
+__device__ __forceinline__ bool ot_dcheck(bool ok, unsigned line, unsigned *word) {
+    if (!ok) atomicCAS(word, 0u, line);
+    return ok;
+}
+#define OT_DEBUG_UNIT(name)                                                          \
+    static __device__ unsigned ot_dbg_line;                                         \
+    cudaError_t dbg_read_clear_##name(unsigned *line) {                             \
+        cudaError_t e = cudaMemcpyFromSymbol(line, ot_dbg_line, sizeof(unsigned)); \
+        if (e != cudaSuccess) return e;                                             \
+        const unsigned zero = 0;                                                    \
+        return cudaMemcpyToSymbol(ot_dbg_line, &zero, sizeof(unsigned));           \
+    }
+#define OT_DCHECK(cond) ::ot::ot_dcheck((cond), (unsigned)__LINE__, &ot_dbg_line)
+#else
+#define OT_DEBUG_UNIT(name)
+#define OT_DCHECK(cond) true
+#endif
+
 // Two fp32 values per instruction (sm_100 and later): IEEE round-to-nearest
 // add, product and fused multiply-add on each lane of the pair, with
 // subnormals kept; each result equals the scalar __fadd_rn / __fmul_rn /

@@ -85,6 +85,13 @@ bool tensor_map_2d(CUtensorMap *tm, CUtensorMapDataType dt, const void *base, ui
                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz);
 
 int num_sms();
+#ifdef OT_DEBUG
+// first failed index check (source line) of each file's kernels since the last read
+cudaError_t dbg_read_clear_gemm(unsigned *line);
+cudaError_t dbg_read_clear_gemv(unsigned *line);
+cudaError_t dbg_read_clear_quant(unsigned *line);
+cudaError_t dbg_read_clear_fold(unsigned *line);
+#endif
 int exact_chunk_kblocks(int bits_a, int bits_w, bool asym_w);
 cudaError_t read_clear_status(int *value, cudaStream_t st);
 cudaError_t launch_wait_timeout(int64_t limit_ns, cudaStream_t st);

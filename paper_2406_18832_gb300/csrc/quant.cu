@@ -9,6 +9,8 @@
 
 namespace ot {
 
+OT_DEBUG_UNIT(quant)
+
 namespace {
 
 constexpr int kQRowsPerThread = 8;              // rows a thread walks with the same z, r
@@ -95,12 +97,14 @@ __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict_
             o.y = pack_f16_codes(c[2], c[3]);
             o.z = pack_f16_codes(c[4], c[5]);
             o.w = pack_f16_codes(c[6], c[7]);
-            *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + m * K + c0) = o;
+            if (OT_DCHECK(m < M && c0 + 8 <= K))
+                *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + m * K + c0) = o;
         } else {
             uint2 o;
             o.x = pack_i8_codes(c[0], c[1], c[2], c[3]);
             o.y = pack_i8_codes(c[4], c[5], c[6], c[7]);
-            *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + m * K + c0) = o;
+            if (OT_DCHECK(m < M && c0 + 8 <= K))
+                *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + m * K + c0) = o;
         }
     }
 }
@@ -153,12 +157,14 @@ __global__ void __launch_bounds__(256) quantize_tokens_kernel(const __half *__re
             o.y = pack_f16_codes(c[2], c[3]);
             o.z = pack_f16_codes(c[4], c[5]);
             o.w = pack_f16_codes(c[6], c[7]);
-            *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + m * K + v * 8) = o;
+            if (OT_DCHECK(v * 8 + 8 <= K))
+                *reinterpret_cast<uint4 *>(reinterpret_cast<__half *>(q) + m * K + v * 8) = o;
         } else {
             uint2 o;
             o.x = pack_i8_codes(c[0], c[1], c[2], c[3]);
             o.y = pack_i8_codes(c[4], c[5], c[6], c[7]);
-            *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + m * K + v * 8) = o;
+            if (OT_DCHECK(v * 8 + 8 <= K))
+                *reinterpret_cast<uint2 *>(reinterpret_cast<int8_t *>(q) + m * K + v * 8) = o;
         }
     }
 }
