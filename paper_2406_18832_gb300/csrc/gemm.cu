@@ -240,8 +240,19 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
         mbar_init(smem_u32(&S.drain), 1);
         mbar_init(smem_u32(&S.pub), kNumEpiWarps);
         S.abort = 0;
-        S.epoch = ws ? __ldcg(pair_ctl(ws, ws_pairs)) + 1 : 0;
         fence_barrier_init();
+        // Launched as a programmatic dependent, the kernel before this one may
+        // still be running: prefetch the first weights into L2 (coherent with
+        // any write it makes), then wait for it before anything reads the
+        // codes or the workspace.
+        if (sch.count > 0) {
+            int u, pk0, pk1;
+            sch.piece(0, u, pk0, pk1);
+            for (int kb = pk0; kb < pk1 && kb < pk0 + kStages; ++kb)
+                tma_prefetch_l2_2d(&tm_w, kb * kBK, (u / m_tiles) * kBM);
+        }
+        grid_dep_wait();
+        S.epoch = ws ? __ldcg(pair_ctl(ws, ws_pairs)) + 1 : 0;
     }
     if (warp == kWarpTma && lane == 0) {
         tma_prefetch_desc(&tm_q);
@@ -255,6 +266,8 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
+    // the next linear on the stream may launch now (it waits for this one before reading anything this writes)
+    grid_dep_launch();
 
     // the TMA and MMA roles run their loops with the whole warp and issue from one elected lane
     // registers: 512 threads x 128 at launch (kTokF16); with the token warps
@@ -262,16 +275,6 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
     if (warp < 4) {
         if constexpr (kTok != kTokF16) regs_dec<48>();
         if (warp == kWarpTma) {
-            // weights of the first tile into L2 while a programmatic predecessor
-            // may still be writing the codes; then wait for it
-            if (sch.count > 0 && elect_one()) {
-                int u, pk0, pk1;
-                sch.piece(0, u, pk0, pk1);
-                for (int kb = pk0; kb < pk1 && kb < pk0 + kStages; ++kb)
-                    tma_prefetch_l2_2d(&tm_w, kb * kBK, (u / m_tiles) * kBM);
-            }
-            __syncwarp();
-            grid_dep_wait();
             uint32_t it = 0;
             bool ok = true;
             for (int p = 0; p < sch.count && ok; ++p) {
@@ -714,8 +717,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         mbar_init(smem_u32(&S.pub), kNumEpiWarps);
         mbar_init(smem_u32(&S.drain), 1);
         S.abort = 0;
-        S.epoch = ws ? __ldcg(pair_ctl(ws, nclusters)) + 1 : 0;
         fence_barrier_init();
+        // Launched as a programmatic dependent, the kernel before this one may
+        // still be running: prefetch the first weights into L2 (coherent with
+        // any write it makes), then wait for it before anything reads the
+        // codes or the workspace.
+        if (sch.count > 0) {
+            int u, pk0, pk1, mt, np;
+            sch.piece(0, u, pk0, pk1);
+            pair_tile(u, m_tiles, n_pairs, group_m, mt, np);
+            tma_prefetch_l2_3d(&tm_w, 0, (np * 2 + (int)rank) * kBM, pk0 >> 1);
+        }
+        grid_dep_wait();
+        S.epoch = ws ? __ldcg(pair_ctl(ws, nclusters)) + 1 : 0;
     }
     if (warp == kWarpTma && lane == 0) {
         tma_prefetch_desc(&tm_q);
@@ -730,22 +744,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     cluster_sync();  // barriers of both CTAs exist before either signals the other
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
+    // the next linear on the stream may launch now (it waits for this one before reading anything this writes)
+    grid_dep_launch();
 
     // registers at launch: 640 threads x 96; after the split 48 / 72 / 144 / 144 / 72 per warpgroup
     if (warp < 4) {
         regs_dec<48>();
         if (warp == kWarpTma) {
-            // the first weights into L2 while a programmatic predecessor may
-            // still be writing the codes; then wait for it
-            if (sch.count > 0 && elect_one()) {
-                int u, pk0, pk1;
-                sch.piece(0, u, pk0, pk1);
-                int mt, np;
-                pair_tile(u, m_tiles, n_pairs, group_m, mt, np);
-                tma_prefetch_l2_3d(&tm_w, 0, (np * 2 + (int)rank) * kBM, pk0 >> 1);
-            }
-            __syncwarp();
-            grid_dep_wait();
             uint32_t gi = 0;
             bool ok = true;
             for (int p = 0; p < sch.count && ok; ++p) {
@@ -1342,8 +1347,15 @@ cudaError_t noalloc_scratch(void **ptr, cudaStream_t st) {
     return cudaSuccess;
 }
 
-cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st) {
-    if (a.M == 0 || a.N == 0) return cudaSuccess;
+cudaError_t launch_linear(const LinearArgs &args, cudaStream_t st) {
+    if (args.M == 0 || args.N == 0) return cudaSuccess;
+    // Every linear launches as a programmatic dependent of the kernel before it
+    // on the stream, and lets the next one launch once its own set-up is done:
+    // consecutive linears overlap one's tail with the next one's launch, set-up
+    // and first weight fetches (each kernel reads codes, outputs and workspace
+    // only after the one before it has ended).
+    LinearArgs a = args;
+    a.pdl = true;
     const int nkb = (int)((a.K + kBK - 1) / kBK);
     int kcb = exact_chunk_kblocks(a.bits_a, a.bits_w, a.zc != nullptr);
     if (kcb > nkb) kcb = nkb;

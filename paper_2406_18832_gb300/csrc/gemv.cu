@@ -85,7 +85,8 @@ struct GvParams {
     int32_t *part;                 // [grid][kGvSlotInts] partial sums of split tiles (stream-K), or null
     unsigned long long *flags;     // [grid] launch epoch once a CTA's slot is complete
     unsigned long long *ctl;       // {epoch of the last launch, CTAs done with this one}
-    int pdl;                       // launched as a programmatic dependent of the codes' producer
+    int pdl;                       // launched as a programmatic dependent of the kernel before it
+    int weights_early;             // that kernel is this call's quantize kernel: weights may load before it ends
     const float *xz, *xr;          // kGvX: z, r [K]
     int qmax_in;                   // kGvX: qmax of the codes
     int *status;        // device status word
@@ -217,13 +218,17 @@ __global__ void __launch_bounds__(kGvThreads, 1)
             loads[s] = 0;
         }
         *abort = 0;
-        *epoch_s = p.whole ? 0 : __ldcg(p.ctl) + 1;
         fence_barrier_init();
-        // launched as a programmatic dependent of the kernel writing the
-        // codes: the first units' weights go out before waiting for it, their
-        // codes after it.  Otherwise the loads go out unit by unit, so that the
+        // Launched as a programmatic dependent, the kernel before this one on
+        // the stream may still be running until grid_dep_wait() returns; until
+        // then only the first units' weights are touched: loaded into the ring
+        // when that kernel is this call's own quantize kernel (weights_early:
+        // it started after every earlier writer of the weights), else
+        // prefetched into L2, which stays coherent with any write that kernel
+        // makes.  The codes and the workspace are read only after the wait.
+        // Without such a launch the loads go out unit by unit, so that the
         // first unit completes first.
-        const int pre = p.pdl ? (S < kGvPdlUnits ? S : kGvPdlUnits) : 0;
+        const int pre = p.weights_early ? (S < kGvPdlUnits ? S : kGvPdlUnits) : 0;
         int64_t tile = tile0;
         int ks = ks0;
         for (int s = 0; s < pre && u_begin + s < u_end; ++s) {
@@ -233,7 +238,20 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 ++tile;
             }
         }
+        if (p.pdl && !p.weights_early) {
+            int64_t t2 = tile0;
+            int k2 = ks0;
+            for (int s = 0; s < S && u_begin + s < u_end; ++s) {
+                tma_prefetch_l2_2d(&tm_w, k2 * kGvKS, (int32_t)(t2 * kGvRows));
+                tma_prefetch_l2_2d(&tm_w, k2 * kGvKS + 128, (int32_t)(t2 * kGvRows));
+                if (++k2 == nks) {
+                    k2 = 0;
+                    ++t2;
+                }
+            }
+        }
         grid_dep_wait();
+        *epoch_s = p.whole ? 0 : __ldcg(p.ctl) + 1;
         for (int s = 0, k2 = ks0; s < pre && u_begin + s < u_end; ++s) {
             load_codes(s, k2);
             if (++k2 == nks) k2 = 0;
@@ -247,6 +265,8 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         }
     }
     __syncthreads();
+    // the next linear on the stream may launch now (it waits for this one before reading anything this writes)
+    grid_dep_launch();
 
     const int t = lane & 3, r = lane >> 2;
     const int win = warp % kGvWindows, rp = warp / kGvWindows;  // window; rows 32 rp .. 32 rp + 31
@@ -526,6 +546,7 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
     p.rq = a.rq;
     p.qmax_out = a.qmax_out;
     p.pdl = a.pdl ? 1 : 0;
+    p.weights_early = a.pdl && a.weights_early ? 1 : 0;
     p.xz = a.xz;
     p.xr = a.xr;
     p.qmax_in = a.qmax_in;

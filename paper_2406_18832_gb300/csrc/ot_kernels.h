@@ -53,8 +53,11 @@ struct LinearArgs {
     const int32_t *rowsum;    // with zc: sum_k q[m,k] [M]
     const float *zq, *rq;     // chained epilogue: the next layer's z', r' [N] (out then holds fp16 codes), or null
     int qmax_out;             // with zq: the next layer's qmax
-    bool pdl;                 // launched as a programmatic dependent of the kernel that wrote q (weights are
-                              // read before that kernel ends, codes only after)
+    bool pdl;                 // (set by launch_linear) launched as a programmatic dependent of the kernel
+                              // before it on the stream: the kernel reads codes, outputs and workspace only
+                              // after that kernel ends, and may prefetch weights into L2 before
+    bool weights_early = false;  // that kernel is this call's own quantize kernel (ot_linear_fused), which
+                                 // started after every earlier writer: weights may be loaded before it ends
     int q_fmt = 0;            // kCodesF16: q holds fp16 codes; kCodesI8: int8 codes; kActF16: fp16
                               // activations [M, ldx] that the kernel quantizes with xz, xr, qmax_in
     const float *xz = nullptr, *xr = nullptr;  // kActF16: z, r [K]
