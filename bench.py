@@ -271,6 +271,17 @@ def run_ours(args):
     cfg, layer_shapes = _workload_desc()
     bits_a, bits_w = BITS
 
+    if args.profile_decode or args.profile_linear:
+        # profiler runs of the decode- / mid-sized linears only: nothing else is set up
+        tokens = args.profile_linear or 0
+        res = bench_decode(dev, peaks, reps=args.steps) if args.profile_decode else \
+            profile_linears(dev, tokens, args.steps, args.warmup)
+        torch.cuda.synchronize()
+        if rank == 0:
+            print(json.dumps({"profile_run": "decode" if args.profile_decode else f"linear-{tokens}",
+                              "steps": args.steps, "result": res}), flush=True)
+        return
+
     # ---- offline: inputs, calibration, fold (each rank its own replica) ----
     layers, xs, calib_ms, calib_bytes, fold_ms = _build_layers(dev, WORKLOAD_CFG, TOKENS, BITS,
                                                                8192 if args.profile else None)
@@ -288,12 +299,6 @@ def run_ours(args):
         step()
     torch.cuda.synchronize()
 
-    if args.profile_decode:
-        dec = bench_decode(dev, peaks, reps=args.steps)
-        torch.cuda.synchronize()
-        if rank == 0:
-            print(json.dumps({"profile_run": "decode", "steps": args.steps, "decode": dec}), flush=True)
-        return
     if args.profile:
         # small, short run for profilers: the steps only, nothing else
         for _ in range(args.steps):
@@ -578,6 +583,30 @@ def bench_asym(dev, layers, xs, ops_step, ms_sym, reps: int = 200, t_cal: int = 
             "ms_per_step": round(ms, 4), "tops": round(ops_step / (ms * 1e-3) / 1e12, 1),
             "over_symmetric_step": round(ms / ms_sym, 4),
             "gemm_us_per_layer": [round(v * 1e3, 2) for v in gemm_ms]}
+
+
+def profile_linears(dev, tokens: int, steps: int, warmup: int):
+    """For profilers: `warmup` then `steps` eager calls of ot_linear on the
+    OPT-13B QKV and fc2 shapes (Int6 codes and weights drawn directly) at
+    `tokens` tokens, QKV then fc2 in each step."""
+    import torch
+
+    from paper_2406_18832_gb300 import binding, synth
+    c = synth.CONFIGS[3]
+    ws = torch.zeros(binding.ot_linear_workspace_size(), dtype=torch.uint8, device=dev)
+    g = torch.Generator(device=dev).manual_seed(4100)
+    args = []
+    for li in (0, 3):
+        N, K = c.layers[li].N, c.layers[li].K
+        qw = torch.randint(-31, 32, (N, K), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+        q = torch.randint(-31, 32, (tokens, K), generator=g, device=dev, dtype=torch.int32).half()
+        args.append((q, qw, torch.rand(N, generator=g, device=dev) * 1e-3, torch.zeros(N, device=dev),
+                     torch.empty(tokens, N, dtype=torch.float16, device=dev)))
+    for k in range(warmup + steps):
+        for q, qw, sw, bf, y in args:
+            binding.ot_linear(q, qw, sw, bf, 6, 6, y, workspace=ws)
+    torch.cuda.synchronize()
+    return {"tokens": tokens, "layers": ["qkv 5120->15360", "fc2 20480->5120"], "calls": 2 * (warmup + steps)}
 
 
 def bench_token_sweep(dev, peaks, reps: int = 20):
@@ -1180,6 +1209,8 @@ def main():
                     help="profiler run of the decode-sized linears only (after the setup)")
     ap.add_argument("--profile", action="store_true",
                     help="profiler run: 8192 calibration tokens, the timed steps only, no report")
+    ap.add_argument("--profile-linear", type=int, default=0, metavar="TOKENS",
+                    help="profiler run of the OPT-13B QKV and fc2 linears at TOKENS tokens only")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
