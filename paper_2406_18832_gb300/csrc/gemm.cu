@@ -444,7 +444,8 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
                     for (int i0 = 0; i0 < BN / 16; i0 += 4) {
                         uint4 v[4];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) v[i] = *reinterpret_cast<const uint4 *>(bt + (r0 + 16 * (i0 + i)) * 128);
+                        for (int i = 0; i < 4; ++i)
+                            v[i] = *reinterpret_cast<const uint4 *>(bt + (r0 + 16 * (i0 + i)) * 128);
 #pragma unroll
                         for (int i = 0; i < 4; ++i)
                             *reinterpret_cast<uint4 *>(bt + (r0 + 16 * (i0 + i)) * 128) =

@@ -592,8 +592,10 @@ cudaError_t launch_linear_gemv(const LinearArgs &a, int kcb, cudaStream_t st) {
         return one ? run_gemv<1, false, kGvX>(tm_w, tm_a, p, st, d) : run_gemv<2, false, kGvX>(tm_w, tm_a, p, st, d);
     if (i8) {
         if (a.out_s32)
-            return one ? run_gemv<1, true, kGvI8>(tm_w, tm_a, p, st, d) : run_gemv<2, true, kGvI8>(tm_w, tm_a, p, st, d);
-        return one ? run_gemv<1, false, kGvI8>(tm_w, tm_a, p, st, d) : run_gemv<2, false, kGvI8>(tm_w, tm_a, p, st, d);
+            return one ? run_gemv<1, true, kGvI8>(tm_w, tm_a, p, st, d)
+                       : run_gemv<2, true, kGvI8>(tm_w, tm_a, p, st, d);
+        return one ? run_gemv<1, false, kGvI8>(tm_w, tm_a, p, st, d)
+                   : run_gemv<2, false, kGvI8>(tm_w, tm_a, p, st, d);
     }
     if (a.out_s32)
         return one ? run_gemv<1, true, kGvF16>(tm_w, tm_a, p, st, d) : run_gemv<2, true, kGvF16>(tm_w, tm_a, p, st, d);
