@@ -35,6 +35,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <algorithm>
 #include <atomic>
 #include <mutex>
 
@@ -1183,27 +1184,44 @@ int pair_max_clusters() {
 }
 
 // Token tiles per group of the pair kernel's tile order (pair_tile), from an
-// estimate of the DRAM bytes each order reads.  With all token tiles in one
-// group (the plain order) the clusters of one round touch every token tile,
-// and when the codes exceed what L2 keeps they are read again every round.  A
-// group of G token tiles whose codes stay in L2 reads the codes once and the
-// weights once per group.  Measured on GB300: OPT-66B fc1 (4096 tokens,
-// K = 9216; 75 MB of codes) read 3.3 GB per launch in the plain order,
-// against 415 MB of operands.
+// estimate of the DRAM bytes each order reads.  Two estimates, the smaller
+// taken:
+//  - L2 keeps a group's codes while the weight tiles stream past them: the
+//    codes are read once, the weights once per group (when G token tiles of
+//    codes fit beside the stream).  Measured on GB300: OPT-66B fc1 (4096
+//    tokens, K = 9216; 75 MB of codes) read 3.3 GB per launch in the plain
+//    order, 1.17 GB with 11 token tiles per group, against 415 MB of operands.
+//  - otherwise the clusters of one round (a tile each, moving along k at
+//    about the same pace) share what they read at about the same time, so a
+//    round reads the distinct token tiles and weight tiles it touches.  With
+//    K = 36864 (OPT-66B fc2) a tile's operands alone are 24 MB: 7 token
+//    tiles per group read 3.0 GB per launch against 4.0 GB in the plain order
+//    (and ran 2 % faster).
 int pair_group_m(int64_t M, int64_t N, int64_t K, int clusters) {
     constexpr double kL2Keep = 48.0 * (1 << 20);  // codes a group may keep in L2 beside the weight stream
     const int64_t m_tiles = (M + kPairBN - 1) / kPairBN;
     const int64_t n_pairs = (N + 2 * kBM - 1) / (2 * kBM);
-    const double tile_codes = (double)kPairBN * (double)K * 2.0;
+    const int64_t cl = clusters > 0 ? clusters : 1;
+    const double tile_codes = (double)kPairBN * (double)K * 2.0, tile_weights = 2.0 * kBM * (double)K;
     const double codes = tile_codes * (double)m_tiles, weights = (double)N * (double)K;
-    const double rounds = (double)(m_tiles * n_pairs) / (double)(clusters > 0 ? clusters : 1);
-    // plain order: codes once if they fit, else once per round (plus the weights once)
-    const double plain = (codes <= kL2Keep ? codes : codes * (rounds > 1.0 ? rounds : 1.0)) + weights;
+    const double rounds = std::max(1.0, (double)(m_tiles * n_pairs) / (double)cl);
+    auto per_rounds = [&](int64_t g) {
+        int64_t toks, prs;
+        if (cl <= g * n_pairs) {
+            toks = std::min(g, cl);
+            prs = (cl + g - 1) / g;
+        } else {
+            toks = std::min(m_tiles, (cl + n_pairs - 1) / n_pairs);
+            prs = n_pairs;
+        }
+        return rounds * ((double)toks * tile_codes + (double)prs * tile_weights);
+    };
+    const double plain = codes <= kL2Keep ? std::min(codes + weights, per_rounds(m_tiles)) : per_rounds(m_tiles);
     int64_t best_g = m_tiles;
     double best = plain;
     for (int64_t g = 1; g < m_tiles; ++g) {
-        if ((double)g * tile_codes > kL2Keep) break;
-        const double t = codes + (double)((m_tiles + g - 1) / g) * weights;
+        double t = per_rounds(g);
+        if ((double)g * tile_codes <= kL2Keep) t = std::min(t, codes + (double)((m_tiles + g - 1) / g) * weights);
         if (t < best) {
             best = t;
             best_g = g;
