@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
     // the TMA and MMA roles run their loops with the whole warp and issue from one elected lane
     // registers: 512 threads x 128 at launch (kTokF16); with the token warps
     // 640 x 96, then per warpgroup 48 / 72 / 144 / 144 / 72
-    if (warp < 4) {
+    if (warp < kWarpConv0) {
         if constexpr (kTok != kTokF16) regs_dec<48>();
         if (warp == kWarpTma) {
             uint32_t it = 0;
