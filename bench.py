@@ -1113,6 +1113,49 @@ def _new_timings():
                 quantize_s=0.0, matmul_s=0.0, epilogue_s=0.0)
 
 
+def cpu_single_thread():
+    """The oracle's plain C functions on one host thread: config 1's whole step
+    (calibration on its 64 tokens, parameters, fold, then quantize / int64
+    product / epilogue of its 16 tokens) and config 2's out layer (4096 ->
+    4096; calibration on 2048 tokens, the whole fold, a 64-token sample of the
+    online steps).  Seconds per step and online TOPS."""
+    import numpy as np
+
+    import oracle
+    from paper_2406_18832_gb300 import synth
+    out = {}
+    for name, cfg, li, tokens, cal in (("config1", 1, 0, 16, 64), ("config2_out", 2, 1, 64, 2048)):
+        layer = synth.CONFIGS[cfg].layers[li]
+        w, b = synth.weights(cfg, li, layer)
+        xc = synth.activations(cfg, li, layer, cal, 3).numpy()
+        x = synth.activations(cfg, li, layer, tokens, 4).numpy()
+        w, b = w.numpy(), b.numpy()
+        st = {}
+        t = time.perf_counter()
+        mn, mx = oracle.calibrate(xc)
+        st["calibrate"] = time.perf_counter() - t
+        t = time.perf_counter()
+        z, s_, r = oracle.params(mn, mx, 8)
+        st["params"] = time.perf_counter() - t
+        t = time.perf_counter()
+        qw, sw, bf = oracle.fold(w, b, z, s_, 8)
+        st["fold"] = time.perf_counter() - t
+        t = time.perf_counter()
+        q = oracle.quantize(x, z, r, 8)
+        st["quantize"] = time.perf_counter() - t
+        t = time.perf_counter()
+        acc = oracle.matmul(q, qw)
+        st["matmul"] = time.perf_counter() - t
+        t = time.perf_counter()
+        oracle.epilogue(acc, sw, bf, layer.relu_out)
+        st["epilogue"] = time.perf_counter() - t
+        online = st["quantize"] + st["matmul"] + st["epilogue"]
+        out[name] = {"tokens": tokens, "K": layer.K, "N": layer.N, "calibration_tokens": cal,
+                     "per_step_s": {k: round(v, 6) for k, v in st.items()},
+                     "online_tops": round(2.0 * tokens * layer.K * layer.N / online / 1e12, 6)}
+    return out
+
+
 def cpu_baseline(host, budget_s=12.0):
     """Time the oracle, as it stands, per step of the headline workload on the
     host cores (its C functions over row ranges in one thread per core):
@@ -1142,7 +1185,8 @@ def cpu_baseline(host, budget_s=12.0):
                            "matmul": round(tm["matmul_s"], 3), "epilogue": round(tm["epilogue_s"], 3)},
             "calibrate_gbs": round(tm["calibrate_bytes"] / tm["calibrate_s"] / 1e9, 2),
             "fold_mweights_per_s": round(tm["fold_weights"] / tm["fold_s"] / 1e6, 1),
-            "threads": "one per core of os.sched_getaffinity, rows (or channels) split evenly"}
+            "threads": "one per core of os.sched_getaffinity, rows (or channels) split evenly",
+            "single_thread": cpu_single_thread()}
 
 
 def run_reference(args):
