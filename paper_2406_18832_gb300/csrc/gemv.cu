@@ -2,8 +2,8 @@
 // counts (M <= 16), where the product is bound by reading the int8 weights
 // from HBM (each weight byte is used by only M tokens).
 //
-// At a few tokens a tcgen05 tile wastes most of its N width and its fixed
-// per-MMA cost caps the weight stream; warp-level mma.sync m16n8k16 (f16 in,
+// At a few tokens a tcgen05 tile wastes most of its N width and its k-loop
+// is bound by its barrier hand-offs; warp-level mma.sync m16n8k16 (f16 in,
 // f32 accumulate) has throughput to spare, so the kernel is a weight stream
 // (measured on GB300, OPT-13B QKV and fc2 shapes: faster than the tcgen05
 // kernel up to 16 tokens, slower from 17):
@@ -18,9 +18,12 @@
 //     special case.  Measured on GB300, the TMA unit of an SM completes about
 //     one box per 176 ns whatever its size up to 8 KB, so boxes must be large:
 //     8 KB boxes held the stream near 2.5 TB/s, 32 KB boxes reach ~7 TB/s;
-//   - the ring has no producer warp: the first S units are issued at start,
-//     and the last of the 16 warps to finish with a slot (a shared counter)
-//     refills it with the unit S places later;
+//   - the first S units are issued at start; a producer warp (warp 16) then
+//     refills each slot with the unit S places later as soon as the 16
+//     consumer warps have arrived on the slot's empty barrier.  Measured on
+//     GB300 (OPT-13B QKV / fc2, 1 token): 15.0 / 20.5 us against 17.3 / 23.1
+//     with the refill issued by the last consumer warp done with the slot,
+//     which then lagged behind the others and tended to be last again;
 //   - the weights are the MMA's m16 operand and the tokens its n8 operand
 //     (ceil(M / 8) token groups): warp w takes the 64-wide window w % 4 of
 //     every stage and weight rows 32 (w / 4) .. + 31 (two m16 groups).  Lane l
@@ -63,7 +66,7 @@ constexpr int kGvKS = 256;                        // K per unit / stage (= the T
 constexpr int kGvWin = 64;                        // K per MMA window
 constexpr int kGvWindows = kGvKS / kGvWin;        // windows per stage (4)
 constexpr int kGvWarps = 16;
-constexpr int kGvThreads = kGvWarps * 32;
+constexpr int kGvThreads = kGvWarps * 32;            // consumer threads (+ one producer warp)
 constexpr int kGvWBox = kGvRows * 128;           // weight box: 128 rows x 128 bytes, 128-byte swizzle
 constexpr int kGvWBytes = 2 * kGvWBox;            // weights of a stage (two boxes)
 constexpr int kGvMaxStages = 8;
@@ -149,20 +152,23 @@ __device__ __forceinline__ void store_out(const GvParams &p, int m, int n, int32
     }
 }
 
+// Named barrier 1 over the 16 consumer warps (the producer warp takes no part).
+__device__ __forceinline__ void consumers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kGvThreads) : "memory"); }
+
 // TN token groups of 8 (the MMA's n8); kTokG: the token box's format.
 template <int TN, bool kS32, int kTokG>
-__global__ void __launch_bounds__(kGvThreads, 1)
+__global__ void __launch_bounds__(kGvThreads + 32, 1)
     linear_gemv_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_a,
                        const GvParams p) {
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment: the swizzle pattern of a TMA box repeats every 1024 bytes
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(base);
-    unsigned *done = reinterpret_cast<unsigned *>(full + kGvMaxStages);  // warps finished with a slot, ever
-    unsigned *loads = done + kGvMaxStages;                                // units loaded into a slot, ever
+    unsigned *loads = reinterpret_cast<unsigned *>(full + kGvMaxStages);  // units loaded into a slot, ever
     volatile int *abort = reinterpret_cast<volatile int *>(loads + kGvMaxStages);
     unsigned long long *epoch_s = reinterpret_cast<unsigned long long *>(base + 192);  // this launch's epoch
     uint64_t *qready = reinterpret_cast<uint64_t *>(base + 256);  // kGvX: the slot's codes are quantized
+    uint64_t *empty = reinterpret_cast<uint64_t *>(base + 320);   // the 16 consumer warps are done with the slot
     int32_t(*red)[kGvRows + 1] = reinterpret_cast<int32_t(*)[kGvRows + 1]>(base + kGvHeader);  // [TN*8]
     uint8_t *ring = base + ((kGvHeader + p.red_bytes + 1023) & ~1023);
 
@@ -207,14 +213,14 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         pol_w = l2_policy_evict_first();
         pol_a = l2_policy_evict_last();
     }
-    for (int i = threadIdx.x; i < TN * 8 * (kGvRows + 1); i += kGvThreads) (&red[0][0])[i] = 0;
+    for (int i = threadIdx.x; i < TN * 8 * (kGvRows + 1); i += blockDim.x) (&red[0][0])[i] = 0;
     if (threadIdx.x == 0) {
         tma_prefetch_desc(&tm_w);
         tma_prefetch_desc(&tm_a);
         for (int s = 0; s < S; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
             mbar_init(smem_u32(&qready[s]), kGvWarps);
-            done[s] = 0;
+            mbar_init(smem_u32(&empty[s]), kGvWarps);
             loads[s] = 0;
         }
         *abort = 0;
@@ -267,6 +273,31 @@ __global__ void __launch_bounds__(kGvThreads, 1)
     __syncthreads();
     // the next linear on the stream may launch now (it waits for this one before reading anything this writes)
     grid_dep_launch();
+    if (warp == kGvWarps) {
+        // producer warp: refills each slot with the unit S places later once
+        // the 16 consumer warps are done with it
+        if (lane == 0) {
+            int64_t tile = tile0;
+            int ks = ks0 + S;
+            while (ks >= nks) {
+                ks -= nks;
+                ++tile;
+            }
+            for (int64_t i = S; u_begin + i < u_end; ++i) {
+                const int slot = (int)(i % S);
+                if (!mbar_wait(smem_u32(&empty[slot]), ((uint32_t)(i / S) & 1) ^ 1, abort, p.status)) break;
+                load_unit(slot, tile, ks);
+                if (++ks == nks) {
+                    ks = 0;
+                    ++tile;
+                }
+            }
+            // teardown: every copy issued must land before the CTA's shared memory goes away
+            for (int s2 = 0; s2 < S; ++s2)
+                if (loads[s2] > 0) wait_teardown_status(smem_u32(&full[s2]), (loads[s2] - 1) & 1, p.status);
+        }
+        return;
+    }
 
     const int t = lane & 3, r = lane >> 2;
     const int win = warp % kGvWindows, rp = warp / kGvWindows;  // window; rows 32 rp .. 32 rp + 31
@@ -403,20 +434,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 }
             }
             __syncwarp();
-            if (lane == 0) {
-                // the last warp done with this slot refills it with the unit S places on
-                __threadfence_block();
-                if (atomicAdd(&done[slot], 1u) % kGvWarps == kGvWarps - 1 && u + S < u_end && !*abort) {
-                    __threadfence_block();
-                    int64_t tile2 = tile;
-                    int ks2 = ks + S;
-                    while (ks2 >= nks) {
-                        ks2 -= nks;
-                        ++tile2;
-                    }
-                    load_unit(slot, tile2, ks2);
-                }
-            }
+            if (lane == 0) mbar_arrive(smem_u32(&empty[slot]));
             if (++slot == S) {
                 slot = 0;
                 phase ^= 1;
@@ -426,7 +444,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
         // ---- end of this CTA's part of the tile: add the warps' totals ----
         in_chunk = 0;
         flush();
-        __syncthreads();
+        consumers_sync();
         const int n0 = (int)(tile * kGvRows);
         if (mine == nks) {
             for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
@@ -445,7 +463,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 red[m][c] = 0;
             }
             __threadfence();
-            __syncthreads();
+            consumers_sync();
             if (threadIdx.x == 0) {
                 __threadfence();
                 atomicExch(p.flags + blockIdx.x, *epoch_s);
@@ -467,7 +485,7 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                     }
                 }
             }
-            __syncthreads();
+            consumers_sync();
             for (int idx = threadIdx.x; idx < M * kGvRows; idx += kGvThreads) {
                 const int m = idx / kGvRows, c = idx % kGvRows;
                 int32_t s = red[m][c];
@@ -476,15 +494,13 @@ __global__ void __launch_bounds__(kGvThreads, 1)
                 if (n0 + c < N) store_out<kS32>(p, m, n0 + c, s);
             }
         }
-        __syncthreads();  // red is reused by the next tile
+        consumers_sync();  // red is reused by the next tile
         ks = 0;
         ++tile;
     }
     // teardown (only matters after a timeout): every copy issued must land
     // before the CTA's shared memory goes away
     if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s)
-            if (loads[s] > 0) wait_teardown_status(smem_u32(&full[s]), (loads[s] - 1) & 1, p.status);
         if (!p.whole && atomicAdd(p.ctl + 1, 1ull) == (unsigned long long)gridDim.x - 1) {
             // the last CTA of the launch: hand the epoch to the next launch
             p.ctl[1] = 0;
@@ -513,7 +529,7 @@ cudaError_t run_gemv(const CUtensorMap &tm_w, const CUtensorMap &tm_a, const GvP
     if (p.stages > kGvMaxStages) p.stages = kGvMaxStages;
     if (p.stages < 2) return cudaErrorInvalidConfiguration;
     const size_t smem = 1024 + ring_off + (size_t)p.stages * p.stage_bytes;
-    return launch_kernel(linear_gemv_kernel<TN, kS32, kTokG>, dim3(p.grid), dim3(kGvThreads), smem, st, pdl, tm_w,
+    return launch_kernel(linear_gemv_kernel<TN, kS32, kTokG>, dim3(p.grid), dim3(kGvThreads + 32), smem, st, pdl, tm_w,
                          tm_a, p);
 }
 
