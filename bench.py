@@ -384,13 +384,28 @@ def run_ours(args):
     del layers, xs, qbufs, ybufs
     torch.cuda.empty_cache()
 
+    def fresh():
+        # each stage allocates its tensors anew rather than from blocks the
+        # caching allocator kept from earlier, larger stages (measured: a
+        # decode point drawn from such blocks ran 15-25 % slow in one run of
+        # three, in the same place each time; fresh allocations did not)
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+
     step6 = bench_step6(dev, peaks, max(5, min(200, args.steps)), args.warmup)
+    fresh()
     block = None if args.no_block else bench_block(dev)
+    fresh()
     decode = bench_decode(dev, peaks)
+    fresh()
     lnq = bench_layernorm(dev, peaks)
+    fresh()
     qsweep = bench_quantize_sweep(dev, peaks)
+    fresh()
     sweep = bench_token_sweep(dev, peaks)
+    fresh()
     per_tok = bench_per_token(dev, peaks)
+    fresh()
     clip = bench_clipping(dev, peaks, step6.pop("_calib_ms0"))
 
     cpu = None
@@ -846,24 +861,43 @@ def bench_clipping(dev, peaks, minmax, reps: int = 3):
             "minmax_ms": round(minmax_ms, 3), "note": "two passes over the data (radix select on fp16 keys)"}
 
 
+def _warm_graph(graph, min_s: float = 0.05):
+    """Replay `graph` until at least `min_s` seconds of it have run (three
+    replays at least).  A point that follows a long high-power one (the block,
+    the headline step, the 4096-token points of the sweep) otherwise times
+    while the clocks are still recovering: measured, such a decode point ran
+    15-25 % slow in some runs."""
+    import torch
+    t0 = time.perf_counter()
+    n = 0
+    while n < 3 or time.perf_counter() - t0 < min_s:
+        graph.replay()
+        torch.cuda.synchronize()
+        n += 1
+
+
 def _graph_ms(calls, reps):
-    """ms per call of `calls` (reps calls) captured in a CUDA graph, replayed 3 times."""
+    """ms per call of `calls` (reps calls) captured in a CUDA graph: warm-up
+    replays (_warm_graph), then the median of three timed rounds of five
+    replays."""
     import torch
     calls()
     torch.cuda.synchronize()
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
         calls()
-    graph.replay()
-    torch.cuda.synchronize()
+    _warm_graph(graph)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
+    rounds = []
     for _ in range(3):
-        graph.replay()
-    e1.record()
-    torch.cuda.synchronize()
+        e0.record()
+        for _ in range(5):
+            graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        rounds.append(e0.elapsed_time(e1) / (5 * reps))
     del graph
-    return e0.elapsed_time(e1) / (3 * reps)
+    return statistics.median(rounds)
 
 
 def bench_decode(dev, peaks, reps: int = 50):
@@ -897,27 +931,13 @@ def bench_decode(dev, peaks, reps: int = 50):
                 for i in range(reps):
                     binding.ot_linear(q, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
 
-            for i in range(max(3, copies)):
-                binding.ot_linear(q, qws[i % copies], sw, bf, 6, 6, y, workspace=ws)
-            torch.cuda.synchronize()
+            ms = _graph_ms(calls, reps)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
             calls()
             e1.record()
             torch.cuda.synchronize()
             eager_ms = e0.elapsed_time(e1) / reps
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph):
-                calls()
-            graph.replay()
-            torch.cuda.synchronize()
-            e0.record()
-            for _ in range(3):
-                graph.replay()
-            e1.record()
-            torch.cuda.synchronize()
-            ms = e0.elapsed_time(e1) / (3 * reps)
-            del graph
             gbs = layer.N * layer.K / (ms * 1e-3) / 1e9
             # with the activation quantization in front: two calls, or the
             # fused call (the linear a programmatic dependent of the quantize)
