@@ -274,7 +274,7 @@ ot_status ot_linear_fused(const void *x_f16, int64_t M, int64_t K, int64_t ldx, 
     if (e != cudaSuccess) return from_cuda(e);
     ot::LinearArgs a{q_f16, qw, sw, b_fold, y_f16, M, N, K, ldy, bits_a, bits_w, relu ? 1 : 0, false,
                      workspace, workspace ? workspace_bytes : 0};
-    a.weights_early = true;  // the quantize kernel just launched started after every earlier writer
+    a.weights_early = true;  // the quantize kernel releases the linear only after every earlier kernel ended
     return from_cuda(ot::launch_linear(a, st));
 }
 

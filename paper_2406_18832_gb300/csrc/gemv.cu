@@ -229,7 +229,8 @@ __global__ void __launch_bounds__(kGvThreads + 32, 1)
         // the stream may still be running until grid_dep_wait() returns; until
         // then only the first units' weights are touched: loaded into the ring
         // when that kernel is this call's own quantize kernel (weights_early:
-        // it started after every earlier writer of the weights), else
+        // it lets this one start only after every earlier kernel, any writer
+        // of the weights, has completed), else
         // prefetched into L2, which stays coherent with any write that kernel
         // makes.  The codes and the workspace are read only after the wait.
         // Without such a launch the loads go out unit by unit, so that the

@@ -197,6 +197,10 @@ template <bool kF16Out, int kCh, int kWpr>
 __global__ void __launch_bounds__(kLnThreads, kCh <= 4 ? 4 : 2) layernorm_quantize_rows_kernel(
     const __half *__restrict__ h, int64_t M, int64_t K, int64_t ldh, const float *__restrict__ gamma_r,
     const float *__restrict__ beta_r, float eps, int qmax, void *q, int32_t *rowsum) {
+    // launched as a programmatic dependent: the kernel before this one has
+    // written h; the next one starts only after that (see quantize_kernel)
+    grid_dep_wait();
+    grid_dep_launch();
     constexpr int kRows = kLnWarps / kWpr;
     __shared__ LnSums part[kLnWarps];
     __shared__ float2 stat[kRows];  // mean, rstd; rstd is NaN for a row with non-finite values
@@ -284,6 +288,8 @@ __global__ void __launch_bounds__(kLnThreads) layernorm_quantize_kernel(const __
                                                                         const float *__restrict__ gamma_r,
                                                                         const float *__restrict__ beta_r, float eps,
                                                                         int qmax, void *q, int32_t *rowsum) {
+    grid_dep_wait();
+    grid_dep_launch();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int64_t m = (int64_t)blockIdx.x * kLnWarps + warp; m < M; m += (int64_t)gridDim.x * kLnWarps) {
         const __half *row = h + m * ldh;
@@ -352,19 +358,17 @@ cudaError_t run_layernorm_quantize(const __half *h, int64_t M, int64_t K, int64_
         return (unsigned)(ctas < (1 << 30) ? ctas : (1 << 30));
     };
 #define OT_LN_ROWS(C, W)                                                                                      \
-    layernorm_quantize_rows_kernel<kF16Out, C, W><<<grid_for(kLnWarps / W), kLnThreads, 0, st>>>(              \
-        h, M, K, ldh, gamma_r, beta_r, eps, qmax, q, rowsum)
-    if (ch <= 4) OT_LN_ROWS(4, 1);
-    else if (ch <= 8) OT_LN_ROWS(4, 2);
-    else if (ch <= 16) OT_LN_ROWS(4, 4);
-    else if (ch <= 32) OT_LN_ROWS(4, 8);
-    else if (ch <= 48) OT_LN_ROWS(6, 8);
-    else if (ch <= 64) OT_LN_ROWS(8, 8);
-    else
-        layernorm_quantize_kernel<kF16Out, 0><<<grid_for(kLnWarps), kLnThreads, 0, st>>>(h, M, K, ldh, gamma_r, beta_r,
-                                                                                        eps, qmax, q, rowsum);
+    launch_kernel(layernorm_quantize_rows_kernel<kF16Out, C, W>, dim3(grid_for(kLnWarps / W)), dim3(kLnThreads), 0, \
+                  st, true, h, M, K, ldh, gamma_r, beta_r, eps, qmax, q, rowsum)
+    if (ch <= 4) return OT_LN_ROWS(4, 1);
+    if (ch <= 8) return OT_LN_ROWS(4, 2);
+    if (ch <= 16) return OT_LN_ROWS(4, 4);
+    if (ch <= 32) return OT_LN_ROWS(4, 8);
+    if (ch <= 48) return OT_LN_ROWS(6, 8);
+    if (ch <= 64) return OT_LN_ROWS(8, 8);
 #undef OT_LN_ROWS
-    return cudaGetLastError();
+    return launch_kernel(layernorm_quantize_kernel<kF16Out, 0>, dim3(grid_for(kLnWarps)), dim3(kLnThreads), 0, st, true,
+                         h, M, K, ldh, gamma_r, beta_r, eps, qmax, q, rowsum);
 }
 
 }  // namespace

@@ -57,7 +57,8 @@ struct LinearArgs {
                               // before it on the stream: the kernel reads codes, outputs and workspace only
                               // after that kernel ends, and may prefetch weights into L2 before
     bool weights_early = false;  // that kernel is this call's own quantize kernel (ot_linear_fused), which
-                                 // started after every earlier writer: weights may be loaded before it ends
+                                 // releases its dependents only after every earlier kernel (any writer of
+                                 // the weights) has completed: weights may be loaded before it ends
     int q_fmt = 0;            // kCodesF16: q holds fp16 codes; kCodesI8: int8 codes; kActF16: fp16
                               // activations [M, ldx] that the kernel quantizes with xz, xr, qmax_in
     const float *xz = nullptr, *xr = nullptr;  // kActF16: z, r [K]

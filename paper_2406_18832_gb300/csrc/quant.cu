@@ -49,7 +49,12 @@ __global__ void __launch_bounds__(256) quantize_kernel(const __half *__restrict_
                                                        int64_t ldx, const float *__restrict__ z,
                                                        const float *__restrict__ r, int qmax, void *q,
                                                        int32_t *rowsum) {
-    grid_dep_launch();  // a linear launched as a programmatic dependent may start its weight loads now
+    // Launched as a programmatic dependent: wait for the kernel before this one
+    // (its writes of x, z, r), then let the next one start -- only then, so a
+    // dependent linear that loads its weights before its own wait starts after
+    // every earlier kernel (any writer of the weights) has completed.
+    grid_dep_wait();
+    grid_dep_launch();
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int64_t c0 = (int64_t)blockIdx.x * 256 + tx * 8;
     const bool active = c0 < K;  // K % 8 == 0: a lane's 8 channels are whole or absent
@@ -198,9 +203,11 @@ cudaError_t launch_quantize(const void *x, int64_t M, int64_t K, int64_t ldx, co
         else
             quantize_kernel<false, true><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, rowsum);
     } else if (fmt == OT_CODE_F16) {
-        quantize_kernel<true, false><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, nullptr);
+        return launch_kernel(quantize_kernel<true, false>, grid, dim3(256), 0, st, true, xh, M, K, ldx, z, r, qmax, q,
+                             (int32_t *)nullptr);
     } else {
-        quantize_kernel<false, false><<<grid, 256, 0, st>>>(xh, M, K, ldx, z, r, qmax, q, nullptr);
+        return launch_kernel(quantize_kernel<false, false>, grid, dim3(256), 0, st, true, xh, M, K, ldx, z, r, qmax, q,
+                             (int32_t *)nullptr);
     }
     return cudaGetLastError();
 }
