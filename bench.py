@@ -271,6 +271,21 @@ def run_ours(args):
     cfg, layer_shapes = _workload_desc()
     bits_a, bits_w = BITS
 
+    if args.profile_opt67b:
+        # profiler runs of the OPT-6.7B step (QKV, out, fc1, fc2 at 2048 tokens, W8A8): quantize then
+        # linear per layer, `warmup` + `steps` steps, nothing else
+        layers, xs, _, _, _ = _build_layers(dev, STEP6_CFG, STEP6_TOKENS, BITS, 8192)
+        c6 = _workload_desc(STEP6_CFG)[0]
+        qb = [torch.empty(STEP6_TOKENS, l.K, dtype=torch.float16, device=dev) for l in c6.layers]
+        yb = [torch.empty(STEP6_TOKENS, l.N, dtype=torch.float16, device=dev) for l in c6.layers]
+        for _ in range(args.warmup + args.steps):
+            for i, (ql, _, _) in enumerate(layers):
+                ql.forward(xs[i], qb[i], yb[i])
+        torch.cuda.synchronize()
+        if rank == 0:
+            print(json.dumps({"profile_run": "opt67b", "steps": args.steps, "warmup": args.warmup}), flush=True)
+        return
+
     if args.profile_decode or args.profile_linear:
         # profiler runs of the decode- / mid-sized linears only: nothing else is set up
         tokens = args.profile_linear or 0
@@ -1273,6 +1288,8 @@ def main():
                     help="profiler run of the decode-sized linears only (after the setup)")
     ap.add_argument("--profile", action="store_true",
                     help="profiler run: 8192 calibration tokens, the timed steps only, no report")
+    ap.add_argument("--profile-opt67b", action="store_true",
+                    help="for profilers: only the OPT-6.7B step (2048 tokens), warmup + steps times")
     ap.add_argument("--profile-linear", type=int, default=0, metavar="TOKENS",
                     help="profiler run of the OPT-13B QKV and fc2 linears at TOKENS tokens only")
     args = ap.parse_args()
