@@ -94,3 +94,43 @@ def test_chained_linears_back_to_back_and_in_a_graph(M):
         graph.replay()
         torch.cuda.synchronize()
         assert np.array_equal(y.cpu().numpy().view(np.uint16), ref.view(np.uint16))
+
+
+@pytest.mark.parametrize("M", [1, 16, 100, 300])
+def test_fused_call_reads_weights_folded_just_before(M):
+    """ot_linear_fused loads its first weights before the codes are ready
+    (decode: into its ring): the quantize kernel in front of it waits for the
+    kernel before it and only then releases the linear.  Two weight sets are
+    folded alternately into the same buffers, each fold followed at once by a
+    fused call on the same stream, nothing synchronized in between: every
+    output must be the oracle's for the weights folded just before it."""
+    from paper_2406_18832_gb300 import binding as B
+    g = torch.Generator().manual_seed(500 + M)
+    K, N, bits = 2048, 3072, 8
+    cal = (torch.randn(256, K, generator=g) * 2).half().numpy()
+    mn, mx = oracle.calibrate(cal)
+    z, s, r = oracle.params(mn, mx, bits)
+    ws_h = [(torch.randn(N, K, generator=g) * 0.03).half().numpy() for _ in range(2)]
+    bs_h = [(torch.randn(N, generator=g) * 0.1).half().numpy() for _ in range(2)]
+    folds = [oracle.fold(w, b, z, s, bits) for w, b in zip(ws_h, bs_h)]
+    xs = [(torch.randn(M, K, generator=g) * 2).half() for _ in range(6)]
+    refs = [oracle.linear(x.numpy(), *folds[i % 2], z, r, bits)[2] for i, x in enumerate(xs)]
+
+    dmn, dmx = _d(mn), _d(mx)
+    dz, ds, dr = (torch.empty(K, device=DEV) for _ in range(3))
+    qw = torch.empty(N, K, dtype=torch.int8, device=DEV)
+    sw, bf = torch.empty(N, device=DEV), torch.empty(N, device=DEV)
+    dw = [_d(w) for w in ws_h]
+    db = [_d(b) for b in bs_h]
+    dx = [x.to(DEV) for x in xs]
+    q = torch.empty(M, K, dtype=torch.float16, device=DEV)
+    ws = torch.zeros(B.ot_linear_workspace_size(), dtype=torch.uint8, device=DEV)
+    ys = [torch.empty(M, N, dtype=torch.float16, device=DEV) for _ in xs]
+    torch.cuda.synchronize()
+    for i, (x, y) in enumerate(zip(dx, ys)):
+        B.ot_fold_weights(dmn, dmx, bits, dw[i % 2], db[i % 2], bits, dz, ds, dr, qw, sw, bf)
+        B.ot_linear_fused(x, dz, dr, bits, qw, sw, bf, bits, q, y, workspace=ws)
+    torch.cuda.synchronize()
+    assert B.ot_get_device_status() == B.OT_OK
+    for i, (y, ref) in enumerate(zip(ys, refs)):
+        assert np.array_equal(y.cpu().numpy().view(np.uint16), ref.view(np.uint16)), f"call {i}"
