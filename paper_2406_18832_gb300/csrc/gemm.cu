@@ -9,10 +9,12 @@
 // kcb k-blocks with kcb * 64 * qmax_a * qmax_w <= 2^24; each chunk's fp32
 // accumulator is converted to int32 (exact) and summed in registers.
 //
-// Two kernels: linear_kernel (below; 16 < M <= 128, and any M when K % 128
-// != 0) and linear_pair_kernel (M > 128: CTA pairs, 192-token tiles; its own
-// comment further down).  The TMA and MMA roles of both run their loops with
-// the whole warp and issue from one elected lane.
+// Two kernels: linear_kernel (below; 16 < M <= 64, int8 codes and the
+// in-producer quantization up to 128 tokens, and any M when K % 128 != 0) and
+// linear_pair_kernel (K % 128 == 0 and M > 64: CTA pairs, 192-token tiles above
+// 128 tokens, 128-token tiles for 65-128; its own comment further down).  The
+// TMA and MMA roles of both run their loops with the whole warp and issue
+// from one elected lane.
 //
 // linear_kernel (one persistent CTA per SM, 16 warps):
 //   warp 0        TMA producer: per 64-wide k-block, the activation-code tile
@@ -597,7 +599,8 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
 }
 
 // ---------------------------------------------------------------------------
-// Wide-tile CTA-pair variant for prefill-sized token counts (M > 128).
+// Wide-tile CTA-pair variant: prefill-sized token counts (M > 128, 192-token
+// tiles) and 65-128 tokens (128-token tiles; PairCfg below).
 //
 // Measured on GB300: a cta_group::2 kind::f16 MMA of 256 x N x 16 runs at
 // the full tensor rate (4096 MACs per clock per SM, dependent accumulation,
@@ -611,14 +614,16 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
 // 192 tokens: per group of four k-blocks each CTA loads its own 128 int8
 // weight rows (32 KB, one copy) and half of the token tile (96 rows of fp16
 // codes, 48 KB, one copy); B is split along N between the pair and each
-// CTA's TMEM receives its 128 rows x 192 tokens of the accumulator.
+// CTA's TMEM receives its 128 rows x 192 tokens of the accumulator (the
+// 128-token tile: 64 token rows per CTA, 32 KB copies).
 // The converters widen each CTA's int8 weight rows to fp16 and store them in
 // TMEM as the MMA's A operand (tcgen05.st), so shared memory carries only
 // the TMA ingest, the converters' read of the int8 rows and the tensor
 // core's read of B.  TMEM (512 columns) holds two 192-column chunk
 // accumulators -- while the MMA fills one, the epilogue converts the other
 // (fp32 -> int32 conversions run at a quarter rate and would otherwise stall
-// the tensor core at every chunk boundary) -- and four 32-column A stages.
+// the tensor core at every chunk boundary) -- and four 32-column A stages
+// (the 128-token tile: two 128-column accumulators and eight A stages).
 // 192-token tiles cover 2048 tokens with 3 % padding.
 //   Rank 0 of the pair issues the MMAs.  The converters and epilogue warps
 //   of both CTAs signal rank 0's barriers; rank 0's commits arrive on the
@@ -629,37 +634,48 @@ __global__ void __launch_bounds__(lin_threads<kTok>(), 1)
 //   Warps: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator (warpgroup 0,
 //   48 regs); 4-7 and 16-19 converters, taking the even and the odd k-blocks
 //   of the CTA's sequence in turn (72 regs: one warp per 32 TMEM lanes could
-//   not keep up); 8-15 epilogue (144 regs: 96 int32 totals).
+//   not keep up); 8-15 epilogue (144 regs: PBN / 2 int32 totals).
 //   Needs K % 128 == 0 (the 3-D views must not reach past a row's end);
 //   other K use linear_kernel.
 // ---------------------------------------------------------------------------
-constexpr int kPairBN = 192;                      // tokens per pair tile (MMA N)
-constexpr int kPairHalf = kPairBN / 2;            // token rows per CTA (B is split along N)
-constexpr int kPairACol = 2 * kPairBN;            // TMEM: accumulators in [0, 2 kPairBN), then A stages
-constexpr int kAStages = (512 - kPairACol) / 32;  // 32-column fp16 A stages (128 rows x 64 k)
 constexpr int kGroupKB = 4;                       // k-blocks per TMA copy
 // 20 warps: 0 TMA producer, 1 MMA issuer, 2 TMEM allocator, 4-7 and 16-19
 // converters (even / odd k-blocks of the CTA's sequence), 8-15 epilogue
 constexpr int kPairThreads = 640;
 constexpr int kWarpConv1 = 16;
 constexpr int kWStages = 2;                       // weight stages: 2 x 128 rows x 128 int8, 128-byte swizzle (32 KB)
-constexpr int kBStages = 3;                       // token stages: 4 x 96 rows x 64 fp16, 128-byte swizzle (48 KB)
+constexpr int kBStages = 3;                       // token stages: 4 x PBN / 2 rows x 64 fp16, 128-byte swizzle
 constexpr uint32_t kWStageBytes = 2 * kBM * 128;
-constexpr uint32_t kBTileBytes = kPairHalf * 128;
-constexpr uint32_t kBStageBytes = kGroupKB * kBTileBytes;
-static_assert(kAStages >= 2, "A stage of k-block i is freed by the commit of k-block i - kAStages");
-static_assert(kPairBN % 32 == 0 && kPairHalf % 32 == 0, "the epilogue drains 32 columns at a time");
-static_assert(kBTileBytes % 1024 == 0, "each k-block of B is a whole number of 1024-byte swizzle atoms");
+// Tile width of a CTA pair: PBN tokens (the MMA's N), PBN / 2 token rows per
+// CTA; TMEM holds two PBN-column chunk accumulators and (512 - 2 PBN) / 32
+// A stages.  192 for prefill (M > 128): 2048 tokens in 11 tiles with 3 %
+// padding; 128 for 17-128 tokens: eight A stages instead of four, so the
+// cross-CTA hand-off round trip no longer bounds the k-loop.
+template <int PBN>
+struct PairCfg {
+    static constexpr int kBN = PBN;                   // tokens per pair tile (MMA N)
+    static constexpr int kHalf = PBN / 2;             // token rows per CTA (B is split along N)
+    static constexpr int kACol = 2 * PBN;             // TMEM: accumulators in [0, 2 kBN), then A stages
+    static constexpr int kAStg = (512 - kACol) / 32;  // 32-column fp16 A stages (128 rows x 64 k)
+    static constexpr uint32_t kBTileBytes = kHalf * 128;
+    static constexpr uint32_t kBStageBytes = kGroupKB * kBTileBytes;
+    static_assert(kAStg >= 2, "A stage of k-block i is freed by the commit of k-block i - kAStg");
+    static_assert(kBN % 32 == 0 && kHalf % 32 == 0, "the epilogue drains 32 columns at a time");
+    static_assert(kBTileBytes % 1024 == 0, "each k-block of B is a whole number of 1024-byte swizzle atoms");
+};
+constexpr int kPairBN = 192;  // the prefill tile
 
+template <int PBN>
 struct alignas(1024) SmemPair {
-    uint8_t b[kBStages][kBStageBytes];  // this CTA's 96 token rows of fp16 codes, [k-block][row][64 fp16]
+    using C = PairCfg<PBN>;
+    uint8_t b[kBStages][C::kBStageBytes];  // this CTA's PBN / 2 token rows of fp16 codes, [k-block][row][64 fp16]
     uint8_t w[kWStages][kWStageBytes];  // this CTA's 128 weight rows of int8 codes, [k-block pair][row][128 int8]
     uint64_t wfull[kWStages];           // own weight copy landed
     uint64_t wempty[kWStages];          // own 4 converter warps read the group's weights
     uint64_t bfull[kBStages];           // own token copy landed
     uint64_t bdone[kBStages];           // pair MMA of the group done (rank 0 commit, both CTAs)
-    uint64_t afull[kAStages];           // rank 0 only: both CTAs' converters wrote their A stages (8 warps)
-    uint64_t adone[kAStages];           // pair MMA of the k-block done (rank 0 commit, both CTAs)
+    uint64_t afull[C::kAStg];           // rank 0 only: both CTAs' converters wrote their A stages (8 warps)
+    uint64_t adone[C::kAStg];           // pair MMA of the k-block done (rank 0 commit, both CTAs)
     uint64_t accfull[2];                // pair MMA finished the chunk (rank 0 commit)
     uint64_t accempty[2];               // rank 0 only: both CTAs' epilogues drained the chunk (2 x 8 warps)
     uint64_t pub;                       // stream-K: the 8 epilogue warps stored their partial sums
@@ -677,7 +693,7 @@ __device__ __forceinline__ bool group_end(int kb, int kb1) {
     return kb == kb1 - 1 || (kb & (kGroupKB - 1)) == kGroupKB - 1;
 }
 
-template <bool kS32, bool kAsym, bool kQOut>
+template <int PBN, bool kS32, bool kAsym, bool kQOut>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     linear_pair_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_w,
                        const float *__restrict__ sw, const float *__restrict__ bfold, void *__restrict__ out, int M,
@@ -685,12 +701,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                        const float *__restrict__ s_tok, const int32_t *__restrict__ zc,
                        const int32_t *__restrict__ rowsum, const float *__restrict__ zq,
                        const float *__restrict__ rq, int qmax_out, int group_m) {
+    using C = PairCfg<PBN>;
     extern __shared__ uint8_t smem_raw[];
-    SmemPair &S = *reinterpret_cast<SmemPair *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    SmemPair<PBN> &S =
+        *reinterpret_cast<SmemPair<PBN> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = warp_id(), lane = lane_id();
     const uint32_t rank = cluster_ctarank();
     const int cluster = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
-    const int m_tiles = (M + kPairBN - 1) / kPairBN;
+    const int m_tiles = (M + C::kBN - 1) / C::kBN;
     const int n_pairs = (N + 2 * kBM - 1) / (2 * kBM);
     const int num_units = m_tiles * n_pairs;
     const int nkb = (K + kBK - 1) / kBK;
@@ -708,7 +726,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             mbar_init(smem_u32(&S.bfull[s]), 1);
             mbar_init(smem_u32(&S.bdone[s]), 1);
         }
-        for (int s = 0; s < kAStages; ++s) {
+        for (int s = 0; s < C::kAStg; ++s) {
             mbar_init(smem_u32(&S.afull[s]), 8);
             mbar_init(smem_u32(&S.adone[s]), 1);
         }
@@ -760,7 +778,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                 sch.piece(p, u, pk0, pk1);
                 int mt, np;
                 pair_tile(u, m_tiles, n_pairs, group_m, mt, np);
-                const int m0 = mt * kPairBN + (int)rank * kPairHalf;
+                const int m0 = mt * C::kBN + (int)rank * C::kHalf;
                 const int n0 = (np * 2 + (int)rank) * kBM;
                 for (int g0 = pk0; g0 < pk1; g0 = (g0 | (kGroupKB - 1)) + 1, ++gi) {
                     const int ws = gi % kWStages, bs = gi % kBStages;
@@ -772,7 +790,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     if (elect_one()) {
                         mbar_arrive_expect_tx(smem_u32(&S.wfull[ws]), kWStageBytes);
                         tma_load_3d(smem_u32(S.w[ws]), &tm_w, smem_u32(&S.wfull[ws]), 0, n0, g0 >> 1);
-                        mbar_arrive_expect_tx(smem_u32(&S.bfull[bs]), kBStageBytes);
+                        mbar_arrive_expect_tx(smem_u32(&S.bfull[bs]), C::kBStageBytes);
                         tma_load_3d(smem_u32(S.b[bs]), &tm_q, smem_u32(&S.bfull[bs]), 0, m0, g0);
                     }
                     __syncwarp();
@@ -788,8 +806,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             __syncwarp();
         } else if (warp == kWarpMma && rank == 0) {
             // the whole warp runs the loop and waits; one elected lane issues the MMAs and commits
-            const uint32_t idesc = idesc_f16_f32(2 * kBM, kPairBN);
-            const uint32_t a_tm = tmem + kPairACol;
+            const uint32_t idesc = idesc_f16_f32(2 * kBM, C::kBN);
+            const uint32_t a_tm = tmem + C::kACol;
             uint32_t it = 0, g = 0, gi = 0, b_base = 0;
             int g0 = 0, bs = 0;
             bool ok = true;
@@ -801,7 +819,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     if (!(ok = mbar_wait_warp(smem_u32(&S.accempty[buf]), ((g >> 1) & 1) ^ 1, abort, &g_status)))
                         break;
                     tc_fence_after();
-                    const uint32_t d = tmem + buf * kPairBN;
+                    const uint32_t d = tmem + buf * C::kBN;
                     const int kb1 = min(pk1, kb0 + kcb);
                     for (int kb = kb0; kb < kb1; ++kb, ++it) {
                         if (group_start(kb, pk0)) {
@@ -810,12 +828,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                             b_base = smem_u32(S.b[bs]);
                             ++gi;
                         }
-                        const int sa = it % kAStages;
+                        const int sa = it % C::kAStg;
                         // both CTAs' converters wrote A stage sa, after their B stage landed
-                        if (!(ok = mbar_wait_warp(smem_u32(&S.afull[sa]), (it / kAStages) & 1, abort, &g_status)))
+                        if (!(ok = mbar_wait_warp(smem_u32(&S.afull[sa]), (it / C::kAStg) & 1, abort, &g_status)))
                             break;
                         tc_fence_after();
-                        const uint64_t bdesc = smem_desc_sw128(b_base + (uint32_t)(kb - g0) * kBTileBytes);
+                        const uint64_t bdesc = smem_desc_sw128(b_base + (uint32_t)(kb - g0) * C::kBTileBytes);
                         if (elect_one()) {
 #pragma unroll
                             for (int kk = 0; kk < kBK / 16; ++kk)
@@ -843,7 +861,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         const uint32_t set = warp >= kWarpConv1 ? 1u : 0u;
         const int row = (warp & 3) * 32 + lane;  // weight row = TMEM lane
         const uint32_t afull0 = mapa_shared(smem_u32(&S.afull[0]), 0);
-        const uint32_t a_tm = tmem + ((uint32_t)((warp & 3) * 32) << 16) + kPairACol;
+        const uint32_t a_tm = tmem + ((uint32_t)((warp & 3) * 32) << 16) + C::kACol;
         uint32_t it = 0, gi = 0;
         int wst = 0, w0 = 0;
         bool gwait = false, ok = true;
@@ -873,7 +891,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                         break;
                     gwait = true;
                 }
-                const int sa = it % kAStages;
+                const int sa = it % C::kAStg;
                 // this row's 64 bytes of k-block kb: line (kb - w0) / 2 of 128 bytes, 16-byte chunks
                 // (kb - w0) % 2 * 4 + c, placed by the 128-byte swizzle at chunk ^ (row % 8)
                 const int j = kb - w0;
@@ -895,10 +913,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     i8x4_to_f16x4(raw[c].z, h[8 * c + 4], h[8 * c + 5]);
                     i8x4_to_f16x4(raw[c].w, h[8 * c + 6], h[8 * c + 7]);
                 }
-                // A stage sa was last read by the MMA of k-block it - kAStages
-                if (it >= (uint32_t)kAStages) {
-                    const uint32_t prev = it - kAStages;
-                    if (!(ok = mbar_wait(smem_u32(&S.adone[sa]), (prev / kAStages) & 1, abort, &g_status)))
+                // A stage sa was last read by the MMA of k-block it - C::kAStg
+                if (it >= (uint32_t)C::kAStg) {
+                    const uint32_t prev = it - C::kAStg;
+                    if (!(ok = mbar_wait(smem_u32(&S.adone[sa]), (prev / C::kAStg) & 1, abort, &g_status)))
                         break;
                     tc_fence_after();
                 }
@@ -913,7 +931,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         regs_inc<144>();
         const int e = warp - kWarpEpi0;
         const int q = warp & 3;
-        const int col0 = (e >> 2) * kPairHalf;
+        const int col0 = (e >> 2) * C::kHalf;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         const uint32_t accempty0 = mapa_shared(smem_u32(&S.accempty[0]), 0);
         uint32_t g = 0;
@@ -927,18 +945,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             sch.piece(p, u, pk0, pk1);
             int mt, np;
             pair_tile(u, m_tiles, n_pairs, group_m, mt, np);
-            const int m0 = mt * kPairBN;
+            const int m0 = mt * C::kBN;
             const int n0 = (np * 2 + (int)rank) * kBM;
-            int32_t tot[kPairHalf];
+            int32_t tot[C::kHalf];
 #pragma unroll
-            for (int j = 0; j < kPairHalf; ++j) tot[j] = 0;
+            for (int j = 0; j < C::kHalf; ++j) tot[j] = 0;
             for (int kb0 = pk0; kb0 < pk1; kb0 += kcb, ++g) {
                 const int buf = g & 1;
                 if (!(ok = mbar_wait(smem_u32(&S.accfull[buf]), (g >> 1) & 1, abort, &g_status))) break;
                 tc_fence_after();
-                const uint32_t base = tmem + lane_base + buf * kPairBN + col0;
+                const uint32_t base = tmem + lane_base + buf * C::kBN + col0;
 #pragma unroll
-                for (int p = 0; p < kPairHalf / 16; ++p) {
+                for (int p = 0; p < C::kHalf / 16; ++p) {
                     uint32_t v[16];
                     tmem_ld16(base + p * 16, v);
                     tmem_wait_ld();
@@ -953,9 +971,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             if (pk1 < nkb) {
                 // partial piece: publish the int32 sums for the pair that ends this tile
                 int32_t *slot = slots + ((size_t)cluster * 2 + rank) * pair_slot_ints();
-                if (OT_DCHECK(cluster < nclusters && col0 + kPairHalf <= 256))
+                if (OT_DCHECK(cluster < nclusters && col0 + C::kHalf <= 256))
 #pragma unroll
-                    for (int j = 0; j < kPairHalf; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
+                    for (int j = 0; j < C::kHalf; ++j) slot[(size_t)(col0 + j) * 128 + row] = tot[j];
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&S.pub));
@@ -984,7 +1002,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     if (!ok) break;
                     const int32_t *slot = slots + ((size_t)c * 2 + rank) * pair_slot_ints();
 #pragma unroll
-                    for (int j = 0; j < kPairHalf; ++j) tot[j] += __ldcg(slot + (size_t)(col0 + j) * 128 + row);
+                    for (int j = 0; j < C::kHalf; ++j) tot[j] += __ldcg(slot + (size_t)(col0 + j) * 128 + row);
                 }
                 if (!ok) break;
             }
@@ -993,7 +1011,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                 if constexpr (kS32) {
                     int32_t *o = reinterpret_cast<int32_t *>(out);
 #pragma unroll
-                    for (int j = 0; j < kPairHalf; ++j) {
+                    for (int j = 0; j < C::kHalf; ++j) {
                         const int m = m0 + col0 + j;
                         if (m < M && OT_DCHECK((int64_t)m * N + n < (int64_t)M * N)) o[(int64_t)m * N + n] = tot[j];
                     }
@@ -1004,7 +1022,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     const float zqn = kQOut ? __ldg(zq + n) : 0.f, rqn = kQOut ? __ldg(rq + n) : 0.f;
                     __half *o = reinterpret_cast<__half *>(out);
 #pragma unroll
-                    for (int j = 0; j < kPairHalf; ++j) {
+                    for (int j = 0; j < C::kHalf; ++j) {
                         const int m = m0 + col0 + j;
                         const int mc = m < M ? m : M - 1;
                         // per-token path (Eq. 3): one fp32 product s_m * sw_n
@@ -1158,10 +1176,10 @@ int pair_max_clusters() {
     cudaGetDevice(&dev);
     std::lock_guard<std::mutex> lock(mu);
     if (dev_cached == dev) return value;
-    const size_t smem = sizeof(SmemPair) + 1024;
+    const size_t smem = sizeof(SmemPair<kPairBN>) + 1024;
     int n = 0;
-    if (cudaFuncSetAttribute(linear_pair_kernel<false, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem) ==
+    if (cudaFuncSetAttribute(linear_pair_kernel<kPairBN, false, false, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
         cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 256);
@@ -1174,7 +1192,8 @@ int pair_max_clusters() {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<false, false, false>, &cfg) != cudaSuccess) n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, linear_pair_kernel<kPairBN, false, false, false>, &cfg) != cudaSuccess)
+            n = 0;
     }
     cudaGetLastError();
     if (n <= 0) n = num_sms() / 2;
@@ -1197,12 +1216,12 @@ int pair_max_clusters() {
 //    K = 36864 (OPT-66B fc2) a tile's operands alone are 24 MB: 7 token
 //    tiles per group read 3.0 GB per launch against 4.0 GB in the plain order
 //    (and ran 2 % faster).
-int pair_group_m(int64_t M, int64_t N, int64_t K, int clusters) {
+int pair_group_m(int64_t M, int64_t N, int64_t K, int clusters, int pbn) {
     constexpr double kL2Keep = 48.0 * (1 << 20);  // codes a group may keep in L2 beside the weight stream
-    const int64_t m_tiles = (M + kPairBN - 1) / kPairBN;
+    const int64_t m_tiles = (M + pbn - 1) / pbn;
     const int64_t n_pairs = (N + 2 * kBM - 1) / (2 * kBM);
     const int64_t cl = clusters > 0 ? clusters : 1;
-    const double tile_codes = (double)kPairBN * (double)K * 2.0, tile_weights = 2.0 * kBM * (double)K;
+    const double tile_codes = (double)pbn * (double)K * 2.0, tile_weights = 2.0 * kBM * (double)K;
     const double codes = tile_codes * (double)m_tiles, weights = (double)N * (double)K;
     const double rounds = std::max(1.0, (double)(m_tiles * n_pairs) / (double)cl);
     auto per_rounds = [&](int64_t g) {
@@ -1230,28 +1249,29 @@ int pair_group_m(int64_t M, int64_t N, int64_t K, int clusters) {
     return best < 0.8 * plain ? (int)best_g : (int)m_tiles;
 }
 
-template <bool kS32, bool kAsym, bool kQOut>
+template <int PBN, bool kS32, bool kAsym, bool kQOut>
 cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
+    using C = PairCfg<PBN>;
     // codes as {64 fp16, M rows, K / 64 k-blocks}: a box of 96 rows x 4 k-blocks;
     // weights as {128 int8, N rows, K / 128 k-block pairs}: a box of 128 rows x 2 pairs.
     // Each inner span is a whole slice of the row (K % 128 == 0), so no copy
     // reaches past a row; rows past M or N and k-blocks past K are zero-filled.
     CUtensorMap tm_q, tm_w;
     if (!make_tmap_3d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.q, kBK, (uint64_t)a.M, (uint64_t)a.K / kBK,
-                      (uint64_t)a.K * 2, kBK * 2, kBK, kPairHalf, kGroupKB, CU_TENSOR_MAP_SWIZZLE_128B) ||
+                      (uint64_t)a.K * 2, kBK * 2, kBK, C::kHalf, kGroupKB, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_tmap_3d(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.qw, 128, (uint64_t)a.N, (uint64_t)a.K / 128,
                       (uint64_t)a.K, 128, 128, kBM, kGroupKB / 2, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
-    const size_t smem = sizeof(SmemPair) + 1024;
+    const size_t smem = sizeof(SmemPair<PBN>) + 1024;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(linear_pair_kernel<kS32, kAsym, kQOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)smem);
+        attr_err = cudaFuncSetAttribute(linear_pair_kernel<PBN, kS32, kAsym, kQOut>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int max_clusters = pair_max_clusters();
-    const int64_t units = ((a.M + kPairBN - 1) / kPairBN) * ((a.N + 2 * kBM - 1) / (2 * kBM));
+    const int64_t units = ((a.M + C::kBN - 1) / C::kBN) * ((a.N + 2 * kBM - 1) / (2 * kBM));
     const int64_t nkb = (a.K + kBK - 1) / kBK;
     // Stream-K shortens the busiest pair's work from ceil(units / pairs) whole
     // tiles to an equal share of k-blocks, at the cost of a partial-sum
@@ -1264,18 +1284,21 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
                          whole - shared >= kStreamKMinSaving && units * nkb < ((int64_t)1 << 30);
     const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
-    const int group_m = pair_group_m(a.M, a.N, a.K, clusters);
-    return launch_kernel(linear_pair_kernel<kS32, kAsym, kQOut>, dim3(2 * clusters), dim3(kPairThreads), smem, st, a.pdl,
-                         tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu, ws,
-                         a.s_tok, a.zc, a.rowsum, a.zq, a.rq, a.qmax_out, group_m);
+    const int group_m = pair_group_m(a.M, a.N, a.K, clusters, C::kBN);
+    return launch_kernel(linear_pair_kernel<PBN, kS32, kAsym, kQOut>, dim3(2 * clusters), dim3(kPairThreads), smem, st,
+                         a.pdl, tm_q, tm_w, a.sw, a.bfold, a.out, (int)a.M, (int)a.N, (int)a.K, (int)a.ldy, kcb, a.relu,
+                         ws, a.s_tok, a.zc, a.rowsum, a.zq, a.rq, a.qmax_out, group_m);
 }
 
 // M <= 16 goes to the decode kernel (gemv.cu) before this dispatch.
 template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
+    // Measured on GB300 (OPT-13B QKV / fc2): the 128-token pair tile is 2-3 % faster than linear_kernel at
+    // 65-128 tokens (QKV 28.2 vs 28.9 us, fc2 36.3 vs 37.2 at 128) and 6-12 % slower at 17-64
+    if (a.K % 128 == 0 && a.M > 128) return run_linear_pair<kPairBN, kS32, kAsym, kQOut>(a, kcb, st);
+    if (a.K % 128 == 0 && a.M > 64) return run_linear_pair<128, kS32, kAsym, kQOut>(a, kcb, st);
     if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
-    if (a.M <= 128 || a.K % 128 != 0) return run_linear<128, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
-    return run_linear_pair<kS32, kAsym, kQOut>(a, kcb, st);
+    return run_linear<128, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
 }
 
 // int8 codes (any M > 16) and fp16 activations quantized in the kernel
