@@ -644,13 +644,16 @@ constexpr int kGroupKB = 4;                       // k-blocks per TMA copy
 constexpr int kPairThreads = 640;
 constexpr int kWarpConv1 = 16;
 constexpr int kWStages = 2;                       // weight stages: 2 x 128 rows x 128 int8, 128-byte swizzle (32 KB)
-constexpr int kBStages = 3;                       // token stages: 4 x PBN / 2 rows x 64 fp16, 128-byte swizzle
 constexpr uint32_t kWStageBytes = 2 * kBM * 128;
 // Tile width of a CTA pair: PBN tokens (the MMA's N), PBN / 2 token rows per
 // CTA; TMEM holds two PBN-column chunk accumulators and (512 - 2 PBN) / 32
-// A stages.  192 for prefill (M > 128): 2048 tokens in 11 tiles with 3 %
-// padding; 128 for 17-128 tokens: eight A stages instead of four, so the
-// cross-CTA hand-off round trip no longer bounds the k-loop.
+// A stages.  Prefill (M > 128) takes 192 or 224 (prefill_tile below): the
+// k-loop costs about the same per k-block for any width (measured on GB300:
+// ~12 % more at 224, whose MMA is longer and which has two A stages), so the
+// fewer token tiles the better -- 4096 tokens in 19 tiles of 224 instead of
+// 22 of 192 (OPT-66B fc1 1660 vs 1718 us), 2048 in 11 of 192 rather than 10
+// of 224 (9 % padding).  65-128 tokens take 128 (eight A stages).
+constexpr int kBStages = 3;                       // token stages: 4 x PBN / 2 rows x 64 fp16, 128-byte swizzle
 template <int PBN>
 struct PairCfg {
     static constexpr int kBN = PBN;                   // tokens per pair tile (MMA N)
@@ -659,21 +662,29 @@ struct PairCfg {
     static constexpr int kAStg = (512 - kACol) / 32;  // 32-column fp16 A stages (128 rows x 64 k)
     static constexpr uint32_t kBTileBytes = kHalf * 128;
     static constexpr uint32_t kBStageBytes = kGroupKB * kBTileBytes;
+    static constexpr int kBStg = PBN > 192 ? 2 : kBStages;  // token stages (224: two, for shared memory)
     static_assert(kAStg >= 2, "A stage of k-block i is freed by the commit of k-block i - kAStg");
-    static_assert(kBN % 32 == 0 && kHalf % 32 == 0, "the epilogue drains 32 columns at a time");
+    static_assert(kBN % 16 == 0 && kHalf % 16 == 0, "the epilogue drains 16 columns at a time");
     static_assert(kBTileBytes % 1024 == 0, "each k-block of B is a whole number of 1024-byte swizzle atoms");
 };
-constexpr int kPairBN = 192;  // the prefill tile
+constexpr int kPairBN = 192;  // the prefill tile (also the one pair_max_clusters measures)
+
+// Prefill tile width for M tokens: 224 when its tile count, weighted by its
+// ~12 % higher cost per k-block, is below that of 192.
+inline int prefill_tile(int64_t M) {
+    const int64_t t192 = (M + 191) / 192, t224 = (M + 223) / 224;
+    return 28 * t224 < 25 * t192 ? 224 : 192;
+}
 
 template <int PBN>
 struct alignas(1024) SmemPair {
     using C = PairCfg<PBN>;
-    uint8_t b[kBStages][C::kBStageBytes];  // this CTA's PBN / 2 token rows of fp16 codes, [k-block][row][64 fp16]
+    uint8_t b[C::kBStg][C::kBStageBytes];  // this CTA's PBN / 2 token rows of fp16 codes, [k-block][row][64 fp16]
     uint8_t w[kWStages][kWStageBytes];  // this CTA's 128 weight rows of int8 codes, [k-block pair][row][128 int8]
     uint64_t wfull[kWStages];           // own weight copy landed
     uint64_t wempty[kWStages];          // own 4 converter warps read the group's weights
-    uint64_t bfull[kBStages];           // own token copy landed
-    uint64_t bdone[kBStages];           // pair MMA of the group done (rank 0 commit, both CTAs)
+    uint64_t bfull[C::kBStg];           // own token copy landed
+    uint64_t bdone[C::kBStg];           // pair MMA of the group done (rank 0 commit, both CTAs)
     uint64_t afull[C::kAStg];           // rank 0 only: both CTAs' converters wrote their A stages (8 warps)
     uint64_t adone[C::kAStg];           // pair MMA of the k-block done (rank 0 commit, both CTAs)
     uint64_t accfull[2];                // pair MMA finished the chunk (rank 0 commit)
@@ -722,7 +733,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             mbar_init(smem_u32(&S.wfull[s]), 1);
             mbar_init(smem_u32(&S.wempty[s]), 8);
         }
-        for (int s = 0; s < kBStages; ++s) {
+        for (int s = 0; s < C::kBStg; ++s) {
             mbar_init(smem_u32(&S.bfull[s]), 1);
             mbar_init(smem_u32(&S.bdone[s]), 1);
         }
@@ -781,11 +792,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                 const int m0 = mt * C::kBN + (int)rank * C::kHalf;
                 const int n0 = (np * 2 + (int)rank) * kBM;
                 for (int g0 = pk0; g0 < pk1; g0 = (g0 | (kGroupKB - 1)) + 1, ++gi) {
-                    const int ws = gi % kWStages, bs = gi % kBStages;
+                    const int ws = gi % kWStages, bs = gi % C::kBStg;
                     // stages last used by group gi - stages: the converters / the pair MMA are done with them
                     if (!(ok = mbar_wait_warp(smem_u32(&S.wempty[ws]), ((gi / kWStages) & 1) ^ 1, abort, &g_status)))
                         break;
-                    if (!(ok = mbar_wait_warp(smem_u32(&S.bdone[bs]), ((gi / kBStages) & 1) ^ 1, abort, &g_status)))
+                    if (!(ok = mbar_wait_warp(smem_u32(&S.bdone[bs]), ((gi / C::kBStg) & 1) ^ 1, abort, &g_status)))
                         break;
                     if (elect_one()) {
                         mbar_arrive_expect_tx(smem_u32(&S.wfull[ws]), kWStageBytes);
@@ -800,8 +811,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             if (lane == 0) {
                 for (uint32_t j = gi > (uint32_t)kWStages ? gi - kWStages : 0; j < gi; ++j)
                     wait_teardown(smem_u32(&S.wfull[j % kWStages]), (j / kWStages) & 1);
-                for (uint32_t j = gi > (uint32_t)kBStages ? gi - kBStages : 0; j < gi; ++j)
-                    wait_teardown(smem_u32(&S.bfull[j % kBStages]), (j / kBStages) & 1);
+                for (uint32_t j = gi > (uint32_t)C::kBStg ? gi - C::kBStg : 0; j < gi; ++j)
+                    wait_teardown(smem_u32(&S.bfull[j % C::kBStg]), (j / C::kBStg) & 1);
             }
             __syncwarp();
         } else if (warp == kWarpMma && rank == 0) {
@@ -823,7 +834,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     const int kb1 = min(pk1, kb0 + kcb);
                     for (int kb = kb0; kb < kb1; ++kb, ++it) {
                         if (group_start(kb, pk0)) {
-                            bs = gi % kBStages;
+                            bs = gi % C::kBStg;
                             g0 = kb;
                             b_base = smem_u32(S.b[bs]);
                             ++gi;
@@ -887,7 +898,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                     const uint32_t gp = gi - 1;
                     if (!(ok = mbar_wait(smem_u32(&S.wfull[wst]), (gp / kWStages) & 1, abort, &g_status))) break;
                     // the pair MMA reads this CTA's half of B: it must have landed before afull
-                    if (!(ok = mbar_wait(smem_u32(&S.bfull[gp % kBStages]), (gp / kBStages) & 1, abort, &g_status)))
+                    if (!(ok = mbar_wait(smem_u32(&S.bfull[gp % C::kBStg]), (gp / C::kBStg) & 1, abort, &g_status)))
                         break;
                     gwait = true;
                 }
@@ -1295,7 +1306,9 @@ template <bool kS32, bool kAsym, bool kQOut>
 cudaError_t dispatch_bn(const LinearArgs &a, int kcb, cudaStream_t st) {
     // Measured on GB300 (OPT-13B QKV / fc2): the 128-token pair tile is 2-3 % faster than linear_kernel at
     // 65-128 tokens (QKV 28.2 vs 28.9 us, fc2 36.3 vs 37.2 at 128) and 6-12 % slower at 17-64
-    if (a.K % 128 == 0 && a.M > 128) return run_linear_pair<kPairBN, kS32, kAsym, kQOut>(a, kcb, st);
+    if (a.K % 128 == 0 && a.M > 128)
+        return prefill_tile(a.M) == 224 ? run_linear_pair<224, kS32, kAsym, kQOut>(a, kcb, st)
+                                        : run_linear_pair<kPairBN, kS32, kAsym, kQOut>(a, kcb, st);
     if (a.K % 128 == 0 && a.M > 64) return run_linear_pair<128, kS32, kAsym, kQOut>(a, kcb, st);
     if (a.M <= 64) return run_linear<64, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
     return run_linear<128, kS32, kAsym, kQOut, kTokF16>(a, kcb, st);
