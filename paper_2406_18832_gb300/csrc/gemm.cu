@@ -1081,7 +1081,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-constexpr int64_t kStreamKMinSaving = 32;  // k-blocks per pair
+constexpr int64_t kStreamKMinSaving = 32;  // k-blocks per worker
+
+// Whether stream-K pays for `units` tiles of `nkb` k-blocks over `workers`:
+// when it shortens the busiest worker's share by at least kStreamKMinSaving
+// k-blocks, or, when there are fewer tiles than workers (some would idle for
+// the whole launch), by at least 1 / idle_div of a tile (idle_div 0: never).
+// Measured on GB300 at 32-192 tokens (OPT-6.7B QKV / fc1, OPT-13B QKV, whose
+// tiles are 63-80 % of the workers): the CTA kernel gains once the share is a
+// fifth shorter (37 %: 15 % faster, 21 %: 5 %; 16 %: 1.5 % slower), the
+// 128-token pair tile once it is a third shorter (37 %: 6.5 % faster; 21 % and
+// 16 %: 2 and 9 % slower), the 192-token pair tile at none of these.
+inline bool streamk_pays(int64_t units, int64_t nkb, int64_t workers, int64_t idle_div) {
+    const int64_t whole = (units + workers - 1) / workers * nkb;
+    const int64_t shared = (units * nkb + workers - 1) / workers;
+    const int64_t saving = whole - shared;
+    return saving >= kStreamKMinSaving || (idle_div > 0 && units < workers && idle_div * saving >= whole);
+}
 
 size_t pair_workspace_bytes(int clusters) {
     return (size_t)clusters * 2 * pair_slot_ints() * sizeof(int32_t) + (size_t)clusters * 2 * sizeof(uint64_t) +
@@ -1164,14 +1180,12 @@ cudaError_t run_linear(const LinearArgs &a, int kcb, cudaStream_t st) {
     const int64_t nkb = (a.K + kBK - 1) / kBK;
     // Stream-K over CTAs, in the prefill kernel's workspace layout (a slot and
     // a flag per CTA; one CTA per SM, at most 2 x pair_max_clusters of them),
-    // when it shortens the busiest CTA's work by at least kStreamKMinSaving
-    // k-blocks (e.g. OPT-13B fc2 at 128 tokens: 40 tiles of 320 k-blocks).
+    // when streamk_pays (e.g. OPT-13B fc2 at 64 tokens: 40 tiles of 320
+    // k-blocks; OPT-6.7B QKV: 96 tiles of 64 k-blocks on 152 CTAs).
     const int pairs = pair_max_clusters();
     const int workers = num_sms() < 2 * pairs ? num_sms() : 2 * pairs;
-    const int64_t whole = (tiles + workers - 1) / workers * nkb;
-    const int64_t shared = (tiles * nkb + workers - 1) / workers;
     const bool streamk = a.workspace != nullptr && a.workspace_bytes >= pair_workspace_bytes(pairs) &&
-                         whole - shared >= kStreamKMinSaving && tiles * nkb < ((int64_t)1 << 30);
+                         streamk_pays(tiles, nkb, workers, 5) && tiles * nkb < ((int64_t)1 << 30);
     const int grid = streamk ? workers : (int)(tiles < num_sms() ? tiles : num_sms());
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
     return launch_kernel(linear_kernel<BN, kS32, kAsym, kQOut, kTok>, dim3(grid), dim3(lin_threads<kTok>()), smem,
@@ -1288,11 +1302,10 @@ cudaError_t run_linear_pair(const LinearArgs &a, int kcb, cudaStream_t st) {
     // tiles to an equal share of k-blocks, at the cost of a partial-sum
     // exchange per split tile.  Measured on GB300 it pays off once it saves
     // about 32 k-blocks per pair (OPT-6.7B QKV and fc2 at 2048 tokens: 7-11 %
-    // faster; out and fc1, which save ~20, are 1-2 % slower).
-    const int64_t whole = (units + max_clusters - 1) / max_clusters * nkb;
-    const int64_t shared = (units * nkb + max_clusters - 1) / max_clusters;
+    // faster; out and fc1, which save ~20, are 1-2 % slower); see streamk_pays.
     const bool streamk = a.workspace != nullptr && a.workspace_bytes >= pair_workspace_bytes(max_clusters) &&
-                         whole - shared >= kStreamKMinSaving && units * nkb < ((int64_t)1 << 30);
+                         streamk_pays(units, nkb, max_clusters, PBN == 128 ? 3 : 0) &&
+                         units * nkb < ((int64_t)1 << 30);
     const int clusters = streamk ? max_clusters : (int)(units < max_clusters ? units : max_clusters);
     int32_t *ws = streamk ? reinterpret_cast<int32_t *>(a.workspace) : nullptr;
     const int group_m = pair_group_m(a.M, a.N, a.K, clusters, C::kBN);

@@ -25,7 +25,9 @@ def _codes(shape, qmax, seed):
 
 
 @pytest.mark.parametrize("M,N,K", [(2048, 12288, 4096), (2048, 4096, 4096), (2048, 4096, 16384),
-                                   (256, 512, 4096), (300, 1000, 2112), (4096, 256, 1024), (129, 256, 64)])
+                                   (256, 512, 4096), (300, 1000, 2112), (4096, 256, 1024), (129, 256, 64),
+                                   # fewer tiles than CTAs or pairs, split when a fifth / a third shorter
+                                   (32, 12288, 4096), (64, 15360, 5120), (100, 12288, 4096)])
 def test_streamk_equals_whole_tiles(M, N, K):
     from paper_2406_18832_gb300 import binding as B
     dev = "cuda"
