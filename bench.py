@@ -442,7 +442,7 @@ def run_ours(args):
         "gpu_launches": args.steps * 2 * len(layer_shapes),
         "e2e": {"value": round(ops_step / (e2e_ms * 1e-3) / 1e12 * world, 2), "unit": "TOPS",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
-                "copies": "pinned host buffers; host->device, layers and device->host on three streams"},
+                "copies": "pinned host buffers; host->device, layers and device->host on three streams, buffers alternating between two sets from step to step"},
         "clocks": clocks,
         "quantize": {"gbs_algorithmic": round(q_alg / (quant_time * 1e-3) / 1e9, 1),
                      "frac_algorithmic": round(q_alg / (quant_time * 1e-3) / 1e9 / peaks["hbm"], 4),
@@ -484,43 +484,51 @@ def run_ours(args):
 
 def _e2e(layers, xs, qbufs, ybufs, steps):
     """ms per step through the public API (QuantizedLinear.forward) with the
-    inputs copied in from pinned host memory and the outputs copied back: the
-    copies run on their own streams, so a layer's input copy overlaps the
-    previous layer and its output copy the next."""
+    inputs copied in from pinned host memory and the outputs copied back, as
+    a pipelined server runs it: the copies go on their own streams, and the
+    device inputs, device outputs and host outputs alternate between two sets
+    from step to step, so a layer's input copy overlaps the layers before it,
+    its output copy the layers after it, and no layer waits for the previous
+    step's copy of the same buffer.  Every step's copies are inside the timed
+    region."""
     import torch
+    nb = 2
     hx = [x.cpu().pin_memory() for x in xs]
-    hy = [torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in ybufs]
-    dx = [torch.empty_like(x) for x in xs]
+    hy = [[torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in ybufs] for _ in range(nb)]
+    dx = [[torch.empty_like(x) for x in xs] for _ in range(nb)]
+    dy = [ybufs] + [[torch.empty_like(y) for y in ybufs] for _ in range(nb - 1)]
     s_c = torch.cuda.current_stream()
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
-    ev_in = [torch.cuda.Event() for _ in layers]
-    ev_done = [torch.cuda.Event() for _ in layers]
-    ev_out = [torch.cuda.Event() for _ in layers]
+    ev = [[[torch.cuda.Event() for _ in layers] for _ in range(nb)] for _ in range(3)]
+    ev_in, ev_done, ev_out = ev
 
-    def e2e_step():
+    def e2e_step(k):
+        b = k % nb
         for i, (ql, _, _) in enumerate(layers):
             with torch.cuda.stream(s_in):
-                s_in.wait_event(ev_done[i])          # the previous step's layer i has read dx[i]
-                dx[i].copy_(hx[i], non_blocking=True)
-                ev_in[i].record(s_in)
-            s_c.wait_event(ev_in[i])
-            s_c.wait_event(ev_out[i])                # the previous step's ybufs[i] is copied out
-            ql.forward(dx[i], qbufs[i], ybufs[i])
-            ev_done[i].record(s_c)
+                s_in.wait_event(ev_done[b][i])       # the layer two steps back has read dx[b][i]
+                dx[b][i].copy_(hx[i], non_blocking=True)
+                ev_in[b][i].record(s_in)
+            s_c.wait_event(ev_in[b][i])
+            s_c.wait_event(ev_out[b][i])             # dy[b][i] of two steps back is copied out
+            ql.forward(dx[b][i], qbufs[i], dy[b][i])
+            ev_done[b][i].record(s_c)
             with torch.cuda.stream(s_out):
-                s_out.wait_event(ev_done[i])
-                hy[i].copy_(ybufs[i], non_blocking=True)
-                ev_out[i].record(s_out)
-    for _ in range(2):
-        e2e_step()
+                s_out.wait_event(ev_done[b][i])
+                hy[b][i].copy_(dy[b][i], non_blocking=True)
+                ev_out[b][i].record(s_out)
+    for k in range(2 * nb):
+        e2e_step(k)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(steps):
-        e2e_step()
+    e0.record(s_c)
+    s_in.wait_event(e0)
+    s_out.wait_event(e0)
+    for k in range(steps):
+        e2e_step(k)
     s_c.wait_stream(s_in)
     s_c.wait_stream(s_out)
-    e1.record()
+    e1.record(s_c)
     torch.cuda.synchronize()
     h2d = sum(x.numel() * 2 for x in xs)
     d2h = sum(y.numel() * 2 for y in ybufs)
